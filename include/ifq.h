@@ -1,0 +1,243 @@
+/*
+ * ifq.h -- C ABI of the GB300 library for the quantized substructure of
+ * IFQ-Net (Gao et al., "IFQ-Net: Integrated Fixed-point Quantization Networks
+ * for Embedded Vision", arXiv:1911.08076).
+ *
+ * The library computes, on one GPU, the quantized convolution of Eq. (1) with
+ * +-1 filters W_b and unsigned 2-bit input codes X_q, and applies the
+ * integrated fixed-point conversion of Sec. 3.2 as its epilogue: the integer
+ * accumulator W_b (x) X_q is compared with per-channel integer thresholds
+ * (Eq. (7) after the floor), which emits the next layer's 2-bit codes.
+ *
+ * Conventions shared by every call:
+ *   - Return value: an ifq_status.  Argument, shape, alignment and range
+ *     errors are returned synchronously, before anything is launched.
+ *   - Pointers marked (device) are CUDA device pointers; (host) are host
+ *     pointers.  The caller owns every buffer; nothing is retained after the
+ *     call returns, and the library allocates no device memory in any call
+ *     named here except ifq_graph_create (which owns the captured graph).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Device work is enqueued on it and the call returns without
+ *     waiting, except where stated.
+ *   - Device-side failures (a bounded wait that ran out, a failed bounds
+ *     check) never trap: they set a device status word that
+ *     ifq_device_status reads.
+ *
+ * Data formats:
+ *   - Codes: NHWC, 2 bits per code, four codes per byte along C; channel c of
+ *     a pixel is bits 2*(c%4)..2*(c%4)+1 of byte c/4 of that pixel.  C must be
+ *     a multiple of 4, so a pixel is C/4 bytes.  Buffers are at least 16-byte
+ *     aligned (cudaMalloc / torch allocations are).
+ *   - Filter signs: one row per output channel over K = kh*kw*cin in
+ *     (dy, dx, c) order (c fastest); bit k%32 of 32-bit word k/32 is 1 for +1
+ *     and 0 for -1; a row is ceil(K/32) words.
+ *   - Thresholds: int32 [cout][2^k - 1], ascending (not necessarily strictly),
+ *     and int8 sign [cout] in {+1, -1}; the code of accumulator A in channel n
+ *     is the number of i with sign[n]*A > T[n][i].
+ *   - Accumulators: int32 NHWC [n][ho][wo][cout].
+ *   - Convolution geometry: cross-correlation, symmetric zero padding `pad`
+ *     (a padded cell is code 0), ho = (h + 2*pad - kh)/stride + 1.
+ *   - Pooling geometry: k x k windows starting at (oy*stride, ox*stride),
+ *     `pad` extra empty cells at the bottom and right that are skipped,
+ *     ho = (h + pad - k)/stride + 1.
+ */
+#ifndef IFQ_H
+#define IFQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  IFQ_OK = 0,
+  IFQ_EINVAL = 1,        /* null pointer or invalid parameter value */
+  IFQ_ESHAPE = 2,        /* inconsistent or unsupported shape */
+  IFQ_EALIGN = 3,        /* pointer not aligned as required */
+  IFQ_ERANGE = 4,        /* a size exceeds what the library supports */
+  IFQ_ECUDA = 5,         /* a CUDA runtime call failed */
+  IFQ_ETIMEOUT = 6,      /* (device status) a bounded wait in a kernel ran out */
+  IFQ_EUNSUPPORTED = 7,  /* valid request that this build does not implement */
+  IFQ_EWORKSPACE = 8     /* workspace missing or too small */
+} ifq_status;
+
+/* Output selection of a convolution. */
+enum { IFQ_OUT_CODES = 1, IFQ_OUT_ACC = 2, IFQ_OUT_BOTH = 3 };
+
+/* Kernel path of a convolution (ifq_conv_desc.path). */
+enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2 };
+
+/* Layer kinds of ifq_forward. */
+enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2 };
+
+/* Text for a status code (static storage; never NULL). */
+const char* ifq_status_str(int status);
+
+/* Library ABI version: 100*major + minor. */
+int ifq_version(void);
+
+/*
+ * ifq_fold_layer -- integrated fixed-point conversion of one quantized
+ * substructure (Sec. 3.2, Eq. (6)-(7), floor of the composed thresholds).
+ * Host only, pure, thread-safe; nothing is launched.
+ *
+ * For output channel n the float substructure is
+ *   y = alpha[n]*delta_in*A + bias[n]                        (Eq. (1))
+ *   z = gamma[n]*(y - mean[n])/sqrt(var[n] + eps) + beta[n]   (Eq. (2), affine BN)
+ *   code = #{ i in 1..L : z > q_base*i + q_offset }           (Eq. (3), L = 2^kbits - 1)
+ * and the fold returns T[n][i-1] and sign[n] such that
+ *   code = #{ i : sign[n]*A > T[n][i-1] }
+ * for every integer A with |A| <= L*K:
+ *   tau_i = ((thr_i - beta)*sqrt(var + eps)/gamma + mean - bias)/(alpha*delta_in)
+ *   gamma > 0: sign = +1, T = floor(tau_i);  gamma < 0: sign = -1, T = floor(-tau_i)
+ *   gamma = 0: sign = +1, T = -L*K-1 if beta > thr_i else L*K
+ * T is clamped to [-L*K-1, L*K].  The arithmetic is IEEE double in the order
+ * written above.
+ *
+ * Arguments (host): alpha, gamma, beta, mean, var: [cout] float; bias: [cout]
+ * or NULL (zero); thr_out: [cout][L] int32; sign_out: [cout] int8.
+ * Requires cout >= 1, K >= 1, 1 <= kbits <= 8, delta_in > 0, q_base > 0,
+ * alpha[n] > 0, var[n] + eps > 0, all values finite (else IFQ_EINVAL).
+ */
+int ifq_fold_layer(int cout, int K, int kbits, const float* alpha, float delta_in, const float* bias,
+                   const float* gamma, const float* beta, const float* mean, const float* var, float eps,
+                   float q_base, float q_offset, int32_t* thr_out, int8_t* sign_out);
+
+/* Packed size in bytes of an n x h x w x c map of kbits-bit codes, 1 <= kbits <= 32 (host, pure). */
+int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
+
+/*
+ * Convolution descriptor.  Input codes NHWC [n][h][w][cin] (cin % 4 == 0),
+ * filters [cout][kh][kw][cin], output [n][ho][wo][cout].  out_mode is one of
+ * IFQ_OUT_*; codes output needs cout % 4 == 0.  path selects a kernel path
+ * (IFQ_PATH_AUTO lets the library choose).  Limits: all sizes >= 1,
+ * K = kh*kw*cin <= 65536, cout <= 65536, n*ho*wo < 2^31.
+ */
+typedef struct {
+  int n, h, w, cin;
+  int cout;
+  int kh, kw, stride, pad;
+  int out_mode;
+  int path;
+} ifq_conv_desc;
+
+/* Output spatial size of a conv descriptor (host, pure). */
+int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo);
+
+/*
+ * Size of the prepared-filter buffer that ifq_pack_weights fills for `d`
+ * (host, pure).  The prepared layout is private to the library.
+ */
+int ifq_weights_prep_bytes(const ifq_conv_desc* d, size_t* bytes);
+
+/*
+ * ifq_pack_weights -- expand the filter sign bits of Eq. (1)'s W_b into the
+ * library's prepared form (tensor-core operand rows and a sign-bit copy).
+ * w_bits (device): [cout][ceil(K/32)] uint32 sign words as in the header;
+ * w_prep (device): ifq_weights_prep_bytes bytes, 16-byte aligned.
+ * Run once per layer; the result is reused by every ifq_conv2bit call.
+ */
+int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_prep, void* stream);
+
+/* Device workspace that ifq_conv2bit needs for `d` (host, pure); may be 0. */
+int ifq_conv_workspace_bytes(const ifq_conv_desc* d, size_t* bytes);
+
+/*
+ * ifq_conv2bit -- one quantized substructure (Eq. (1) integer core followed
+ * by the thresholds of Eq. (7)).  For every output pixel and channel n:
+ *   A = sum over (dy, dx, c) of w[n][dy][dx][c] * x[b][oy*s+dy-pad][ox*s+dx-pad][c]
+ *   y_codes = #{ i : sign[n]*A > thr[n][i] }  (2-bit codes, packed)
+ *   y_acc   = A                                (int32), per out_mode
+ * x (device): packed codes; w_prep (device): from ifq_pack_weights;
+ * thr (device): int32 [cout][3]; sign (device): int8 [cout];
+ * y_codes (device, out_mode & CODES): packed [n][ho][wo][cout/4] bytes;
+ * y_acc (device, out_mode & ACC): int32 [n][ho][wo][cout];
+ * ws (device): ifq_conv_workspace_bytes bytes (may be NULL if that is 0).
+ * The results are exact integers; x must not alias the outputs.
+ */
+int ifq_conv2bit(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr,
+                 const int8_t* sign, void* y_codes, int32_t* y_acc, void* ws, size_t ws_bytes, void* stream);
+
+/* Pooling descriptor (geometry in the header comment); c % 4 == 0. */
+typedef struct {
+  int n, h, w, c;
+  int k, stride, pad;
+} ifq_pool_desc;
+
+int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo);
+
+/*
+ * ifq_maxpool2bit -- max pooling placed between conv and BN (Sec. 2.1),
+ * computed on the codes.  With sign (device, int8 [c]) given, channel c takes
+ * the max of its codes where sign = +1 and the min where sign = -1; since the
+ * composed conv/BN/quantizer map is monotone in the accumulator (increasing
+ * for +1, decreasing for -1), this equals quantizing the max of Y^conv.  With
+ * sign NULL it is the plain max of the codes (pooling after the quantizer).
+ * x, y (device): packed codes.
+ */
+int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, void* stream);
+
+/*
+ * One layer of a stack for ifq_forward.  src is the index of the layer whose
+ * output codes are this layer's input (-1: the stack input x).  For a conv,
+ * `conv`, w_prep, thr and sign describe it and y_codes / y_acc receive its
+ * outputs per conv.out_mode; for a pool, `pool` describes it, sign is the
+ * pooled layer's channel signs (or NULL for a plain max) and y_codes receives
+ * the pooled codes.  All pointers are device pointers owned by the caller.
+ */
+typedef struct {
+  int kind;
+  int src;
+  ifq_conv_desc conv;
+  ifq_pool_desc pool;
+  const void* w_prep;
+  const int32_t* thr;
+  const int8_t* sign;
+  void* y_codes;
+  int32_t* y_acc;
+} ifq_layer;
+
+/* Workspace that ifq_forward needs for `layers` (host, pure); may be 0. */
+int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* bytes);
+
+/*
+ * ifq_forward -- run a layer stack in order on one stream (Sec. 3.1: a
+ * quantized network is a chain of substructures; the codes of one are the
+ * input of the next, and the output scale of one is the input step of the
+ * next).  Shapes are checked along the chain before any launch.
+ * x (device): the stack input codes; ws (device): workspace.
+ */
+int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * CUDA-graph form of ifq_forward: ifq_graph_create captures the launches of
+ * ifq_forward(layers, nlayers, x, ws, ws_bytes) on `stream` into a graph that
+ * ifq_graph_launch replays on any stream with the same buffers.  The graph is
+ * owned by the returned handle; ifq_graph_destroy frees it.
+ */
+typedef struct ifq_graph ifq_graph;
+int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream,
+                     ifq_graph** out);
+int ifq_graph_launch(ifq_graph* g, void* stream);
+int ifq_graph_destroy(ifq_graph* g);
+
+/* Codes <-> packed format helpers (device buffers; n % 4 == 0 codes). */
+int ifq_pack_codes(const uint8_t* codes, void* packed, size_t n, void* stream);
+int ifq_unpack_codes(const void* packed, uint8_t* codes, size_t n, void* stream);
+/* +-1 int8 filters [rows][K] (device) -> sign words [rows][ceil(K/32)] (device). */
+int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* stream);
+
+/*
+ * ifq_device_status -- synchronize `stream`, then read and clear the device
+ * status word of the current device: IFQ_OK, or the first device-side error
+ * recorded (IFQ_ETIMEOUT, IFQ_ERANGE) since the last read.
+ */
+int ifq_device_status(void* stream, int* status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* IFQ_H */

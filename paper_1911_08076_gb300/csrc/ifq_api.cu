@@ -1,0 +1,486 @@
+// C ABI entry points that launch device work: filter preparation, the
+// quantized convolution (tensor-core and bit-serial paths), 2-bit pooling,
+// the layer-stack driver and its CUDA-graph form, packing helpers and the
+// device status word.  Host-only calls (the fold, shapes) live in ifq_host.cpp.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "conv_bitserial.cuh"
+#include "conv_tc.cuh"
+#include "ifq.h"
+#include "pool_pack.cuh"
+
+namespace {
+
+using namespace ifq;
+
+constexpr int kMaxK = 65536;
+constexpr int kTcMaxK = 10922;   // 3K < 2^15: accumulators exact in the fp32 tensor-memory path
+constexpr int kMaxDevices = 64;
+
+inline bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+inline size_t round_up(size_t a, size_t b) { return (a + b - 1) / b * b; }
+inline cudaStream_t S(void* s) { return (cudaStream_t)s; }
+
+// ---------------------------------------------------------------- driver entry point for TMA descriptors
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool get_encode() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+  });
+  return g_encode != nullptr;
+}
+
+// ---------------------------------------------------------------- kernel instances
+
+template <int BN>
+struct TcStages;
+template <> struct TcStages<256> { static constexpr int st = 4, raw = 5; };
+template <> struct TcStages<128> { static constexpr int st = 4, raw = 5; };
+template <> struct TcStages<64> { static constexpr int st = 3, raw = 4; };
+template <> struct TcStages<32> { static constexpr int st = 3, raw = 4; };
+
+template <int BN, int GB>
+struct TcInst {
+  static constexpr int ST = TcStages<BN>::st;
+  static constexpr int RAW = GB >= 4 ? TcStages<BN>::raw : 0;
+  using L = TcSmem<BN, ST, RAW>;
+  static void* fn() { return (void*)conv_tc_kernel<BN, ST, RAW, GB>; }
+  static cudaError_t set_attr() {
+    return cudaFuncSetAttribute(conv_tc_kernel<BN, ST, RAW, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                L::bytes);
+  }
+  static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, cudaStream_t st) {
+    dim3 grid(ceil_div(a.M, kBM), ceil_div(a.cout, BN));
+    conv_tc_kernel<BN, ST, RAW, GB><<<grid, kTcThreads, L::bytes, st>>>(tm, a);
+    return cudaGetLastError();
+  }
+};
+
+template <int GB>
+cudaError_t set_attrs_gb() {
+  cudaError_t e;
+  if ((e = TcInst<256, GB>::set_attr()) != cudaSuccess) return e;
+  if ((e = TcInst<128, GB>::set_attr()) != cudaSuccess) return e;
+  if ((e = TcInst<64, GB>::set_attr()) != cudaSuccess) return e;
+  return TcInst<32, GB>::set_attr();
+}
+
+struct DevState {
+  bool init = false;
+  int nsm = 0;
+};
+DevState g_dev[kMaxDevices];
+std::mutex g_dev_mu;
+
+// Per-device one-time setup (shared-memory limits of the kernels, SM count).
+int ensure_init(int* nsm_out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return IFQ_ECUDA;
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DevState& d = g_dev[dev];
+  if (!d.init) {
+    if (set_attrs_gb<16>() != cudaSuccess || set_attrs_gb<4>() != cudaSuccess || set_attrs_gb<1>() != cudaSuccess)
+      return IFQ_ECUDA;
+    if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
+    d.init = true;
+  }
+  if (nsm_out) *nsm_out = d.nsm;
+  return IFQ_OK;
+}
+
+int env_int(const char* name, int dflt) {
+  const char* v = getenv(name);
+  return (v && *v) ? atoi(v) : dflt;
+}
+
+// ---------------------------------------------------------------- descriptors and planning
+
+struct ConvGeom {
+  int ho, wo, M, K, Kpad, kwords;
+};
+
+int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
+  if (!d) return IFQ_EINVAL;
+  int rc = ifq_conv_out_shape(d, &g->ho, &g->wo);
+  if (rc) return rc;
+  if (d->cin % 4 != 0) return IFQ_ESHAPE;
+  if (d->out_mode < IFQ_OUT_CODES || d->out_mode > IFQ_OUT_BOTH) return IFQ_EINVAL;
+  if ((d->out_mode & IFQ_OUT_CODES) && d->cout % 4 != 0) return IFQ_ESHAPE;
+  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_BITSERIAL) return IFQ_EINVAL;
+  const long long K = (long long)d->kh * d->kw * d->cin;
+  const long long M = (long long)d->n * g->ho * g->wo;
+  if (K > kMaxK || d->cout > 65536 || M >= (1LL << 31)) return IFQ_ERANGE;
+  if ((long long)d->n * d->h * d->w * d->cin >= (1LL << 40)) return IFQ_ERANGE;
+  g->M = (int)M;
+  g->K = (int)K;
+  g->Kpad = (int)round_up((size_t)K, kBK);
+  g->kwords = ceil_div((int)K, 32);
+  return IFQ_OK;
+}
+
+size_t prep_bits_offset(const ifq_conv_desc* d, const ConvGeom& g) {
+  return round_up((size_t)d->cout * g.Kpad, 256);
+}
+
+int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
+  int path = d->path;
+  if (path == IFQ_PATH_AUTO) {
+    const int forced = env_int("IFQ_FORCE_PATH", 0);
+    path = forced ? forced : IFQ_PATH_TC;
+  }
+  if (path == IFQ_PATH_TC && g.K > kTcMaxK) path = IFQ_PATH_BITSERIAL;
+  return path;
+}
+
+// Output-channel tile: the largest of 256/128/64/32 covering cout, halved while
+// the grid has fewer CTAs than SMs (down to 64).
+int choose_bn(const ConvGeom& g, int cout, int nsm) {
+  const int forced = env_int("IFQ_TC_BN", 0);
+  if (forced == 32 || forced == 64 || forced == 128 || forced == 256) return forced;
+  int bn = 32;
+  while (bn < 256 && bn < cout) bn *= 2;
+  const int mt = ceil_div(g.M, kBM);
+  while (bn > 64 && (long long)mt * ceil_div(cout, bn) < nsm) bn /= 2;
+  return bn;
+}
+
+template <int GB>
+cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, cudaStream_t st) {
+  switch (bn) {
+    case 256: return TcInst<256, GB>::launch(tm, a, st);
+    case 128: return TcInst<128, GB>::launch(tm, a, st);
+    case 64: return TcInst<64, GB>::launch(tm, a, st);
+    default: return TcInst<32, GB>::launch(tm, a, st);
+  }
+}
+
+int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
+             void* y_codes, int32_t* y_acc, cudaStream_t st) {
+  ConvGeom g;
+  int rc = check_conv(d, &g);
+  if (rc) return rc;
+  if (!x || !w_prep) return IFQ_EINVAL;
+  if ((d->out_mode & IFQ_OUT_CODES) && (!y_codes || !thr || !sign)) return IFQ_EINVAL;
+  if ((d->out_mode & IFQ_OUT_ACC) && !y_acc) return IFQ_EINVAL;
+  if (!aligned16(x) || !aligned16(w_prep) || (y_codes && !aligned16(y_codes)) || (y_acc && !aligned16(y_acc)))
+    return IFQ_EALIGN;
+  int nsm = 0;
+  if ((rc = ensure_init(&nsm))) return rc;
+  uint8_t* yc = (d->out_mode & IFQ_OUT_CODES) ? (uint8_t*)y_codes : nullptr;
+  int32_t* ya = (d->out_mode & IFQ_OUT_ACC) ? y_acc : nullptr;
+  const int path = choose_path(d, g);
+  cudaError_t e;
+  if (path == IFQ_PATH_TC) {
+    if (!get_encode()) return IFQ_ECUDA;
+    const int bn = choose_bn(g, d->cout, nsm);
+    CUtensorMap tm;
+    cuuint64_t gdim[2] = {(cuuint64_t)g.Kpad, (cuuint64_t)d->cout};
+    cuuint64_t gstride[1] = {(cuuint64_t)g.Kpad};
+    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)bn};
+    cuuint32_t estr[2] = {1, 1};
+    if (g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(w_prep), gdim, gstride, box, estr,
+                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return IFQ_ECUDA;
+    ConvArgs a;
+    a.x = (const uint8_t*)x;
+    a.thr = thr;
+    a.sign = sign;
+    a.y_codes = yc;
+    a.y_acc = ya;
+    a.n = d->n; a.h = d->h; a.w = d->w; a.cin = d->cin; a.cout = d->cout;
+    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad; a.ho = g.ho; a.wo = g.wo;
+    a.M = g.M;
+    a.K = g.K;
+    a.nk = g.Kpad / kBK;
+    if (d->cin % 64 == 0) e = launch_tc_gb<16>(bn, tm, a, st);
+    else if (d->cin % 16 == 0) e = launch_tc_gb<4>(bn, tm, a, st);
+    else e = launch_tc_gb<1>(bn, tm, a, st);
+  } else {
+    BsArgs a;
+    a.x = (const uint8_t*)x;
+    a.wbits = (const uint32_t*)((const uint8_t*)w_prep + prep_bits_offset(d, g));
+    a.thr = thr;
+    a.sign = sign;
+    a.y_codes = yc;
+    a.y_acc = ya;
+    a.n = d->n; a.h = d->h; a.w = d->w; a.cin = d->cin; a.cout = d->cout;
+    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad; a.ho = g.ho; a.wo = g.wo;
+    a.M = g.M;
+    a.K = g.K;
+    a.kwords = g.kwords;
+    dim3 grid(ceil_div(g.M, kBsTM), ceil_div(d->cout, kBsTN));
+    conv_bitserial_kernel<<<grid, kBsThreads, 0, st>>>(a);
+    e = cudaGetLastError();
+  }
+  return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int launch_1d_blocks(size_t items, int threads, int nsm) {
+  size_t b = (items + threads - 1) / threads;
+  if (b > (size_t)nsm * 32) b = (size_t)nsm * 32;
+  return b < 1 ? 1 : (int)b;
+}
+
+int check_pool(const ifq_pool_desc* d, int* ho, int* wo) {
+  int rc = ifq_pool_out_shape(d, ho, wo);
+  if (rc) return rc;
+  if (d->c % 4 != 0 || d->pad >= d->k) return IFQ_ESHAPE;
+  if ((long long)d->n * d->h * d->w * d->c >= (1LL << 40)) return IFQ_ERANGE;
+  return IFQ_OK;
+}
+
+int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, cudaStream_t st) {
+  int ho, wo;
+  int rc = check_pool(d, &ho, &wo);
+  if (rc) return rc;
+  if (!x || !y) return IFQ_EINVAL;
+  if (!aligned16(x) || !aligned16(y)) return IFQ_EALIGN;
+  int nsm = 0;
+  if ((rc = ensure_init(&nsm))) return rc;
+  PoolArgs a;
+  a.x = (const uint8_t*)x;
+  a.sign = sign;
+  a.y = (uint8_t*)y;
+  a.n = d->n; a.h = d->h; a.w = d->w; a.c = d->c; a.k = d->k; a.stride = d->stride; a.pad = d->pad;
+  a.ho = ho; a.wo = wo;
+  const size_t pix = (size_t)d->n * ho * wo;
+  if (d->c % 64 == 0)
+    maxpool2bit_kernel<4><<<launch_1d_blocks(pix * (d->c / 64), 256, nsm), 256, 0, st>>>(a);
+  else if (d->c % 16 == 0)
+    maxpool2bit_kernel<1><<<launch_1d_blocks(pix * (d->c / 16), 256, nsm), 256, 0, st>>>(a);
+  else
+    maxpool2bit_bytes_kernel<<<launch_1d_blocks(pix * (d->c / 4), 256, nsm), 256, 0, st>>>(a);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+// Output shape (n, h, w, c) of a layer, and whether it produces codes.
+int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes) {
+  if (l.kind == IFQ_LAYER_CONV) {
+    ConvGeom g;
+    int rc = check_conv(&l.conv, &g);
+    if (rc) return rc;
+    *n = l.conv.n; *h = g.ho; *w = g.wo; *c = l.conv.cout;
+    *codes = (l.conv.out_mode & IFQ_OUT_CODES) != 0;
+    return IFQ_OK;
+  }
+  if (l.kind == IFQ_LAYER_POOL) {
+    int ho, wo;
+    int rc = check_pool(&l.pool, &ho, &wo);
+    if (rc) return rc;
+    *n = l.pool.n; *h = ho; *w = wo; *c = l.pool.c;
+    *codes = true;
+    return IFQ_OK;
+  }
+  return IFQ_EINVAL;
+}
+
+int check_stack(const ifq_layer* layers, int nlayers, const void* x) {
+  if (!layers || nlayers < 1 || !x) return IFQ_EINVAL;
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_layer& l = layers[i];
+    int n, h, w, c;
+    bool codes;
+    int rc = layer_out(l, &n, &h, &w, &c, &codes);
+    if (rc) return rc;
+    if (l.src < -1 || l.src >= i) return IFQ_EINVAL;
+    if (l.src >= 0) {
+      int sn, sh, sw, sc;
+      bool sc_codes;
+      layer_out(layers[l.src], &sn, &sh, &sw, &sc, &sc_codes);
+      if (!sc_codes) return IFQ_ESHAPE;
+      const int in_n = l.kind == IFQ_LAYER_CONV ? l.conv.n : l.pool.n;
+      const int in_h = l.kind == IFQ_LAYER_CONV ? l.conv.h : l.pool.h;
+      const int in_w = l.kind == IFQ_LAYER_CONV ? l.conv.w : l.pool.w;
+      const int in_c = l.kind == IFQ_LAYER_CONV ? l.conv.cin : l.pool.c;
+      if (in_n != sn || in_h != sh || in_w != sw || in_c != sc) return IFQ_ESHAPE;
+    }
+  }
+  return IFQ_OK;
+}
+
+int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t st) {
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_layer& l = layers[i];
+    const void* in = l.src < 0 ? x : layers[l.src].y_codes;
+    int rc;
+    if (l.kind == IFQ_LAYER_CONV)
+      rc = run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st);
+    else
+      rc = run_pool(&l.pool, in, l.sign, l.y_codes, st);
+    if (rc) return rc;
+  }
+  return IFQ_OK;
+}
+
+}  // namespace
+
+struct ifq_graph {
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+};
+
+extern "C" {
+
+int ifq_weights_prep_bytes(const ifq_conv_desc* d, size_t* bytes) {
+  ConvGeom g;
+  if (!bytes) return IFQ_EINVAL;
+  int rc = check_conv(d, &g);
+  if (rc) return rc;
+  *bytes = prep_bits_offset(d, g) + (size_t)d->cout * g.kwords * 4;
+  return IFQ_OK;
+}
+
+int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_prep, void* stream) {
+  ConvGeom g;
+  int rc = check_conv(d, &g);
+  if (rc) return rc;
+  if (!w_bits || !w_prep) return IFQ_EINVAL;
+  if (!aligned16(w_prep) || ((uintptr_t)w_bits & 3u)) return IFQ_EALIGN;
+  int nsm = 0;
+  if ((rc = ensure_init(&nsm))) return rc;
+  uint8_t* base = (uint8_t*)w_prep;
+  const int blocks = launch_1d_blocks((size_t)d->cout * (g.Kpad / 4), 256, nsm);
+  prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
+                                                     d->cout, g.K, g.Kpad, g.kwords);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_conv_workspace_bytes(const ifq_conv_desc* d, size_t* bytes) {
+  ConvGeom g;
+  if (!bytes) return IFQ_EINVAL;
+  int rc = check_conv(d, &g);
+  if (rc) return rc;
+  *bytes = 0;
+  return IFQ_OK;
+}
+
+int ifq_conv2bit(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
+                 void* y_codes, int32_t* y_acc, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  return run_conv(d, x, w_prep, thr, sign, y_codes, y_acc, S(stream));
+}
+
+int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, void* stream) {
+  return run_pool(d, x, sign, y, S(stream));
+}
+
+int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* bytes) {
+  if (!layers || nlayers < 1 || !bytes) return IFQ_EINVAL;
+  *bytes = 0;
+  return IFQ_OK;
+}
+
+int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  int rc = check_stack(layers, nlayers, x);
+  if (rc) return rc;
+  return run_stack(layers, nlayers, x, S(stream));
+}
+
+int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream,
+                     ifq_graph** out) {
+  if (!out) return IFQ_EINVAL;
+  *out = nullptr;
+  int rc = check_stack(layers, nlayers, x);
+  if (rc) return rc;
+  if ((rc = ensure_init(nullptr))) return rc;
+  if (!get_encode()) return IFQ_ECUDA;
+  cudaStream_t cap = S(stream);
+  bool own = false;
+  if (cap == nullptr) {
+    if (cudaStreamCreateWithFlags(&cap, cudaStreamNonBlocking) != cudaSuccess) return IFQ_ECUDA;
+    own = true;
+  }
+  ifq_graph* g = new ifq_graph();
+  rc = IFQ_OK;
+  if (cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) rc = IFQ_ECUDA;
+  if (!rc) {
+    const int frc = ifq_forward(layers, nlayers, x, ws, ws_bytes, cap);
+    const cudaError_t e = cudaStreamEndCapture(cap, &g->graph);
+    if (frc) rc = frc;
+    else if (e != cudaSuccess) rc = IFQ_ECUDA;
+  }
+  if (!rc && cudaGraphInstantiate(&g->exec, g->graph, 0) != cudaSuccess) rc = IFQ_ECUDA;
+  if (own) cudaStreamDestroy(cap);
+  if (rc) {
+    ifq_graph_destroy(g);
+    return rc;
+  }
+  *out = g;
+  return IFQ_OK;
+}
+
+int ifq_graph_launch(ifq_graph* g, void* stream) {
+  if (!g || !g->exec) return IFQ_EINVAL;
+  return cudaGraphLaunch(g->exec, S(stream)) == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_graph_destroy(ifq_graph* g) {
+  if (!g) return IFQ_EINVAL;
+  if (g->exec) cudaGraphExecDestroy(g->exec);
+  if (g->graph) cudaGraphDestroy(g->graph);
+  delete g;
+  return IFQ_OK;
+}
+
+int ifq_pack_codes(const uint8_t* codes, void* packed, size_t n, void* stream) {
+  if (!codes || !packed || n % 4 != 0) return IFQ_EINVAL;
+  if ((uintptr_t)codes & 3u) return IFQ_EALIGN;
+  if (n == 0) return IFQ_OK;
+  int nsm = 0, rc;
+  if ((rc = ensure_init(&nsm))) return rc;
+  pack_codes_kernel<<<launch_1d_blocks(n / 4, 256, nsm), 256, 0, S(stream)>>>(codes, (uint8_t*)packed, n / 4);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_unpack_codes(const void* packed, uint8_t* codes, size_t n, void* stream) {
+  if (!codes || !packed || n % 4 != 0) return IFQ_EINVAL;
+  if ((uintptr_t)codes & 3u) return IFQ_EALIGN;
+  if (n == 0) return IFQ_OK;
+  int nsm = 0, rc;
+  if ((rc = ensure_init(&nsm))) return rc;
+  unpack_codes_kernel<<<launch_1d_blocks(n / 4, 256, nsm), 256, 0, S(stream)>>>((const uint8_t*)packed, codes, n / 4);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* stream) {
+  if (!w || !bits || rows < 1 || K < 1) return IFQ_EINVAL;
+  if ((uintptr_t)bits & 3u) return IFQ_EALIGN;
+  int nsm = 0, rc;
+  if ((rc = ensure_init(&nsm))) return rc;
+  const int kwords = ceil_div(K, 32);
+  pack_signs_kernel<<<launch_1d_blocks((size_t)rows * kwords, 256, nsm), 256, 0, S(stream)>>>(w, bits, rows, K,
+                                                                                               kwords);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_device_status(void* stream, int* status) {
+  if (!status) return IFQ_EINVAL;
+  if (cudaStreamSynchronize(S(stream)) != cudaSuccess) return IFQ_ECUDA;
+  int v = 0, zero = 0;
+  if (cudaMemcpyFromSymbol(&v, ifq::g_status, sizeof(int)) != cudaSuccess) return IFQ_ECUDA;
+  if (v != 0 && cudaMemcpyToSymbol(ifq::g_status, &zero, sizeof(int)) != cudaSuccess) return IFQ_ECUDA;
+  *status = v;
+  return IFQ_OK;
+}
+
+}  // extern "C"

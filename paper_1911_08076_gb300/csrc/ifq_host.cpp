@@ -1,0 +1,102 @@
+// Host-only parts of the C ABI: the integrated fixed-point fold (Sec. 3.2,
+// Eq. (6)-(7) + floor), packed sizes, output shapes and status strings.
+// Compiled with -ffp-contract=off so the double arithmetic of the fold is
+// rounded exactly in the order written.
+#include <cmath>
+#include <cstddef>
+#include <cstdint>
+
+#include "ifq.h"
+
+extern "C" const char* ifq_status_str(int s) {
+  switch (s) {
+    case IFQ_OK: return "ok";
+    case IFQ_EINVAL: return "invalid argument";
+    case IFQ_ESHAPE: return "invalid or unsupported shape";
+    case IFQ_EALIGN: return "misaligned pointer";
+    case IFQ_ERANGE: return "size out of supported range";
+    case IFQ_ECUDA: return "CUDA runtime error";
+    case IFQ_ETIMEOUT: return "bounded device wait ran out";
+    case IFQ_EUNSUPPORTED: return "unsupported configuration";
+    case IFQ_EWORKSPACE: return "workspace missing or too small";
+    default: return "unknown status";
+  }
+}
+
+extern "C" int ifq_version(void) { return 100; }
+
+// Eq. (3)'s uniform level i (1-based) in the compact form of Sec. 3.2.
+static inline double level(int i, double q_base, double q_offset) { return (double)i * q_base + q_offset; }
+
+extern "C" int ifq_fold_layer(int cout, int K, int kbits, const float* alpha, float delta_in, const float* bias,
+                              const float* gamma, const float* beta, const float* mean, const float* var, float eps,
+                              float q_base, float q_offset, int32_t* thr_out, int8_t* sign_out) {
+  if (cout < 1 || K < 1 || kbits < 1 || kbits > 8) return IFQ_EINVAL;
+  if (!alpha || !gamma || !beta || !mean || !var || !thr_out || !sign_out) return IFQ_EINVAL;
+  const double din = delta_in, qb = q_base, qo = q_offset, ep = eps;
+  if (!(din > 0.0) || !std::isfinite(din) || !(qb > 0.0) || !std::isfinite(qb) || !std::isfinite(qo) ||
+      !std::isfinite(ep))
+    return IFQ_EINVAL;
+  const int L = (1 << kbits) - 1;
+  const double amax = (double)L * (double)K;
+  // validate everything before writing anything
+  for (int n = 0; n < cout; ++n) {
+    const double a = alpha[n], g = gamma[n], be = beta[n], mu = mean[n], v = var[n];
+    const double b = bias ? (double)bias[n] : 0.0;
+    if (!(a > 0.0) || !std::isfinite(a) || !std::isfinite(g) || !std::isfinite(be) || !std::isfinite(mu) ||
+        !std::isfinite(v) || !std::isfinite(b) || !(v + ep > 0.0))
+      return IFQ_EINVAL;
+  }
+  for (int n = 0; n < cout; ++n) {
+    const double a = alpha[n], g = gamma[n], be = beta[n], mu = mean[n], v = var[n];
+    const double b = bias ? (double)bias[n] : 0.0;
+    const double s_acc = a * din;          // alpha * beta of Eq. (1): scale of the integer accumulator
+    const double sigma = std::sqrt(v + ep);  // BN denominator of Eq. (2)
+    sign_out[n] = (int8_t)(g < 0.0 ? -1 : 1);
+    for (int i = 1; i <= L; ++i) {
+      const double thr = level(i, qb, qo);
+      double t;
+      if (g == 0.0) {
+        // constant output beta: every accumulator is above (or not above) level i
+        t = (be > thr) ? -amax - 1.0 : amax;
+      } else {
+        // Eq. (7): z > thr_i  <=>  A > tau_i (gamma > 0)  or  A < tau_i (gamma < 0)
+        const double tau = ((thr - be) * sigma / g + mu - b) / s_acc;
+        t = g > 0.0 ? std::floor(tau) : std::floor(-tau);
+        if (!(t >= -amax - 1.0)) t = -amax - 1.0;
+        if (t > amax) t = amax;
+      }
+      thr_out[(size_t)n * L + (i - 1)] = (int32_t)t;
+    }
+  }
+  return IFQ_OK;
+}
+
+extern "C" int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes) {
+  if (!bytes || n < 0 || h < 0 || w < 0 || c < 0 || kbits < 1 || kbits > 32) return IFQ_EINVAL;
+  const unsigned long long bits = (unsigned long long)n * h * w * c * (unsigned long long)kbits;
+  *bytes = (size_t)((bits + 7) / 8);
+  return IFQ_OK;
+}
+
+extern "C" int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo) {
+  if (!d || !ho || !wo) return IFQ_EINVAL;
+  if (d->n < 1 || d->h < 1 || d->w < 1 || d->cin < 1 || d->cout < 1 || d->kh < 1 || d->kw < 1 || d->stride < 1 ||
+      d->pad < 0)
+    return IFQ_ESHAPE;
+  const int a = d->h + 2 * d->pad - d->kh, b = d->w + 2 * d->pad - d->kw;
+  if (a < 0 || b < 0) return IFQ_ESHAPE;
+  *ho = a / d->stride + 1;
+  *wo = b / d->stride + 1;
+  return IFQ_OK;
+}
+
+extern "C" int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo) {
+  if (!d || !ho || !wo) return IFQ_EINVAL;
+  if (d->n < 1 || d->h < 1 || d->w < 1 || d->c < 1 || d->k < 1 || d->stride < 1 || d->pad < 0) return IFQ_ESHAPE;
+  const int a = d->h + d->pad - d->k, b = d->w + d->pad - d->k;
+  if (a < 0 || b < 0) return IFQ_ESHAPE;
+  *ho = a / d->stride + 1;
+  *wo = b / d->stride + 1;
+  return IFQ_OK;
+}

@@ -1,0 +1,248 @@
+"""Thin Python binding of the C ABI in include/ifq.h (argument marshalling only).
+
+Every function has the name of the C entry point it calls.  Device buffers are
+torch CUDA tensors (or raw integer addresses); host buffers of the fold are
+numpy arrays.  A non-zero status raises IfqError.  There is no fallback: if
+libifq.so is missing or cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional, Sequence
+
+import numpy as np
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+IFQ_OK, IFQ_EINVAL, IFQ_ESHAPE, IFQ_EALIGN, IFQ_ERANGE, IFQ_ECUDA, IFQ_ETIMEOUT, IFQ_EUNSUPPORTED, IFQ_EWORKSPACE = range(9)
+IFQ_OUT_CODES, IFQ_OUT_ACC, IFQ_OUT_BOTH = 1, 2, 3
+IFQ_PATH_AUTO, IFQ_PATH_TC, IFQ_PATH_BITSERIAL = 0, 1, 2
+IFQ_LAYER_CONV, IFQ_LAYER_POOL = 1, 2
+
+
+class IfqError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {ifq_status_str(status)} (status {status})")
+        self.status = status
+
+
+class ConvDesc(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int) for f in
+                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path")]
+
+
+class PoolDesc(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int) for f in ("n", "h", "w", "c", "k", "stride", "pad")]
+
+
+class Layer(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("src", ctypes.c_int), ("conv", ConvDesc), ("pool", PoolDesc),
+                ("w_prep", ctypes.c_void_p), ("thr", ctypes.c_void_p), ("sign", ctypes.c_void_p),
+                ("y_codes", ctypes.c_void_p), ("y_acc", ctypes.c_void_p)]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_SZ = ctypes.c_size_t
+_F = ctypes.c_float
+
+_SIGS = {
+    "ifq_status_str": ([_I], ctypes.c_char_p),
+    "ifq_version": ([], _I),
+    "ifq_fold_layer": ([_I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
+    "ifq_codes_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "ifq_conv_out_shape": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
+    "ifq_weights_prep_bytes": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_SZ)], _I),
+    "ifq_pack_weights": ([ctypes.POINTER(ConvDesc), _P, _P, _P], _I),
+    "ifq_conv_workspace_bytes": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_SZ)], _I),
+    "ifq_conv2bit": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ifq_pool_out_shape": ([ctypes.POINTER(PoolDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
+    "ifq_maxpool2bit": ([ctypes.POINTER(PoolDesc), _P, _P, _P, _P], _I),
+    "ifq_forward_workspace_bytes": ([ctypes.POINTER(Layer), _I, ctypes.POINTER(_SZ)], _I),
+    "ifq_forward": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P], _I),
+    "ifq_graph_create": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, ctypes.POINTER(_P)], _I),
+    "ifq_graph_launch": ([_P, _P], _I),
+    "ifq_graph_destroy": ([_P], _I),
+    "ifq_pack_codes": ([_P, _P, _SZ, _P], _I),
+    "ifq_unpack_codes": ([_P, _P, _SZ, _P], _I),
+    "ifq_pack_signs": ([_P, _P, _I, _I, _P], _I),
+    "ifq_device_status": ([_P, ctypes.POINTER(_I)], _I),
+}
+
+# Every symbol that include/ifq.h declares.
+EXPORTS = tuple(_SIGS)
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def lib(build_if_missing: bool = True):
+    """The loaded libifq.so (built in-tree on first use if missing)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            try:  # let torch load its CUDA runtime first so one libcudart serves both
+                import torch  # noqa: F401
+            except Exception:
+                pass
+            path = _build.build() if build_if_missing else _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"libifq.so not found at {path}; build it with paper_1911_08076_gb300.build")
+            L = ctypes.CDLL(path)
+            for name, (args, res) in _SIGS.items():
+                f = getattr(L, name)
+                f.argtypes = args
+                f.restype = res
+            _lib = L
+    return _lib
+
+
+def _ptr(t) -> Optional[int]:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ok(rc: int, what: str):
+    if rc != IFQ_OK:
+        raise IfqError(rc, what)
+
+
+def ifq_status_str(status: int) -> str:
+    return lib().ifq_status_str(int(status)).decode()
+
+
+def ifq_version() -> int:
+    return lib().ifq_version()
+
+
+def ifq_fold_layer(K: int, alpha, gamma, beta, mean, var, delta_in: float = 0.5, bias=None, eps: float = 1e-5,
+                   q_base: float = 0.5, q_offset: float = -0.25, kbits: int = 2):
+    """Integrated fixed-point fold (host): returns (T int32 [cout][2^k-1], sign int8 [cout])."""
+    f32 = lambda a: None if a is None else np.ascontiguousarray(a, dtype=np.float32)
+    al, ga, be, mu, va, bi = map(f32, (alpha, gamma, beta, mean, var, bias))
+    cout = al.shape[0]
+    L = (1 << kbits) - 1
+    T = np.empty((cout, L), np.int32)
+    s = np.empty(cout, np.int8)
+    _ok(lib().ifq_fold_layer(cout, int(K), kbits, _ptr(al), delta_in, _ptr(bi), _ptr(ga), _ptr(be), _ptr(mu),
+                             _ptr(va), eps, q_base, q_offset, _ptr(T), _ptr(s)), "ifq_fold_layer")
+    return T, s
+
+
+def ifq_codes_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> int:
+    out = _SZ()
+    _ok(lib().ifq_codes_bytes(n, h, w, c, kbits, ctypes.byref(out)), "ifq_codes_bytes")
+    return out.value
+
+
+def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None):
+    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path)
+
+
+def ifq_conv_out_shape(d: ConvDesc):
+    ho, wo = _I(), _I()
+    _ok(lib().ifq_conv_out_shape(ctypes.byref(d), ctypes.byref(ho), ctypes.byref(wo)), "ifq_conv_out_shape")
+    return ho.value, wo.value
+
+
+def ifq_pool_out_shape(d: PoolDesc):
+    ho, wo = _I(), _I()
+    _ok(lib().ifq_pool_out_shape(ctypes.byref(d), ctypes.byref(ho), ctypes.byref(wo)), "ifq_pool_out_shape")
+    return ho.value, wo.value
+
+
+def ifq_weights_prep_bytes(d: ConvDesc) -> int:
+    out = _SZ()
+    _ok(lib().ifq_weights_prep_bytes(ctypes.byref(d), ctypes.byref(out)), "ifq_weights_prep_bytes")
+    return out.value
+
+
+def ifq_pack_weights(d: ConvDesc, w_bits, w_prep, stream=None):
+    _ok(lib().ifq_pack_weights(ctypes.byref(d), _ptr(w_bits), _ptr(w_prep), _stream(stream)), "ifq_pack_weights")
+
+
+def ifq_conv_workspace_bytes(d: ConvDesc) -> int:
+    out = _SZ()
+    _ok(lib().ifq_conv_workspace_bytes(ctypes.byref(d), ctypes.byref(out)), "ifq_conv_workspace_bytes")
+    return out.value
+
+
+def ifq_conv2bit(d: ConvDesc, x, w_prep, thr, sign, y_codes=None, y_acc=None, ws=None, ws_bytes: int = 0,
+                 stream=None):
+    _ok(lib().ifq_conv2bit(ctypes.byref(d), _ptr(x), _ptr(w_prep), _ptr(thr), _ptr(sign), _ptr(y_codes),
+                           _ptr(y_acc), _ptr(ws), ws_bytes, _stream(stream)), "ifq_conv2bit")
+
+
+def ifq_maxpool2bit(d: PoolDesc, x, sign, y, stream=None):
+    _ok(lib().ifq_maxpool2bit(ctypes.byref(d), _ptr(x), _ptr(sign), _ptr(y), _stream(stream)), "ifq_maxpool2bit")
+
+
+def _layer_array(layers: Sequence[Layer]):
+    arr = (Layer * len(layers))(*layers)
+    return arr, len(layers)
+
+
+def ifq_forward_workspace_bytes(layers: Sequence[Layer]) -> int:
+    arr, n = _layer_array(layers)
+    out = _SZ()
+    _ok(lib().ifq_forward_workspace_bytes(arr, n, ctypes.byref(out)), "ifq_forward_workspace_bytes")
+    return out.value
+
+
+def ifq_forward(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=None):
+    arr, n = _layer_array(layers)
+    _ok(lib().ifq_forward(arr, n, _ptr(x), _ptr(ws), ws_bytes, _stream(stream)), "ifq_forward")
+
+
+def ifq_graph_create(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=None) -> int:
+    arr, n = _layer_array(layers)
+    g = _P()
+    _ok(lib().ifq_graph_create(arr, n, _ptr(x), _ptr(ws), ws_bytes, _stream(stream), ctypes.byref(g)),
+        "ifq_graph_create")
+    return g.value
+
+
+def ifq_graph_launch(g: int, stream=None):
+    _ok(lib().ifq_graph_launch(g, _stream(stream)), "ifq_graph_launch")
+
+
+def ifq_graph_destroy(g: int):
+    _ok(lib().ifq_graph_destroy(g), "ifq_graph_destroy")
+
+
+def ifq_pack_codes(codes, packed, n: int, stream=None):
+    _ok(lib().ifq_pack_codes(_ptr(codes), _ptr(packed), n, _stream(stream)), "ifq_pack_codes")
+
+
+def ifq_unpack_codes(packed, codes, n: int, stream=None):
+    _ok(lib().ifq_unpack_codes(_ptr(packed), _ptr(codes), n, _stream(stream)), "ifq_unpack_codes")
+
+
+def ifq_pack_signs(w, bits, rows: int, K: int, stream=None):
+    _ok(lib().ifq_pack_signs(_ptr(w), _ptr(bits), rows, K, _stream(stream)), "ifq_pack_signs")
+
+
+def ifq_device_status(stream=None) -> int:
+    s = _I()
+    _ok(lib().ifq_device_status(_stream(stream), ctypes.byref(s)), "ifq_device_status")
+    return s.value

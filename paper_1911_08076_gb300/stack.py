@@ -1,0 +1,119 @@
+"""Device-resident layer stacks for ifq_forward (buffer management and marshalling only).
+
+A DeviceStack takes a layer table (paper_1911_08076_gb300.synth) and its float
+parameters, folds every quantized substructure with ifq_fold_layer, packs and
+prepares the filters on the device with ifq_pack_signs / ifq_pack_weights,
+allocates every output buffer with torch, and fills the ifq_layer records that
+ifq_forward and ifq_graph_create consume.  All compute is in libifq.so.
+"""
+from __future__ import annotations
+
+from typing import Dict, List, Optional
+
+import numpy as np
+import torch
+
+from . import ifq
+
+
+class DeviceStack:
+    def __init__(self, workload, params, batch: Optional[int] = None, device: str = "cuda", path: int = 0,
+                 kbits: int = 2):
+        self.wl = workload
+        self.batch = workload.batch if batch is None else batch
+        self.device = torch.device(device)
+        self.thr: Dict[int, torch.Tensor] = {}
+        self.sign: Dict[int, torch.Tensor] = {}
+        self.w_prep: Dict[int, torch.Tensor] = {}
+        self.y_codes: Dict[int, torch.Tensor] = {}
+        self.y_acc: Dict[int, torch.Tensor] = {}
+        self.layers: List[ifq.Layer] = []
+        self.host_thr: Dict[int, np.ndarray] = {}
+        self.host_sign: Dict[int, np.ndarray] = {}
+        B = self.batch
+        for li, l in enumerate(workload.layers):
+            rec = ifq.Layer()
+            rec.kind = ifq.IFQ_LAYER_CONV if l.kind == "conv" else ifq.IFQ_LAYER_POOL
+            rec.src = l.src
+            if l.kind == "conv":
+                p = params[li]
+                mode = {"codes": ifq.IFQ_OUT_CODES, "acc": ifq.IFQ_OUT_ACC, "both": ifq.IFQ_OUT_BOTH}[l.out]
+                d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path)
+                K = l.k * l.k * l.cin
+                T, s = ifq.ifq_fold_layer(K, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias, p.eps,
+                                          p.q_base, p.q_offset, kbits)
+                self.host_thr[li], self.host_sign[li] = T, s
+                self.thr[li] = torch.from_numpy(T).to(self.device)
+                self.sign[li] = torch.from_numpy(s).to(self.device)
+                w = torch.from_numpy(np.ascontiguousarray(p.w.reshape(l.cout, K))).to(self.device)
+                kwords = (K + 31) // 32
+                bits = torch.empty((l.cout, kwords), dtype=torch.int32, device=self.device)
+                ifq.ifq_pack_signs(w, bits, l.cout, K)
+                prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=self.device)
+                ifq.ifq_pack_weights(d, bits, prep)
+                self.w_prep[li] = prep
+                ho, wo = ifq.ifq_conv_out_shape(d)
+                assert (ho, wo) == (l.ho, l.wo), (l.name, ho, wo)
+                if mode & ifq.IFQ_OUT_CODES:
+                    self.y_codes[li] = torch.empty((B, ho, wo, l.cout // 4), dtype=torch.uint8, device=self.device)
+                if mode & ifq.IFQ_OUT_ACC:
+                    self.y_acc[li] = torch.empty((B, ho, wo, l.cout), dtype=torch.int32, device=self.device)
+                rec.conv = d
+                rec.w_prep = prep.data_ptr()
+                rec.thr = self.thr[li].data_ptr()
+                rec.sign = self.sign[li].data_ptr()
+                rec.y_codes = self.y_codes[li].data_ptr() if li in self.y_codes else None
+                rec.y_acc = self.y_acc[li].data_ptr() if li in self.y_acc else None
+            else:
+                d = ifq.PoolDesc(B, l.h, l.w, l.c, l.k, l.stride, l.pad)
+                ho, wo = ifq.ifq_pool_out_shape(d)
+                assert (ho, wo) == (l.ho, l.wo), (l.name, ho, wo)
+                self.y_codes[li] = torch.empty((B, ho, wo, l.c // 4), dtype=torch.uint8, device=self.device)
+                rec.pool = d
+                rec.sign = self.sign[l.src].data_ptr() if l.signed else None
+                rec.y_codes = self.y_codes[li].data_ptr()
+            self.layers.append(rec)
+        self.ws_bytes = ifq.ifq_forward_workspace_bytes(self.layers)
+        self.ws = torch.empty(max(self.ws_bytes, 1), dtype=torch.uint8, device=self.device)
+        self._graph = None
+
+    def input_buffer(self) -> torch.Tensor:
+        wl = self.wl
+        return torch.empty((self.batch, wl.h, wl.w, wl.c // 4), dtype=torch.uint8, device=self.device)
+
+    def forward(self, x: torch.Tensor, stream=None):
+        ifq.ifq_forward(self.layers, x, self.ws, self.ws_bytes, stream)
+
+    def capture(self, x: torch.Tensor, stream=None) -> int:
+        """Capture ifq_forward on input buffer x into a CUDA graph (replaced on each call)."""
+        self.release()
+        self._graph = ifq.ifq_graph_create(self.layers, x, self.ws, self.ws_bytes, stream)
+        return self._graph
+
+    def replay(self, stream=None):
+        ifq.ifq_graph_launch(self._graph, stream)
+
+    def release(self):
+        if self._graph is not None:
+            ifq.ifq_graph_destroy(self._graph)
+            self._graph = None
+
+    def __del__(self):
+        try:
+            self.release()
+        except Exception:
+            pass
+
+    def leaf_layers(self) -> List[int]:
+        """Layers whose output no other layer consumes (the stack's results)."""
+        used = {l.src for l in self.wl.layers}
+        return [i for i in range(len(self.wl.layers)) if i not in used]
+
+    def output(self, li: int):
+        """Host copy of layer li's output: codes (packed uint8) and/or int32 accumulators."""
+        out = {}
+        if li in self.y_codes:
+            out["codes"] = self.y_codes[li].cpu().numpy()
+        if li in self.y_acc:
+            out["acc"] = self.y_acc[li].cpu().numpy()
+        return out

@@ -29,7 +29,7 @@ import numpy as np
 
 SEED_BASE = 1911_08076
 STEP = 0.5          # quantizer step of every layer (the paper's beta / beta')
-EPS = 1e-5
+EPS = float(np.float32(1e-5))   # BN epsilon as the float32 the C ABI receives
 
 
 @dataclass

@@ -1,0 +1,155 @@
+"""Host-side checks of the C ABI (no GPU): exported symbols, the product fold
+against the oracle fold, synchronous argument errors, shapes and packed sizes."""
+import ctypes
+import re
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_1911_08076_gb300 import ifq, synth
+
+HEADER = __import__("os").path.join(__import__("os").path.dirname(__file__), "..", "include", "ifq.h")
+
+
+def test_library_exports_every_declared_symbol():
+    src = open(HEADER).read()
+    declared = set(re.findall(r"^(?:int|const char\*)\s+(ifq_\w+)\(", src, re.M))
+    assert declared, "no declarations parsed"
+    L = ctypes.CDLL(ifq.lib_path()) if ifq.lib() else None
+    missing = [n for n in sorted(declared) if not hasattr(L, n)]
+    assert not missing, missing
+    assert declared == set(ifq.EXPORTS), declared ^ set(ifq.EXPORTS)
+
+
+def _fold_both(K, alpha, gamma, beta, mean, var, bias=None, eps=synth.EPS, kbits=2, delta=0.5, qb=0.5, qo=-0.25):
+    T1, s1 = ifq.ifq_fold_layer(K, alpha, gamma, beta, mean, var, delta, bias, eps, qb, qo, kbits)
+    f = lambda a: None if a is None else np.asarray(a, np.float32).astype(np.float64)
+    p = O.Params(f(alpha), f(gamma), f(beta), f(mean), f(var), f(bias), delta, qb, qo, float(np.float32(eps)), kbits)
+    T2, s2 = O.fold(p, K)
+    return T1, s1, T2, s2
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_product_fold_equals_oracle_fold(seed):
+    rng = np.random.default_rng(seed)
+    n = 4096
+    K = int(rng.choice([9, 72, 576, 2304, 9216]))
+    gamma = rng.normal(0.5, 1.0, n)
+    gamma[:16] = 0.0
+    T1, s1, T2, s2 = _fold_both(K, rng.uniform(1e-3, 3, n), gamma, rng.normal(0, 1, n), rng.normal(0, 5, n),
+                                rng.uniform(1e-3, 4, n), rng.normal(0, 2, n) if seed % 2 else None,
+                                kbits=1 + seed % 4)
+    assert (T1 == T2).all() and (s1 == s2).all()
+
+
+@pytest.mark.parametrize("wl_name", list(synth.WORKLOADS))
+def test_product_fold_equals_oracle_fold_on_workloads(wl_name):
+    wl = synth.get(wl_name)
+    rng = np.random.default_rng(wl.seed)
+    for l in wl.layers:
+        if l.kind != "conv":
+            continue
+        p = synth.draw_conv_params(rng, l)
+        T1, s1, T2, s2 = _fold_both(l.k * l.k * l.cin, p.alpha, p.gamma, p.beta, p.mean, p.var)
+        assert (T1 == T2).all() and (s1 == s2).all()
+
+
+def test_fold_rejects_invalid_parameters():
+    ok = dict(alpha=[1.0], gamma=[1.0], beta=[0.0], mean=[0.0], var=[1.0])
+    for key, bad in (("alpha", [0.0]), ("alpha", [-1.0]), ("var", [-1.0]), ("gamma", [np.nan]), ("mean", [np.inf])):
+        args = dict(ok, **{key: bad})
+        with pytest.raises(ifq.IfqError) as e:
+            ifq.ifq_fold_layer(9, **args)
+        assert e.value.status == ifq.IFQ_EINVAL
+    with pytest.raises(ifq.IfqError):
+        ifq.ifq_fold_layer(9, **ok, q_base=0.0)
+    with pytest.raises(ifq.IfqError):
+        ifq.ifq_fold_layer(9, **ok, delta_in=-0.5)
+    with pytest.raises(ifq.IfqError):
+        ifq.ifq_fold_layer(0, **ok)
+
+
+def test_feature_map_memory_numbers_of_the_paper():
+    """Table 4 / Sec. 4.1.3: conv1 output 55x55x96; k=2 -> 0.6 Mbit, k=4 -> 1.1 Mbit; Lin et al.
+    112x112x96 at 9 / 10 bits -> 10.8 / 12.0 Mbit; 18x and 10.9x savings."""
+    mb = lambda b: b * 8 / 1e6
+    k2 = mb(ifq.ifq_codes_bytes(1, 55, 55, 96, 2))
+    k4 = mb(ifq.ifq_codes_bytes(1, 55, 55, 96, 4))
+    lin9 = mb(ifq.ifq_codes_bytes(1, 112, 112, 96, 9))
+    lin10 = mb(ifq.ifq_codes_bytes(1, 112, 112, 96, 10))
+    assert round(k2, 1) == 0.6 and int(k4 * 10) / 10 == 1.1
+    assert round(lin9, 1) == 10.8 and round(lin10, 1) == 12.0
+    assert int(lin9 / k2) == 18
+    assert round(round(lin10, 1) / int(k4 * 10) * 10, 1) == 10.9
+    assert ifq.ifq_codes_bytes(1, 55, 55, 96, 2) == 72600
+
+
+@pytest.mark.parametrize("shape", [(1, 9, 9, 8, 4, 3, 1, 1), (2, 27, 27, 96, 256, 5, 1, 2), (1, 56, 56, 64, 128, 1, 2, 0),
+                                   (3, 6, 6, 256, 4096, 6, 1, 0), (1, 14, 14, 256, 512, 3, 2, 1)])
+def test_conv_out_shape_matches_oracle(shape):
+    n, h, w, cin, cout, k, s, p = shape
+    assert ifq.ifq_conv_out_shape(ifq.conv_desc(n, h, w, cin, cout, k, s, p)) == (O.conv_out(h, k, s, p),
+                                                                                 O.conv_out(w, k, s, p))
+
+
+@pytest.mark.parametrize("shape", [(1, 27, 27, 256, 3, 2, 0), (1, 13, 13, 512, 2, 1, 1), (2, 208, 208, 32, 2, 2, 0)])
+def test_pool_out_shape_matches_oracle(shape):
+    n, h, w, c, k, s, p = shape
+    assert ifq.ifq_pool_out_shape(ifq.PoolDesc(n, h, w, c, k, s, p)) == (O.pool_out(h, k, s, p),
+                                                                          O.pool_out(w, k, s, p))
+
+
+def test_argument_errors_are_synchronous():
+    """Bad descriptors and pointers are rejected before any launch (works without a GPU)."""
+    good = dict(n=1, h=8, w=8, cin=64, cout=64, k=3, stride=1, pad=1)
+    fake = 1 << 20  # never dereferenced: validation fails first
+
+    def conv(status, x=fake, w=fake, thr=fake, sign=fake, yc=fake, ya=None, **kw):
+        d = ifq.conv_desc(**dict(good, **kw))
+        with pytest.raises(ifq.IfqError) as e:
+            ifq.ifq_conv2bit(d, x, w, thr, sign, yc, ya, stream=0)
+        assert e.value.status == status, e.value
+
+    conv(ifq.IFQ_ESHAPE, cin=62)
+    conv(ifq.IFQ_ESHAPE, cout=30)                       # codes need cout % 4 == 0
+    conv(ifq.IFQ_ESHAPE, k=11)                          # window larger than padded input
+    conv(ifq.IFQ_EINVAL, out_mode=7)
+    conv(ifq.IFQ_EINVAL, path=9)
+    conv(ifq.IFQ_ERANGE, cin=8192, k=3)                 # K = 73728 > 65536
+    conv(ifq.IFQ_EINVAL, x=None)
+    conv(ifq.IFQ_EINVAL, yc=None)
+    conv(ifq.IFQ_EINVAL, thr=None)
+    conv(ifq.IFQ_EINVAL, out_mode=ifq.IFQ_OUT_ACC, ya=None)
+    conv(ifq.IFQ_EALIGN, x=fake + 4)
+    conv(ifq.IFQ_EALIGN, yc=fake + 8)
+    pd = ifq.PoolDesc(1, 8, 8, 64, 2, 2, 2)             # pad >= k
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_maxpool2bit(pd, fake, None, fake, stream=0)
+    assert e.value.status == ifq.IFQ_ESHAPE
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_maxpool2bit(ifq.PoolDesc(1, 8, 8, 66, 2, 2, 0), fake, None, fake, stream=0)
+    assert e.value.status == ifq.IFQ_ESHAPE
+
+
+def test_stack_validation_rejects_broken_chains():
+    fake = 1 << 20
+    L0 = ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=-1, conv=ifq.conv_desc(1, 8, 8, 64, 32, 3, 1, 1), w_prep=fake,
+                   thr=fake, sign=fake, y_codes=fake)
+    # next layer claims 16 input channels but layer 0 produces 32
+    L1 = ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=0, conv=ifq.conv_desc(1, 8, 8, 16, 32, 3, 1, 1), w_prep=fake,
+                   thr=fake, sign=fake, y_codes=fake)
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_forward([L0, L1], fake, stream=0)
+    assert e.value.status == ifq.IFQ_ESHAPE
+    L2 = ifq.Layer(kind=ifq.IFQ_LAYER_POOL, src=3, pool=ifq.PoolDesc(1, 8, 8, 32, 2, 2, 0), y_codes=fake)
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_forward([L0, L2], fake, stream=0)
+    assert e.value.status == ifq.IFQ_EINVAL
+    # a layer that only writes accumulators cannot feed another layer
+    L3 = ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=-1,
+                   conv=ifq.conv_desc(1, 8, 8, 64, 32, 3, 1, 1, out_mode=ifq.IFQ_OUT_ACC), w_prep=fake, y_acc=fake)
+    L4 = ifq.Layer(kind=ifq.IFQ_LAYER_POOL, src=0, pool=ifq.PoolDesc(1, 8, 8, 32, 2, 2, 0), y_codes=fake)
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_forward([L3, L4], fake, stream=0)
+    assert e.value.status == ifq.IFQ_ESHAPE

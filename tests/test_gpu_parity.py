@@ -1,0 +1,255 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle, bit-exact.
+
+Every comparison is element by element on seeded inputs: int32 accumulators
+(the integer core of Eq. (1)) and 2-bit codes (the thresholds of Eq. (7) after
+the floor of Sec. 3.2).  The oracle's own fold and chains give the expected
+values; the GPU gets thresholds from the library's host fold.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_1911_08076_gb300 import ifq, synth
+from paper_1911_08076_gb300.stack import DeviceStack
+
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
+
+DEV = "cuda"
+
+
+def _params(rng, cout, K):
+    """Float parameters scaled so that the accumulators of random data reach every code."""
+    sd = np.sqrt(K * 3.5)
+    return O.Params(rng.uniform(0.5, 1.5, cout) * 4.0 / sd, rng.normal(1.0, 0.6, cout), rng.normal(0, 0.5, cout),
+                    rng.normal(0, 1.0, cout), rng.uniform(0.5, 2.0, cout), None, 0.5, 0.5, -0.25, synth.EPS)
+
+
+def _fold_gpu(p, K):
+    T, s = ifq.ifq_fold_layer(K, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias, p.eps, p.q_base,
+                              p.q_offset)
+    return T, s
+
+
+def _run_conv(x, w, T, s, stride, pad, out_mode, path, bn=None):
+    B, H, W, C = x.shape
+    cout, k, _, _ = w.shape
+    K = k * k * C
+    d = ifq.conv_desc(B, H, W, C, cout, k, stride, pad, out_mode, path)
+    xp = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    bits = torch.from_numpy(synth.pack_signs(w).view(np.int32)).to(DEV)
+    prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=DEV)
+    ifq.ifq_pack_weights(d, bits, prep)
+    ho, wo = ifq.ifq_conv_out_shape(d)
+    yc = ya = None
+    if out_mode & ifq.IFQ_OUT_CODES:
+        yc = torch.full((B, ho, wo, cout // 4), 0x5A, dtype=torch.uint8, device=DEV)
+    if out_mode & ifq.IFQ_OUT_ACC:
+        ya = torch.full((B, ho, wo, cout), -777777, dtype=torch.int32, device=DEV)
+    thr = torch.from_numpy(T).to(DEV)
+    sg = torch.from_numpy(s).to(DEV)
+    old = os.environ.get("IFQ_TC_BN")
+    if bn:
+        os.environ["IFQ_TC_BN"] = str(bn)
+    try:
+        ifq.ifq_conv2bit(d, xp, prep, thr, sg, yc, ya)
+    finally:
+        if bn:
+            if old is None:
+                del os.environ["IFQ_TC_BN"]
+            else:
+                os.environ["IFQ_TC_BN"] = old
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    codes = None if yc is None else synth.unpack_codes(yc.cpu().numpy(), cout)
+    acc = None if ya is None else ya.cpu().numpy()
+    return codes, acc
+
+
+CONV_CASES = [
+    # B, H, W, C, cout, k, stride, pad, out_mode
+    (1, 16, 16, 64, 64, 3, 1, 1, 3),      # single 3x3 64->64 layer
+    (2, 9, 7, 64, 96, 3, 2, 1, 3),        # ragged M, partial N tile
+    (3, 11, 13, 128, 256, 3, 1, 1, 3),    # several M tiles with a ragged tail
+    (2, 8, 8, 256, 320, 1, 1, 0, 3),      # 1x1, two N tiles
+    (1, 27, 27, 96, 64, 5, 1, 2, 3),      # 5x5, cin % 64 != 0
+    (2, 12, 12, 48, 32, 3, 1, 1, 3),
+    (2, 10, 10, 16, 32, 3, 1, 1, 3),      # K = 144 (partial K stage)
+    (2, 10, 10, 8, 16, 3, 1, 1, 3),       # narrow cin
+    (1, 9, 9, 4, 8, 3, 1, 1, 3),
+    (1, 7, 7, 12, 20, 3, 1, 1, 3),
+    (4, 6, 6, 256, 512, 6, 1, 0, 3),      # FC-as-conv, K = 9216
+    (3, 1, 1, 4096, 128, 1, 1, 0, 3),     # K = 4096, M = 3
+    (2, 13, 13, 1024, 30, 1, 1, 0, 2),    # accumulators only, cout = 30
+    (1, 14, 14, 256, 512, 3, 2, 1, 1),    # stride 2, codes only
+    (1, 5, 5, 64, 64, 3, 1, 0, 1),        # no padding
+]
+
+
+@pytest.mark.parametrize("path", [ifq.IFQ_PATH_TC, ifq.IFQ_PATH_BITSERIAL], ids=["tc", "bitserial"])
+@pytest.mark.parametrize("case", CONV_CASES, ids=[str(c) for c in CONV_CASES])
+def test_conv_matches_oracle(case, path):
+    B, H, W, C, cout, k, s, p, mode = case
+    rng = np.random.default_rng(abs(hash(case)) % (2 ** 32))
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, k, k, C)) == 1, 1, -1).astype(np.int8)
+    K = k * k * C
+    prm = _params(rng, cout, K)
+    T, sg = _fold_gpu(prm, K)
+    codes, acc = _run_conv(x, w, T, sg, s, p, mode, path)
+    A = O.conv_acc(x, w, s, p)
+    if acc is not None:
+        assert (acc == A).all(), f"accumulators differ at {np.argwhere(acc != A)[:5].tolist()}"
+    if codes is not None:
+        To, so = O.fold(prm, K)
+        ref, _ = O.check_chains(A, prm, To, so)
+        assert len(np.unique(ref)) >= 3
+        assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
+
+
+@pytest.mark.parametrize("bn", [32, 64, 128, 256])
+def test_tc_every_channel_tile(bn):
+    rng = np.random.default_rng(bn)
+    B, H, W, C, cout, k = 2, 12, 11, 64, 200, 3
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, k, k, C)) == 1, 1, -1).astype(np.int8)
+    prm = _params(rng, cout, k * k * C)
+    T, sg = _fold_gpu(prm, k * k * C)
+    codes, acc = _run_conv(x, w, T, sg, 1, 1, 3, ifq.IFQ_PATH_TC, bn=bn)
+    A = O.conv_acc(x, w, 1, 1)
+    assert (acc == A).all()
+    assert (codes == O.int_chain(A, *O.fold(prm, k * k * C))).all()
+
+
+@pytest.mark.parametrize("K_case", [(3, 1024, 3, 0), (1, 10880, 1, 0)], ids=["K9216", "K10880"])
+def test_tc_extreme_accumulators_are_exact(K_case):
+    """All codes 3 with all +1 (or all -1) filters give |A| = 3K, the largest the path accepts."""
+    H, C, k, p = K_case
+    B = 130 if H == 1 else 2
+    x = np.full((B, H, H, C), 3, np.uint8)
+    w = np.ones((64, k, k, C), np.int8)
+    w[1::2] = -1
+    w[5, ..., ::3] = -1
+    K = k * k * C
+    prm = _params(np.random.default_rng(1), 64, K)
+    T, sg = _fold_gpu(prm, K)
+    codes, acc = _run_conv(x, w, T, sg, 1, p, 3, ifq.IFQ_PATH_TC)
+    A = O.conv_acc(x, w, 1, p)
+    assert abs(int(A[..., 0].max())) == 3 * K
+    assert (acc == A).all()
+    assert (codes == O.int_chain(A, *O.fold(prm, K))).all()
+
+
+def test_auto_path_beyond_tc_range_is_exact():
+    rng = np.random.default_rng(3)
+    B, C, cout = 40, 11008, 32
+    x = rng.integers(0, 4, (B, 1, 1, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, 1, 1, C)) == 1, 1, -1).astype(np.int8)
+    prm = _params(rng, cout, C)
+    T, sg = _fold_gpu(prm, C)
+    codes, acc = _run_conv(x, w, T, sg, 1, 0, 3, ifq.IFQ_PATH_AUTO)
+    A = O.conv_acc(x, w, 1, 0)
+    assert (acc == A).all()
+    assert (codes == O.int_chain(A, *O.fold(prm, C))).all()
+
+
+POOL_CASES = [
+    # B, H, W, C, k, stride, pad, signed
+    (2, 27, 27, 256, 3, 2, 0, True),
+    (2, 13, 13, 256, 3, 2, 0, True),
+    (2, 8, 8, 32, 2, 2, 0, True),
+    (1, 13, 13, 512, 2, 1, 1, True),
+    (2, 9, 9, 16, 2, 2, 0, False),
+    (1, 7, 7, 8, 2, 2, 0, True),
+    (1, 7, 5, 4, 3, 2, 1, True),
+    (3, 208, 208, 32, 2, 2, 0, True),
+]
+
+
+@pytest.mark.parametrize("case", POOL_CASES, ids=[str(c) for c in POOL_CASES])
+def test_maxpool_matches_oracle(case):
+    B, H, W, C, k, s, p, signed = case
+    rng = np.random.default_rng(sum(case[:7]))
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    sign = np.where(rng.integers(0, 10, C) == 0, -1, 1).astype(np.int8)
+    sign[0] = -1
+    d = ifq.PoolDesc(B, H, W, C, k, s, p)
+    ho, wo = ifq.ifq_pool_out_shape(d)
+    y = torch.full((B, ho, wo, C // 4), 0xA5, dtype=torch.uint8, device=DEV)
+    sg = torch.from_numpy(sign).to(DEV) if signed else None
+    ifq.ifq_maxpool2bit(d, torch.from_numpy(synth.pack_codes(x)).to(DEV), sg, y)
+    torch.cuda.synchronize()
+    got = synth.unpack_codes(y.cpu().numpy())
+    ref = O.maxpool_codes(x, k, s, p, sign if signed else None)
+    assert (got == ref).all()
+
+
+def test_pack_helpers_match_formats():
+    rng = np.random.default_rng(9)
+    c = rng.integers(0, 4, 4 * 1237, dtype=np.uint8)
+    ct = torch.from_numpy(c).to(DEV)
+    packed = torch.empty(c.size // 4, dtype=torch.uint8, device=DEV)
+    ifq.ifq_pack_codes(ct, packed, c.size)
+    assert (packed.cpu().numpy() == synth.pack_codes(c)).all()
+    back = torch.empty_like(ct)
+    ifq.ifq_unpack_codes(packed, back, c.size)
+    assert (back.cpu().numpy() == c).all()
+    w = np.where(rng.integers(0, 2, (37, 291)) == 1, 1, -1).astype(np.int8)
+    bits = torch.empty((37, (291 + 31) // 32), dtype=torch.int32, device=DEV)
+    ifq.ifq_pack_signs(torch.from_numpy(w).to(DEV), bits, 37, 291)
+    assert (bits.cpu().numpy().view(np.uint32) == synth.pack_signs(w)).all()
+
+
+# ----------------------------------------------------------------------------- whole workloads
+
+WORKLOADS = ["pr1", "resnet18", "alexnet", "tinyyolo", "tinieryolo", "roofline3x3", "roofline1x1"]
+
+
+@pytest.mark.parametrize("name", WORKLOADS)
+def test_workload_matches_oracle(name):
+    """Full-size workload on the GPU; the oracle recomputes the first and last image through
+    every layer (all images for the single-image workload)."""
+    wl = synth.get(name)
+    x, params = synth.draw_workload(wl)
+    st = DeviceStack(wl, params)
+    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    st.forward(xd)
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    imgs = [0] if wl.batch == 1 else [0, wl.batch - 1]
+    ref = O.forward(wl, x, params, images=imgs)
+    for li, l in enumerate(wl.layers):
+        out = st.output(li)
+        r = ref[li]
+        if l.kind == "conv" and l.out == "both":
+            assert (synth.unpack_codes(out["codes"][imgs], l.cout) == r["codes"]).all(), l.name
+            assert (out["acc"][imgs] == r["acc"]).all(), l.name
+        elif l.kind == "conv" and l.out == "acc":
+            assert (out["acc"][imgs] == r).all(), l.name
+        else:
+            c = l.cout if l.kind == "conv" else l.c
+            assert (synth.unpack_codes(out["codes"][imgs], c) == r).all(), l.name
+
+
+def test_graph_replay_equals_forward():
+    wl = synth.get("resnet18", batch=3)
+    x, params = synth.draw_workload(wl)
+    st = DeviceStack(wl, params)
+    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    st.forward(xd)
+    torch.cuda.synchronize()
+    direct = {li: {k: v.copy() for k, v in st.output(li).items()} for li in range(len(wl.layers))}
+    for t in st.y_codes.values():
+        t.fill_(0)
+    stream = torch.cuda.Stream()
+    st.capture(xd, stream)
+    st.replay(stream)
+    stream.synchronize()
+    for li in range(len(wl.layers)):
+        for k, v in st.output(li).items():
+            assert (v == direct[li][k]).all()
+    st.release()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
