@@ -1,0 +1,412 @@
+#!/usr/bin/env python
+"""Throughput benchmark of the quantized-substructure path on GB300.
+
+A step is one pass of the layer stack over one batch: for the default workload,
+the ResNet-18 body (16 3x3 + 3 1x1 binary x 2-bit convs, batch 32) through
+ifq_forward, replayed as a CUDA graph.  Inputs are seeded synthetic 2-bit codes
+already resident in HBM; L2 is flushed (a 256 MB write) between timed steps
+and the flush is outside the per-step CUDA events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload NAME]
+
+Rank 0 prints one JSON line.  Under torchrun each rank runs an independent
+replica (no data-path collective; a barrier and a max over ranks time the job).
+`--impl reference` times the CPU oracle on the host cores on bounded samples
+of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_1911_08076_gb300 import synth  # noqa: E402
+
+METRIC = "binary×2-bit conv TOPS and images/s at 1 GB300; % of dense INT8 peak"
+UNIT = "TOPS"
+# mma.sync.m16n8k32 s8 rate measured on this machine's GB300 (sm_103a has no tcgen05 integer MMA);
+# see profiles/tensor_peaks_gb300.md.
+INT8_PEAK_TOPS = 151.4
+FP8_PER_BF16 = 2.0          # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
+FALLBACK_BF16_TFLOPS = 1900.0
+PROFILE = os.path.join(ROOT, "profiles", "conv_tc_resnet18_b32.md")
+KERNEL_SRC = os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", "conv_tc.cuh")
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def dist_info():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)),
+            int(os.environ.get("LOCAL_RANK", 0)))
+
+
+def conv_ops(layer, batch):
+    return 2.0 * batch * layer.ho * layer.wo * layer.cout * layer.k * layer.k * layer.cin
+
+
+def alg_bytes(layer, batch):
+    """Bytes the method must move for one conv launch: 2-bit input codes read once, 1-bit
+    filters, 13 B of thresholds+sign per channel, 2-bit output codes (int32 for accumulators)."""
+    inp = batch * layer.h * layer.w * layer.cin / 4
+    wts = layer.cout * layer.k * layer.k * layer.cin / 8
+    thr = 13 * layer.cout
+    out = batch * layer.ho * layer.wo * layer.cout
+    out = out / 4 if layer.out == "codes" else (out * 4 if layer.out == "acc" else out * 4.25)
+    return inp + wts + thr + out
+
+
+def read_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), \
+            float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_BF16_TFLOPS, 1700.0, 6800.0, "fallback"
+
+
+def kernel_sha():
+    with open(KERNEL_SRC, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic():
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on this kernel source."""
+    try:
+        txt = open(PROFILE).read()
+    except OSError:
+        return None
+    sha = re.search(r"kernel_sha:\s*([0-9a-f]+)", txt)
+    tb = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    if not sha or not tb or sha.group(1) != kernel_sha():
+        return None
+    return float(tb.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.out = None
+
+    def start(self):
+        try:
+            self.out = tempfile.TemporaryFile(mode="w+")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception as e:  # no nvidia-smi: report nothing rather than guess
+            log("clock sampler unavailable:", e)
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.out.seek(0)
+        rows = [l.strip().split(", ") for l in self.out.read().splitlines() if l.strip()]
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_baseline(wl, x, params):
+    """The oracle as it stands (float and integer chains, naive loops) on the host cores, over the
+    whole batch of the workload, images split across threads."""
+    from oracle import oracle as O
+    O.build()
+    threads = len(os.sched_getaffinity(0))
+    n = wl.batch
+    t0 = time.perf_counter()
+    O.forward(wl, x[:n], params, images=list(range(n)), threads=threads)
+    dt = time.perf_counter() - t0
+    ops = sum(conv_ops(l, n) for l in wl.layers if l.kind == "conv")
+    return {"value": ops / dt / 1e12, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"all {n} images of the batch through all {len(wl.layers)} layers, float and integer "
+                      f"chains, {dt:.2f} s wall", "images_per_s": n / dt}
+
+
+def run_reference(args):
+    """CPU oracle arm: each step is one bounded sample of the workload (a slice of the output
+    channels of one conv layer for one image, cycling through the layers), sized so that the
+    whole run stays within a few minutes for any --steps/--warmup."""
+    rank, world, _ = dist_info()
+    if rank != 0:
+        return
+    from concurrent.futures import ThreadPoolExecutor
+    from oracle import oracle as O
+    O.build()
+    wl = synth.get(args.workload, args.batch)
+    x, params = synth.draw_workload(wl)
+    outs = O.forward(wl, x, params, images=[0], check_float=False)
+    convs = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
+    threads = len(os.sched_getaffinity(0))
+    inputs, folded = {}, {}
+    for li in convs:
+        l = wl.layers[li]
+        src = x[0:1] if l.src < 0 else outs[l.src]
+        inputs[li] = src["codes"] if isinstance(src, dict) else src
+        p = O.Params.from_synth(params[li])
+        folded[li] = (p,) + O.fold(p, l.k * l.k * l.cin)
+    # calibrate the oracle's rate (MAC/s per thread) on a few channels of the first layer
+    l0 = wl.layers[convs[0]]
+    t0 = time.perf_counter()
+    O.conv_acc(inputs[convs[0]], params[convs[0]].w[:4], l0.stride, l0.pad)
+    rate = 4 * l0.ho * l0.wo * l0.k * l0.k * l0.cin / max(time.perf_counter() - t0, 1e-6)
+    budget = min(1.0, 100.0 / max(1, args.steps + args.warmup))
+
+    def sample(step):
+        li = convs[step % len(convs)]
+        l = wl.layers[li]
+        per_ch = l.ho * l.wo * l.k * l.k * l.cin
+        c_sub = int(np.clip(budget * rate * threads / per_ch, 1, l.cout))
+        chunks = np.array_split(np.arange(c_sub), min(threads, c_sub))
+        p, T, s = folded[li]
+
+        def one(ch):
+            sub = O.Params(p.alpha[ch], p.gamma[ch], p.beta[ch], p.mean[ch], p.var[ch], None, p.delta_in,
+                           p.q_base, p.q_offset, p.eps)
+            A = O.conv_acc(inputs[li], params[li].w[ch], l.stride, l.pad)
+            O.check_chains(A, sub, T[ch], s[ch])
+
+        with ThreadPoolExecutor(len(chunks)) as ex:
+            list(ex.map(one, chunks))
+        return 2.0 * per_ch * c_sub
+
+    for i in range(args.warmup):
+        sample(i)
+    tot_ops, tot_t = 0.0, 0.0
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        ops = sample(i)
+        tot_t += time.perf_counter() - t0
+        tot_ops += ops
+    value = tot_ops / tot_t / 1e12
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32 (naive loops) + f64",
+            "data": "synthetic",
+            "config": {"workload": wl.name, "batch": wl.batch,
+                       "sample": "per step: a slice of the output channels of one conv layer for one image"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                             "sample": f"{args.steps} steps of one conv layer's channel slice for image 0 "
+                                       f"(cycling over {len(convs)} layers), both chains"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_1911_08076_gb300 import ifq
+    from paper_1911_08076_gb300.stack import DeviceStack
+
+    rank, world, local = dist_info()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(v):
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    wl = synth.get(args.workload, args.batch)
+    B = wl.batch
+    x, params = synth.draw_workload(wl)
+    path = {"auto": ifq.IFQ_PATH_AUTO, "tc": ifq.IFQ_PATH_TC, "bitserial": ifq.IFQ_PATH_BITSERIAL}[args.path]
+    st = DeviceStack(wl, params, device=str(dev), path=path)
+    x_host = torch.from_numpy(synth.pack_codes(x)).pin_memory()
+    xd = st.input_buffer()
+    xd.copy_(x_host)
+    stream = torch.cuda.Stream(device=dev)
+    torch.cuda.synchronize()
+    st.capture(xd, stream)
+    n_kernels = len(wl.layers)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    convs = [l for l in wl.layers if l.kind == "conv"]
+    ops = sum(conv_ops(l, B) for l in convs)
+    K, W = args.steps, args.warmup
+
+    with torch.cuda.stream(stream):
+        # ---------------- timed region: graph replays, L2 flushed between steps
+        for i in range(W):
+            st.replay(stream)
+            flush.fill_(i & 0xFF)
+        torch.cuda.synchronize()
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+        gid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+        sampler = ClockSampler(gid)
+        sampler.start()
+        barrier()
+        torch.cuda.synchronize()
+        wall0 = time.perf_counter()
+        for i in range(K):
+            starts[i].record(stream)
+            st.replay(stream)
+            ends[i].record(stream)
+            flush.fill_(i & 0xFF)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - wall0
+        barrier()
+        clocks = sampler.stop()
+        step_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / K
+        step_ms = max_over_ranks(step_ms)
+        status = ifq.ifq_device_status(stream)
+        if status != ifq.IFQ_OK:
+            raise RuntimeError(f"device status after timed region: {ifq.ifq_status_str(status)}")
+
+        # ---------------- per-launch durations of the conv kernel (eager launches, same stream)
+        KR = min(K, 300)
+        ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in wl.layers] for _ in range(KR)]
+        for i in range(KR):
+            flush.fill_(i & 0xFF)
+            st.forward_layers(xd, before=lambda li, i=i: ev[i][li][0].record(stream),
+                              after=lambda li, i=i: ev[i][li][1].record(stream), stream=stream)
+        torch.cuda.synchronize()
+        per_layer_ms = [sum(ev[i][li][0].elapsed_time(ev[i][li][1]) for i in range(KR)) / KR
+                        for li in range(len(wl.layers))]
+        conv_idx = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
+        conv_ms = sum(per_layer_ms[i] for i in conv_idx)
+        conv_ops_total = sum(conv_ops(wl.layers[i], B) for i in conv_idx)
+        conv_bytes_total = sum(alg_bytes(wl.layers[i], B) for i in conv_idx)
+
+        # ---------------- end to end through the C ABI with host buffers
+        leaves = st.leaf_layers()
+        outs_dev = [st.y_codes[li] if li in st.y_codes else st.y_acc[li] for li in leaves]
+        outs_host = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs_dev]
+        h2d = x_host.numel() * x_host.element_size()
+        d2h = sum(t.numel() * t.element_size() for t in outs_dev)
+        KE = min(K, 1000)
+        es = [torch.cuda.Event(enable_timing=True) for _ in range(KE)]
+        ee = [torch.cuda.Event(enable_timing=True) for _ in range(KE)]
+        for i in range(min(W, 20)):
+            xd.copy_(x_host, non_blocking=True)
+            st.replay(stream)
+            for h, d in zip(outs_host, outs_dev):
+                h.copy_(d, non_blocking=True)
+        torch.cuda.synchronize()
+        barrier()
+        for i in range(KE):
+            es[i].record(stream)
+            xd.copy_(x_host, non_blocking=True)
+            st.replay(stream)
+            for h, d in zip(outs_host, outs_dev):
+                h.copy_(d, non_blocking=True)
+            ee[i].record(stream)
+            flush.fill_(i & 0xFF)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(sum(s.elapsed_time(e) for s, e in zip(es, ee)) / KE)
+
+    value = world * ops / (step_ms * 1e-3) / 1e12
+    imgs = world * B / (step_ms * 1e-3)
+    bf16, bf16_sus, hbm, src = read_peaks()
+    peak = bf16 * FP8_PER_BF16
+    achieved = conv_ops_total / (conv_ms * 1e-3) / 1e12
+    traffic = profiled_traffic()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "e4m3xe4m3->f32 (exact integer: u2 codes x +-1 signs)", "data": "synthetic",
+        "config": {"workload": wl.name, "batch_per_gpu": B, "layers": len(wl.layers),
+                   "ops_per_step": ops, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "l2": "flushed between steps (256 MB write outside the step events)",
+                   "path": args.path},
+        "images_per_s": imgs,
+        "pct_of_int8_peak": 100.0 * value / (world * INT8_PEAK_TOPS),
+        "int8_peak_tops": INT8_PEAK_TOPS,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic,
+                     "kernel": "conv_tc_kernel (all conv launches of a step)",
+                     "peak_source": f"{src} bf16 burst {bf16} x {FP8_PER_BF16} (fp8/bf16 nominal)",
+                     "algorithmic_bytes_per_launch": conv_bytes_total / len(conv_idx),
+                     "ops_per_launch": conv_ops_total / len(conv_idx),
+                     "avg_launch_us": 1e3 * conv_ms / len(conv_idx)},
+        "e2e": {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "gpu_launches": K * n_kernels,
+        "clocks": clocks,
+        "timed_wall_s": wall,
+    }
+    log("per-layer us:", ", ".join(f"{l.name}={1e3 * t:.2f}" for l, t in zip(wl.layers, per_layer_ms)))
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, x, params)
+    st.release()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="resnet18", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--path", default="auto", choices=["auto", "tc", "bitserial"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -84,6 +84,21 @@ class DeviceStack:
     def forward(self, x: torch.Tensor, stream=None):
         ifq.ifq_forward(self.layers, x, self.ws, self.ws_bytes, stream)
 
+    def forward_layers(self, x: torch.Tensor, before=None, after=None, stream=None):
+        """ifq_forward's launches issued one ifq_conv2bit / ifq_maxpool2bit call at a time, with
+        optional callbacks before and after each layer (for per-launch CUDA events)."""
+        for li, rec in enumerate(self.layers):
+            src = x if rec.src < 0 else self.y_codes[rec.src]
+            if before:
+                before(li)
+            if rec.kind == ifq.IFQ_LAYER_CONV:
+                ifq.ifq_conv2bit(rec.conv, src, rec.w_prep, rec.thr, rec.sign, rec.y_codes, rec.y_acc, self.ws,
+                                 self.ws_bytes, stream)
+            else:
+                ifq.ifq_maxpool2bit(rec.pool, src, rec.sign, rec.y_codes, stream)
+            if after:
+                after(li)
+
     def capture(self, x: torch.Tensor, stream=None) -> int:
         """Capture ifq_forward on input buffer x into a CUDA graph (replaced on each call)."""
         self.release()
