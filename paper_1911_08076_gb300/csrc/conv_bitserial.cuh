@@ -36,6 +36,8 @@ __global__ void __launch_bounds__(kBsThreads) conv_bitserial_kernel(const BsArgs
   __shared__ uint32_t sW[kBsTN][kBsKC + 1];
   __shared__ int sS[kBsTM];
 
+  grid_dep_launch();
+  grid_dep_wait();
   const int tid = threadIdx.x;
   const int m0 = blockIdx.x * kBsTM, n0 = blockIdx.y * kBsTN;
   // each thread: one pixel (tid % 32) and 8 consecutive channels ((tid / 32) * 8 ..)

@@ -10,6 +10,8 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <algorithm>
+#include <utility>
 
 #include "conv_bitserial.cuh"
 #include "conv_tc.cuh"
@@ -48,37 +50,70 @@ bool get_encode() {
 
 // ---------------------------------------------------------------- kernel instances
 
-template <int BN>
-struct TcStages;
-template <> struct TcStages<256> { static constexpr int st = 4, raw = 5; };
-template <> struct TcStages<128> { static constexpr int st = 4, raw = 5; };
-template <> struct TcStages<64> { static constexpr int st = 3, raw = 4; };
-template <> struct TcStages<32> { static constexpr int st = 3, raw = 4; };
+// Programmatic dependent launch (on unless IFQ_PDL=0): a kernel may start its
+// prologue while the previous kernel in the stream finishes; every kernel here
+// waits (griddepcontrol.wait) before it touches global memory.
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = getenv("IFQ_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
 
-template <int BN, int GB>
+template <typename... Exp, typename... Act>
+cudaError_t launch_k(void (*kern)(Exp...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Act&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
+}
+
+// Tile variants of the tensor-core kernel: (BN, SUB) with their pipeline depths
+// (expanded A/B stages, raw packed-code stages) sized to the 227 KB of shared memory.
+template <int BN, int SUB>
+struct TcCfg;
+template <> struct TcCfg<256, 1> { static constexpr int st = 4, raw = 4; };
+template <> struct TcCfg<128, 2> { static constexpr int st = 3, raw = 6; };
+template <> struct TcCfg<128, 1> { static constexpr int st = 5, raw = 6; };
+template <> struct TcCfg<64, 2> { static constexpr int st = 4, raw = 6; };
+template <> struct TcCfg<64, 1> { static constexpr int st = 6, raw = 8; };
+template <> struct TcCfg<32, 2> { static constexpr int st = 4, raw = 6; };
+
+template <int BN, int SUB, int GB>
 struct TcInst {
-  static constexpr int ST = TcStages<BN>::st;
-  static constexpr int RAW = GB >= 4 ? TcStages<BN>::raw : 0;
-  using L = TcSmem<BN, ST, RAW>;
-  static void* fn() { return (void*)conv_tc_kernel<BN, ST, RAW, GB>; }
+  static constexpr int ST = TcCfg<BN, SUB>::st;
+  static constexpr int RAW = GB >= 4 ? TcCfg<BN, SUB>::raw : 0;
+  using L = TcSmem<BN, SUB, ST, RAW>;
+  static_assert(L::bytes <= 232448, "shared memory budget");
   static cudaError_t set_attr() {
-    return cudaFuncSetAttribute(conv_tc_kernel<BN, ST, RAW, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    return cudaFuncSetAttribute(conv_tc_kernel<BN, SUB, ST, RAW, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 L::bytes);
   }
-  static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, cudaStream_t st) {
-    dim3 grid(ceil_div(a.M, kBM), ceil_div(a.cout, BN));
-    conv_tc_kernel<BN, ST, RAW, GB><<<grid, kTcThreads, L::bytes, st>>>(tm, a);
-    return cudaGetLastError();
+  static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
+    const int grid = a.ntiles < nsm ? a.ntiles : nsm;
+    return launch_k(conv_tc_kernel<BN, SUB, ST, RAW, GB>, dim3(grid), dim3(kTcThreads), (size_t)L::bytes, st, tm, a);
   }
 };
 
+// The tile variants, in one list used for attribute setup and dispatch.
+#define IFQ_TC_VARIANTS(X, GB) X(256, 1, GB) X(128, 2, GB) X(128, 1, GB) X(64, 2, GB) X(64, 1, GB) X(32, 2, GB)
+
 template <int GB>
 cudaError_t set_attrs_gb() {
-  cudaError_t e;
-  if ((e = TcInst<256, GB>::set_attr()) != cudaSuccess) return e;
-  if ((e = TcInst<128, GB>::set_attr()) != cudaSuccess) return e;
-  if ((e = TcInst<64, GB>::set_attr()) != cudaSuccess) return e;
-  return TcInst<32, GB>::set_attr();
+  cudaError_t e = cudaSuccess;
+#define IFQ_SET(BN, SUB, G) \
+  if (e == cudaSuccess) e = TcInst<BN, SUB, G>::set_attr();
+  IFQ_TC_VARIANTS(IFQ_SET, GB)
+#undef IFQ_SET
+  return e;
 }
 
 struct DevState {
@@ -138,36 +173,66 @@ size_t prep_bits_offset(const ifq_conv_desc* d, const ConvGeom& g) {
   return round_up((size_t)d->cout * g.Kpad, 256);
 }
 
+bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g);
+
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
     path = forced ? forced : IFQ_PATH_TC;
   }
-  if (path == IFQ_PATH_TC && g.K > kTcMaxK) path = IFQ_PATH_BITSERIAL;
+  if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
   return path;
 }
 
-// Output-channel tile: the largest of 256/128/64/32 covering cout, halved while
-// the grid has fewer CTAs than SMs (down to 64).
-int choose_bn(const ConvGeom& g, int cout, int nsm) {
-  const int forced = env_int("IFQ_TC_BN", 0);
-  if (forced == 32 || forced == 64 || forced == 128 || forced == 256) return forced;
-  int bn = 32;
-  while (bn < 256 && bn < cout) bn *= 2;
-  const int mt = ceil_div(g.M, kBM);
-  while (bn > 64 && (long long)mt * ceil_div(cout, bn) < nsm) bn /= 2;
-  return bn;
+// Tile of the persistent tensor-core kernel: BN output channels x SUB*128
+// pixels.  Cost model (cycles, measured on GB300): one 128 x BN x 32 e4m3 MMA
+// occupies the tensor pipe for max(53, 0.535*BN) cycles, and a chain of MMAs on
+// one accumulator advances one MMA per ~128 cycles; a K stage issues 4*SUB MMAs
+// as SUB independent chains, so it takes max(4*SUB*t(BN), 4*128).  The choice
+// minimises ceil(tiles / SMs) * stage time; ties go to the larger tile.
+struct TcTile {
+  int bn, sub;
+};
+
+TcTile choose_tile(const ConvGeom& g, int cout, int nsm) {
+  const int fbn = env_int("IFQ_TC_BN", 0), fsub = env_int("IFQ_TC_SUB", 0);
+  static const TcTile kTiles[] = {{256, 1}, {128, 2}, {128, 1}, {64, 2}, {64, 1}, {32, 2}};
+  TcTile best = {32, 2};
+  double best_cost = 1e300;
+  for (const TcTile& t : kTiles) {
+    if (fbn && t.bn != fbn) continue;
+    if (fsub && t.sub != fsub) continue;
+    if (!fbn && t.bn > 32 && t.bn / 2 >= cout) continue;   // no wider than needed to cover cout
+    const long long tiles = (long long)ceil_div(g.M, 128 * t.sub) * ceil_div(cout, t.bn);
+    const double mma = t.bn <= 64 ? 53.0 : 0.535 * t.bn;
+    const double stage = std::max(4.0 * t.sub * mma, 4.0 * 128.0);
+    const double cost = (double)((tiles + nsm - 1) / nsm) * stage;
+    if (cost < best_cost * (1.0 - 1e-9) || (cost <= best_cost * (1.0 + 1e-9) && t.bn * t.sub > best.bn * best.sub)) {
+      best_cost = cost;
+      best = t;
+    }
+  }
+  return best;
 }
 
 template <int GB>
-cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, cudaStream_t st) {
-  switch (bn) {
-    case 256: return TcInst<256, GB>::launch(tm, a, st);
-    case 128: return TcInst<128, GB>::launch(tm, a, st);
-    case 64: return TcInst<64, GB>::launch(tm, a, st);
-    default: return TcInst<32, GB>::launch(tm, a, st);
-  }
+cudaError_t launch_tc_gb(TcTile t, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
+#define IFQ_LAUNCH(BN, SUB, G) \
+  if (t.bn == BN && t.sub == SUB) return TcInst<BN, SUB, G>::launch(tm, a, nsm, st);
+  IFQ_TC_VARIANTS(IFQ_LAUNCH, GB)
+#undef IFQ_LAUNCH
+  return cudaErrorInvalidValue;
+}
+
+// Whether the tensor-core kernel supports this shape: exact fp32 accumulation
+// (3K < 2^15), taps addressable by 32-bit masks, and a K-granule table that fits.
+bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  if (g.K > kTcMaxK || d->kh > 32 || d->kw > 32) return false;
+  const int gran = d->cin % 64 == 0 ? 64 : (d->cin % 16 == 0 ? 16 : 4);
+  if (g.Kpad / gran > kMaxTab) return false;
+  const long long span = ((long long)(d->kh - 1) * d->w + d->kw) * (d->cin / 4) + d->cin / 4;
+  return span < (1LL << 31);
 }
 
 int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
@@ -188,7 +253,8 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   cudaError_t e;
   if (path == IFQ_PATH_TC) {
     if (!get_encode()) return IFQ_ECUDA;
-    const int bn = choose_bn(g, d->cout, nsm);
+    const TcTile tile = choose_tile(g, d->cout, nsm);
+    const int bn = tile.bn;
     CUtensorMap tm;
     cuuint64_t gdim[2] = {(cuuint64_t)g.Kpad, (cuuint64_t)d->cout};
     cuuint64_t gstride[1] = {(cuuint64_t)g.Kpad};
@@ -209,9 +275,13 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     a.M = g.M;
     a.K = g.K;
     a.nk = g.Kpad / kBK;
-    if (d->cin % 64 == 0) e = launch_tc_gb<16>(bn, tm, a, st);
-    else if (d->cin % 16 == 0) e = launch_tc_gb<4>(bn, tm, a, st);
-    else e = launch_tc_gb<1>(bn, tm, a, st);
+    a.nt = ceil_div(d->cout, bn);
+    a.ntiles = ceil_div(g.M, 128 * tile.sub) * a.nt;
+    const int gran = d->cin % 64 == 0 ? 64 : (d->cin % 16 == 0 ? 16 : 4);
+    a.ntab = g.Kpad / gran;
+    if (gran == 64) e = launch_tc_gb<16>(tile, tm, a, nsm, st);
+    else if (gran == 16) e = launch_tc_gb<4>(tile, tm, a, nsm, st);
+    else e = launch_tc_gb<1>(tile, tm, a, nsm, st);
   } else {
     BsArgs a;
     a.x = (const uint8_t*)x;
@@ -226,8 +296,7 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     a.K = g.K;
     a.kwords = g.kwords;
     dim3 grid(ceil_div(g.M, kBsTM), ceil_div(d->cout, kBsTN));
-    conv_bitserial_kernel<<<grid, kBsThreads, 0, st>>>(a);
-    e = cudaGetLastError();
+    e = launch_k(conv_bitserial_kernel, grid, dim3(kBsThreads), 0, st, a);
   }
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
@@ -261,13 +330,14 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   a.n = d->n; a.h = d->h; a.w = d->w; a.c = d->c; a.k = d->k; a.stride = d->stride; a.pad = d->pad;
   a.ho = ho; a.wo = wo;
   const size_t pix = (size_t)d->n * ho * wo;
+  cudaError_t e;
   if (d->c % 64 == 0)
-    maxpool2bit_kernel<4><<<launch_1d_blocks(pix * (d->c / 64), 256, nsm), 256, 0, st>>>(a);
+    e = launch_k(maxpool2bit_kernel<4>, dim3(launch_1d_blocks(pix * (d->c / 64), 256, nsm)), dim3(256), 0, st, a);
   else if (d->c % 16 == 0)
-    maxpool2bit_kernel<1><<<launch_1d_blocks(pix * (d->c / 16), 256, nsm), 256, 0, st>>>(a);
+    e = launch_k(maxpool2bit_kernel<1>, dim3(launch_1d_blocks(pix * (d->c / 16), 256, nsm)), dim3(256), 0, st, a);
   else
-    maxpool2bit_bytes_kernel<<<launch_1d_blocks(pix * (d->c / 4), 256, nsm), 256, 0, st>>>(a);
-  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+    e = launch_k(maxpool2bit_bytes_kernel, dim3(launch_1d_blocks(pix * (d->c / 4), 256, nsm)), dim3(256), 0, st, a);
+  return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
 // Output shape (n, h, w, c) of a layer, and whether it produces codes.

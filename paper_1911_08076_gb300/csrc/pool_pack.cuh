@@ -51,6 +51,8 @@ struct PoolArgs {
 // U = 32-bit words handled per thread (4: 64 channels, 1: 16 channels).
 template <int U>
 __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int cw = a.c >> 4;                  // 32-bit words per pixel (c % 16 == 0)
   const int groups = cw / U;
   const long total = (long)a.n * a.ho * a.wo * groups;
@@ -103,6 +105,8 @@ __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
 
 // byte-granular variant for c % 16 != 0 (c % 4 == 0)
 __global__ void __launch_bounds__(256) maxpool2bit_bytes_kernel(const PoolArgs a) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int cb = a.c >> 2;
   const long total = (long)a.n * a.ho * a.wo * cb;
   for (long it = (long)blockIdx.x * blockDim.x + threadIdx.x; it < total; it += (long)gridDim.x * blockDim.x) {
