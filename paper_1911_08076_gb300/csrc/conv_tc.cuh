@@ -7,8 +7,8 @@
 //
 // Exact integer arithmetic on the fp8 tensor cores (sm_103a has no tcgen05
 // integer MMA):
-//   * A: code c in {0,1,2,3} is stored as the e4m3 byte c, i.e. the subnormal
-//     value c * 2^-9; the 2-bit -> 8-bit expansion is a mask per byte lane.
+//   * A: code c in {0,1,2,3} is the e4m3 byte c, i.e. the subnormal value
+//     c * 2^-9; the 2-bit -> 8-bit expansion is a mask per byte lane.
 //   * B: +1 / -1 are the e4m3 bytes 0x38 / 0xB8 (+-1.0).
 //   * Every product is c * 2^-9 exactly; every partial sum is an integer
 //     multiple of 2^-9 of magnitude <= 3K * 2^-9; with 3K < 2^15 it needs at
@@ -22,20 +22,27 @@
 // transpose).  The prepared filter rows use the same order, so the dot
 // product over K is unchanged.
 //
-// Persistent, warp-specialized CTA (one per SM).  A tile is SUB x 128 output
-// pixels by BN output channels; with SUB = 2 the two 128-row halves have their
-// own accumulators and their MMAs interleave, so consecutive MMAs do not wait
-// on each other.  18 warps:
-//   warps 0-7    gather: each thread owns one 16-byte unit (64 codes) of a
-//                row per K stage, fetched with cp.async several stages ahead
-//                (zero fill for padding) and expanded into the 128B-swizzled
-//                K-major A tile;
-//   warp 8       TMA producer of the prepared filter tile (B);
-//   warp 9       TMEM allocation and the single-thread tcgen05.mma issue;
-//   warps 10-17  epilogue: tcgen05.ld of the finished accumulator buffer
-//                (two buffers, so it overlaps the next tile's mainloop),
-//                thresholds, 2-bit packing, stores.
-// The K-stage pipeline runs continuously across a CTA's tiles.
+// Data path.  The expanded A operand never touches shared memory: gather
+// threads load packed codes from global memory into registers several K
+// stages ahead, expand them in registers and write them to tensor memory
+// (tcgen05.st), and tcgen05.mma reads A from tensor memory.  Lane m of tensor
+// memory holds output pixel m; 32-bit column c of an A stage holds K bytes
+// 4c..4c+3.  Shared memory only carries the filter tiles (B), loaded by TMA in
+// the 128B-swizzled K-major layout.
+//
+// Persistent, warp-specialized CTA (one per SM), tiles of 128 output pixels x
+// BN output channels (BN <= 128) handed out round-robin; 26 warps:
+//   warps 0-15   gather, in 4 groups of 4 warps; group g fills the K stages
+//                g, g+4, g+8, ... so four stages are filled concurrently; warp
+//                w writes rows 32*(w%4)..+31 (the tensor-memory lanes it may
+//                access), all 128 K positions of the stage;
+//   warp 16      TMA producer of the prepared filter tile;
+//   warp 17      TMEM allocation and the tcgen05.mma issue (one elected lane);
+//   warps 18-25  epilogue: tcgen05.ld of the finished accumulator (two
+//                buffers, so it overlaps the next tile's mainloop), thresholds,
+//                2-bit packing, stores.
+// Tensor memory (512 columns): accumulators in [0, 2*BN), A stages in
+// [256, 256 + 32*STAGES).  The K-stage pipeline runs continuously across tiles.
 #pragma once
 #include <cuda.h>
 
@@ -44,6 +51,14 @@
 #include "ptx.cuh"
 
 namespace ifq {
+
+// n / d for 0 <= n < 2^31 by multiply-high (Granlund-Montgomery), set up on the host.
+struct FastDiv {
+  uint32_t d, mul, shift;
+};
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, FastDiv f) {
+  return (uint32_t)(((uint64_t)__umulhi(n, f.mul) + n) >> f.shift);
+}
 
 struct ConvArgs {
   const uint8_t* x;      // packed input codes, NHWC
@@ -58,50 +73,34 @@ struct ConvArgs {
   int nt;                // number of BN-wide output-channel tiles
   int ntiles;            // M tiles * nt
   int ntab;              // entries of the K-granule table (Kpad / codes per granule)
+  FastDiv div_hw, div_wo, div_nt;   // by ho*wo, wo, nt
 };
 
+constexpr int kBM = 128;         // output pixels per tile (MMA M)
 constexpr int kBK = 128;         // K elements (= bytes) per pipeline stage
-constexpr int kRawRow = 32;      // packed bytes of one A row per stage (128 codes)
-constexpr int kGatherWarps = 8;
+constexpr int kGatherGroups = 4;
+constexpr int kGatherWarps = 4 * kGatherGroups;
 constexpr int kEpiWarps = 8;
-constexpr int kTcThreads = 32 * (kGatherWarps + 2 + kEpiWarps);   // 576
+constexpr int kTcThreads = 32 * (kGatherWarps + 2 + kEpiWarps);   // 832
 constexpr int kWarpTma = kGatherWarps, kWarpMma = kGatherWarps + 1, kWarpEpi0 = kGatherWarps + 2;
 constexpr int kMaxTab = 1024;    // K-granule table entries
+constexpr int kStages = 8;       // K stages in flight (A in tensor memory, B in shared memory)
+constexpr int kTmemA = 256;      // first tensor-memory column of the A stages
+constexpr int kAhead = 2;        // own K stages of packed codes a gather thread keeps in registers
 
-// Byte offset of 16-byte chunk `chunk` of row r inside a K-major 128B-swizzled tile.
-__device__ __forceinline__ uint32_t sw128_chunk(int r, int chunk) {
-  return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((chunk ^ (r & 7)) << 4));
-}
-// Raw staging: row r, 32 bytes; 16-byte halves swapped on alternate groups of 4 rows.
-__device__ __forceinline__ uint32_t raw_off(int r, int half) {
-  return (uint32_t)(r * kRawRow + (((half ^ (r >> 2)) & 1) << 4));
-}
-
-template <int BN, int SUB, int STAGES, int RAW>
+template <int BN>
 struct TcSmem {
-  static constexpr int kRows = 128 * SUB;
-  static constexpr int kA = kRows * kBK;          // expanded A per stage
   static constexpr int kB = BN * kBK;
-  static constexpr int kRaw = kRows * kRawRow;    // packed A per stage
-  static constexpr int offA = 0;
-  static constexpr int offB = offA + STAGES * kA;
-  static constexpr int offRaw = offB + STAGES * kB;
-  static constexpr int offThr = offRaw + RAW * kRaw;       // 2 buffers of BN float4
+  static constexpr int offB = 0;
+  static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN float4
   static constexpr int offTab = offThr + 2 * BN * 16;      // kMaxTab x int2
   static constexpr int offBar = offTab + kMaxTab * 8;
-  static constexpr int nBar = 3 * STAGES + 5;              // full_a, full_b, empty, acc_full[2], acc_empty[2], done
+  static constexpr int nBar = 2 * kStages + 5;             // full, empty, acc_full[2], acc_empty[2], done
   static constexpr int offTmem = offBar + nBar * 8;
   static constexpr int bytes = offTmem + 16 + 1024;        // + alignment slack
 };
 
-__device__ __forceinline__ void expand_store(uint32_t addr, uint32_t u) {
-  // 16 codes -> 16 e4m3 bytes; byte t of word q holds code 4t + q
-  const uint32_t o0 = u & 0x03030303u, o1 = (u >> 2) & 0x03030303u;
-  const uint32_t o2 = (u >> 4) & 0x03030303u, o3 = (u >> 6) & 0x03030303u;
-  asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(addr), "r"(o0), "r"(o1), "r"(o2), "r"(o3) : "memory");
-}
-
-// The input row (output pixel) that a gather unit reads in one tile: a base
+// The input row (output pixel) that a gather thread reads in one tile: a base
 // pointer for tap (0,0) (possibly outside the image; dereferenced only when
 // valid) and bitmasks of the taps dy / dx that fall inside the image.
 struct RowGeom {
@@ -109,48 +108,104 @@ struct RowGeom {
   uint32_t vy, vx;
 };
 
+// bits lo..hi-1 of a tap mask (empty when hi <= lo); hi - lo <= 32
+__device__ __forceinline__ uint32_t bit_range(int lo, int hi) {
+  return hi > lo ? (uint32_t)(((1ull << (hi - lo)) - 1ull) << lo) : 0u;
+}
+
 __device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
   RowGeom g;
   g.base = a.x;
   g.vy = g.vx = 0;
   if (m < a.M) {
-    const int hw = a.ho * a.wo;
-    const int b = m / hw, rem = m - b * hw;
-    const int oy = rem / a.wo, ox = rem - oy * a.wo;
+    const int b = (int)fdiv((uint32_t)m, a.div_hw), rem = m - b * a.ho * a.wo;
+    const int oy = (int)fdiv((uint32_t)rem, a.div_wo), ox = rem - oy * a.wo;
     const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
-    const int cinb = a.cin >> 2;
-    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * cinb;
-    for (int d = 0; d < a.kh; ++d)
-      if ((unsigned)(iy0 + d) < (unsigned)a.h) g.vy |= 1u << d;
-    for (int d = 0; d < a.kw; ++d)
-      if ((unsigned)(ix0 + d) < (unsigned)a.w) g.vx |= 1u << d;
+    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * (a.cin >> 2);
+    g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));
+    g.vx = bit_range(max(0, -ix0), min(a.kw, a.w - ix0));
   }
   return g;
 }
 
+__device__ __forceinline__ bool tap_ok(const RowGeom& g, int2 e) {
+  const int dy = e.y >> 8, dx = e.y & 0xFF;
+  return dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
+}
+
+// 16 bytes (64 codes) of row g at K positions stage*128 + half*64 .. +64, zero outside the image.
+template <int GB>
+__device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int stage, int half) {
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if constexpr (GB == 16) {
+    const int2 e = tab[stage * 2 + half];
+    if (tap_ok(g, e)) v = __ldg((const uint4*)(g.base + e.x));
+  } else if constexpr (GB == 4) {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int2 e = tab[stage * 8 + half * 4 + q];
+      w[q] = tap_ok(g, e) ? __ldg((const uint32_t*)(g.base + e.x)) : 0u;
+    }
+    v = make_uint4(w[0], w[1], w[2], w[3]);
+  } else {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint32_t u = 0;
+#pragma unroll
+      for (int bq = 0; bq < 4; ++bq) {
+        const int2 e = tab[stage * 32 + half * 16 + q * 4 + bq];
+        if (tap_ok(g, e)) u |= (uint32_t)__ldg(g.base + e.x) << (8 * bq);
+      }
+      w[q] = u;
+    }
+    v = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  return v;
+}
+
+// 64 packed codes -> 16 tensor-memory columns of e4m3 bytes (column 4j+q holds
+// byte t = code 4t + q of the 16 codes in word j).
+__device__ __forceinline__ void expand_tmem_store(uint32_t taddr, uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[16];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
+      "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
+      : "memory");
+}
+
 // GB: bytes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1 (cin % 4 == 0).
-template <int BN, int SUB, int STAGES, int RAW, int GB>
+template <int BN, int GB>
 __global__ void __launch_bounds__(kTcThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
-  using L = TcSmem<BN, SUB, STAGES, RAW>;
-  constexpr int kRows = L::kRows;
+  static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
+  using L = TcSmem<BN>;
   extern __shared__ uint8_t smem_raw_[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sA = sbase + L::offA, sB = sbase + L::offB, sRaw = sbase + L::offRaw;
+  const uint32_t sB = sbase + L::offB;
   float4* sThr = (float4*)(smem + L::offThr);
   int2* sTab = (int2*)(smem + L::offTab);
   const uint32_t barBase = sbase + L::offBar;
-  auto full_a = [&](int s) { return barBase + 8u * s; };
-  auto full_b = [&](int s) { return barBase + 8u * (STAGES + s); };
-  auto empty = [&](int s) { return barBase + 8u * (2 * STAGES + s); };
-  auto acc_full = [&](int b) { return barBase + 8u * (3 * STAGES + b); };
-  auto acc_empty = [&](int b) { return barBase + 8u * (3 * STAGES + 2 + b); };
-  const uint32_t done_bar = barBase + 8u * (3 * STAGES + 4);
+  // full[s]: the arrivals of the 4 warps of the gather group that owns stage s, plus
+  // the TMA producer's (with the B bytes)
+  auto full = [&](int s) { return barBase + 8u * s; };
+  auto empty = [&](int s) { return barBase + 8u * (kStages + s); };
+  auto acc_full = [&](int b) { return barBase + 8u * (2 * kStages + b); };
+  auto acc_empty = [&](int b) { return barBase + 8u * (2 * kStages + 2 + b); };
+  const uint32_t done_bar = barBase + 8u * (2 * kStages + 4);
   uint32_t* tmem_slot = (uint32_t*)(smem + L::offTmem);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  constexpr uint32_t kCols = 2 * SUB * BN;   // two buffers x SUB accumulators
+  constexpr uint32_t kCols = 512;
   const int G = gridDim.x;
   const int n_local = (args.ntiles - (int)blockIdx.x + G - 1) / G;
   const int nk = args.nk;
@@ -161,9 +216,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tmem_relinquish();
   }
   if (tid == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(full_a(s), kGatherWarps);
-      mbar_init(full_b(s), 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full(s), 4 + 1);   // one gather group (4 warps) + the TMA producer
       mbar_init(empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -197,201 +251,143 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   grid_dep_wait();
 
   if (warp < kGatherWarps) {
-    // =================== gather (im2col + expansion) ===================
-    // unit u = tid + 256*i (i < SUB): row u % kRows, half (64 codes) u / kRows
-    constexpr int kUnits = SUB;
-    int urow[kUnits], uhalf[kUnits];
-#pragma unroll
-    for (int i = 0; i < kUnits; ++i) {
-      const int u = tid + 256 * i;
-      urow[i] = u % kRows;
-      uhalf[i] = u / kRows;
-    }
+    // =================== gather: packed codes -> registers -> tensor memory ===================
+    const int group = warp >> 2, quarter = warp & 3;
+    const int r = quarter * 32 + lane;                       // A row = tensor-memory lane
+    const uint32_t tA = tmem + (uint32_t)kTmemA + ((uint32_t)(quarter * 32) << 16);
     const int total = n_local * nk;
-    auto geom = [&](int jt, RowGeom (&g)[kUnits]) {
-      const int t = (int)blockIdx.x + jt * G;
-      const int mt = t / args.nt;
-#pragma unroll
-      for (int i = 0; i < kUnits; ++i) g[i] = row_geom(args, mt * kRows + urow[i]);
-    };
-    auto gather_unit = [&](const RowGeom& g, int stage_k, int half, uint32_t dst) {
-      // 16 bytes of packed codes for K positions stage_k*128 + half*64 .. +64
-      if constexpr (GB == 16) {
-        const int2 e = sTab[stage_k * 2 + half];
-        const int dy = e.y >> 8, dx = e.y & 0xFF;
-        const bool ok = dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
-        cp_async_16(dst, ok ? g.base + e.x : args.x, ok ? 16u : 0u);
-      } else if constexpr (GB == 4) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const int2 e = sTab[stage_k * 8 + half * 4 + q];
-          const int dy = e.y >> 8, dx = e.y & 0xFF;
-          const bool ok = dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
-          cp_async_4(dst + 4 * q, ok ? g.base + e.x : args.x, ok ? 4u : 0u);
-        }
+    const int own = total > group ? (total - group + kGatherGroups - 1) / kGatherGroups : 0;   // stages of this group
+    // load cursor over this group's stages it = group + 4*j: tile l_tile, K stage l_k
+    int l_tile = 0, l_k = group;
+    while (l_k >= nk) { l_k -= nk; ++l_tile; }
+    RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r
+                                                : args.M);
+    auto next_load = [&](uint4& lo, uint4& hi) {
+      lo = load_unit<GB>(sTab, g, l_k, 0);
+      hi = load_unit<GB>(sTab, g, l_k, 1);
+      l_k += kGatherGroups;
+      if (l_k >= nk) {
+        do { l_k -= nk; ++l_tile; } while (l_k >= nk);
+        if (l_tile < n_local) g = row_geom(args, (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r);
       }
     };
-    if constexpr (GB >= 4) {
-      constexpr int D = RAW - 1;   // stages in flight ahead of the expansion
-      int i_tile = 0, i_k = 0;
-      RowGeom g[kUnits];
-      geom(0, g);
-      auto issue = [&](int it) {
-        const uint32_t slot = sRaw + (uint32_t)((it % RAW) * L::kRaw);
+    uint4 ring_lo[kAhead], ring_hi[kAhead];
 #pragma unroll
-        for (int i = 0; i < kUnits; ++i) gather_unit(g[i], i_k, uhalf[i], slot + raw_off(urow[i], uhalf[i]));
-        if (++i_k == nk) {
-          i_k = 0;
-          if (++i_tile < n_local) geom(i_tile, g);
-        }
-      };
+    for (int d = 0; d < kAhead; ++d) {
+      ring_lo[d] = ring_hi[d] = make_uint4(0u, 0u, 0u, 0u);
+      if (d < own) next_load(ring_lo[d], ring_hi[d]);
+    }
+    bool ok = true;
 #pragma unroll 1
-      for (int d = 0; d < D; ++d) {
-        if (d < total) issue(d);
-        cp_async_commit();
-      }
-#pragma unroll 1
-      for (int it = 0; it < total; ++it) {
-        const int s = it % STAGES;
-        const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-        if (it + D < total) issue(it + D);
-        cp_async_commit();
-        cp_async_wait<D>();
-        if (!mbar_wait(empty(s), ph ^ 1u)) break;
-        const uint32_t slot = sRaw + (uint32_t)((it % RAW) * L::kRaw);
-        const uint32_t dstA = sA + (uint32_t)(s * L::kA);
+    for (int base = 0; base < own && ok; base += kAhead) {
 #pragma unroll
-        for (int i = 0; i < kUnits; ++i) {
-          uint32_t u0, u1, u2, u3;
-          asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];"
-                       : "=r"(u0), "=r"(u1), "=r"(u2), "=r"(u3)
-                       : "r"(slot + raw_off(urow[i], uhalf[i])));
-          const int r = urow[i] & 127, c0 = uhalf[i] * 4;
-          const uint32_t rowA = dstA + (uint32_t)((urow[i] >> 7) * 16384);
-          expand_store(rowA + sw128_chunk(r, c0 + 0), u0);
-          expand_store(rowA + sw128_chunk(r, c0 + 1), u1);
-          expand_store(rowA + sw128_chunk(r, c0 + 2), u2);
-          expand_store(rowA + sw128_chunk(r, c0 + 3), u3);
-        }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(full_a(s));
-      }
-      cp_async_wait<0>();
-    } else {
-      // narrow channels (cin % 16 != 0): byte loads, 4 codes per byte, 16 bytes per unit
-      int it = 0;
-      bool ok = true;
-#pragma unroll 1
-      for (int jt = 0; jt < n_local && ok; ++jt) {
-        RowGeom g[kUnits];
-        geom(jt, g);
-#pragma unroll 1
-        for (int k = 0; k < nk; ++k, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-          uint32_t word[kUnits][4];
-#pragma unroll
-          for (int i = 0; i < kUnits; ++i)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              uint32_t v = 0;
-#pragma unroll
-              for (int bq = 0; bq < 4; ++bq) {
-                const int2 e = sTab[k * 32 + uhalf[i] * 16 + q * 4 + bq];
-                const int dy = e.y >> 8, dx = e.y & 0xFF;
-                const bool okb = dy != 0xFF && ((g[i].vy >> dy) & (g[i].vx >> dx) & 1u);
-                if (okb) v |= (uint32_t)__ldg(g[i].base + e.x) << (8 * bq);
-              }
-              word[i][q] = v;
-            }
-          if (!mbar_wait(empty(s), ph ^ 1u)) { ok = false; break; }
-          const uint32_t dstA = sA + (uint32_t)(s * L::kA);
-#pragma unroll
-          for (int i = 0; i < kUnits; ++i) {
-            const int r = urow[i] & 127, c0 = uhalf[i] * 4;
-            const uint32_t rowA = dstA + (uint32_t)((urow[i] >> 7) * 16384);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) expand_store(rowA + sw128_chunk(r, c0 + q), word[i][q]);
-          }
-          fence_proxy_async_smem();
+      for (int d = 0; d < kAhead; ++d) {
+        const int j = base + d;
+        if (j < own) {
+          const uint4 lo = ring_lo[d], hi = ring_hi[d];
+          if (j + kAhead < own) next_load(ring_lo[d], ring_hi[d]);
+          const int it = group + kGatherGroups * j;
+          const int s = it % kStages;
+          const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+          if (!__all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u))) { ok = false; break; }
+          tc_fence_after();
+          expand_tmem_store(tA + (uint32_t)(s * 32), lo);
+          expand_tmem_store(tA + (uint32_t)(s * 32 + 16), hi);
+          asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+          tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(full_a(s));
+          if (lane == 0) mbar_arrive(full(s));
         }
       }
     }
   } else if (warp == kWarpTma) {
     // =================== TMA producer (filters) ===================
-    if (lane == 0) {
-      int it = 0;
-      bool ok = true;
+    // the whole warp runs the loop; one elected lane issues
+    int it = 0;
+    bool ok = true;
 #pragma unroll 1
-      for (int jt = 0; jt < n_local && ok; ++jt) {
-        const int t = (int)blockIdx.x + jt * G;
-        const int n0 = (t % args.nt) * BN;
+    for (int jt = 0; jt < n_local && ok; ++jt) {
+      const int t = (int)blockIdx.x + jt * G;
+      const int n0 = (t - (int)fdiv((uint32_t)t, args.div_nt) * args.nt) * BN;
 #pragma unroll 1
-        for (int k = 0; k < nk; ++k, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-          if (!mbar_wait(empty(s), ph ^ 1u)) { ok = false; break; }
-          mbar_arrive_expect_tx(full_b(s), (uint32_t)L::kB);
-          tma_load_2d(sB + (uint32_t)(s * L::kB), &tmap_w, full_b(s), k * kBK, n0);
+      for (int k = 0; k < nk; ++k, ++it) {
+        const int s = it % kStages;
+        const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+        if (!__all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u))) { ok = false; break; }
+        if (elect_one()) {
+          mbar_arrive_expect_tx(full(s), (uint32_t)L::kB);
+          tma_load_2d(sB + (uint32_t)(s * L::kB), &tmap_w, full(s), k * kBK, n0);
         }
+        __syncwarp();
       }
-      // drain: the last load into each slot has landed before the CTA may exit
-      for (int i = it - STAGES < 0 ? 0 : it - STAGES; i < it; ++i)
-        mbar_wait(full_b(i % STAGES), (uint32_t)(i / STAGES) & 1u);
+    }
+    // drain: every load issued into a slot has landed before the CTA may exit
+    // (full(s) completes only when the gather warps and the bytes have arrived)
+    if (!ok) {
+      for (int i = it - kStages < 0 ? 0 : it - kStages; i < it; ++i)
+        mbar_wait(full(i % kStages), (uint32_t)(i / kStages) & 1u);
     }
     __syncwarp();
   } else if (warp == kWarpMma) {
     // =================== MMA issue ===================
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_e4m3_f32(128, BN);
-      int it = 0;
-      bool ok = true;
+    // the whole warp runs the loop; one elected lane issues the MMAs and commits
+    constexpr uint32_t idesc = idesc_e4m3_f32(kBM, BN);
+    int it = 0;
+    bool ok = true;
 #pragma unroll 1
-      for (int jt = 0; jt < n_local && ok; ++jt) {
-        const int ab = jt & 1;
-        if (!mbar_wait(acc_empty(ab), ((uint32_t)(jt >> 1) & 1u) ^ 1u)) break;
+    for (int jt = 0; jt < n_local && ok; ++jt) {
+      const int ab = jt & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(acc_empty(ab), ((uint32_t)(jt >> 1) & 1u) ^ 1u))) break;
+      tc_fence_after();
+      const uint32_t dacc = tmem + (uint32_t)(ab * BN);
+      // two K stages per round: one vote, fence and elect for 8 MMAs
+#pragma unroll 1
+      for (int k = 0; k < nk; k += 2, it += 2) {
+        const bool two = k + 1 < nk;
+        const int s0 = it % kStages, s1 = (it + 1) % kStages;
+        const uint32_t ph0 = (uint32_t)(it / kStages) & 1u, ph1 = (uint32_t)((it + 1) / kStages) & 1u;
+        bool got = mbar_wait(full(s0), ph0);
+        if (two) got = got && mbar_wait(full(s1), ph1);
+        if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t dacc = tmem + (uint32_t)(ab * SUB * BN);
-#pragma unroll 1
-        for (int k = 0; k < nk; ++k, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
-          if (!mbar_wait(full_a(s), ph) || !mbar_wait(full_b(s), ph)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t a0 = sA + (uint32_t)(s * L::kA), b0 = sB + (uint32_t)(s * L::kB);
+        if (elect_one()) {
+          const uint32_t a0 = tmem + (uint32_t)(kTmemA + s0 * 32), b0 = sB + (uint32_t)(s0 * L::kB);
 #pragma unroll
           for (int kk = 0; kk < kBK / 32; ++kk)
+            mma_e4m3_tmem_a(dacc, a0 + (uint32_t)(8 * kk), sdesc_sw128(b0 + 32 * kk), idesc, (k | kk) != 0 ? 1u : 0u);
+          mma_commit(empty(s0));
+          if (two) {
+            const uint32_t a1 = tmem + (uint32_t)(kTmemA + s1 * 32), b1 = sB + (uint32_t)(s1 * L::kB);
 #pragma unroll
-            for (int sub = 0; sub < SUB; ++sub)
-              mma_e4m3(dacc + (uint32_t)(sub * BN), sdesc_sw128(a0 + sub * 16384 + 32 * kk),
-                       sdesc_sw128(b0 + 32 * kk), idesc, (k | kk) != 0 ? 1u : 0u);
-          mma_commit(empty(s));
+            for (int kk = 0; kk < kBK / 32; ++kk)
+              mma_e4m3_tmem_a(dacc, a1 + (uint32_t)(8 * kk), sdesc_sw128(b1 + 32 * kk), idesc, 1u);
+            mma_commit(empty(s1));
+          }
         }
-        if (ok) mma_commit(acc_full(ab));
+        __syncwarp();
       }
-      mma_commit(done_bar);   // fires once every MMA issued above has completed
+      if (nk & 1) it -= 1;   // the last round covered a single stage
+      if (ok && elect_one()) mma_commit(acc_full(ab));
+      __syncwarp();
     }
+    if (elect_one()) mma_commit(done_bar);   // fires once every MMA issued above has completed
     __syncwarp();
   } else {
     // =================== epilogue ===================
-    // SUB = 2: warp pair e, e+4 covers lane quarter (warp % 4) of accumulators 0 and 1, all columns.
-    // SUB = 1: warp pair e, e+4 covers lane quarter (warp % 4), column halves 0 and 1.
-    constexpr int CW = SUB == 2 ? BN : BN / 2;   // columns per thread
+    // warp pair e, e+4 covers lane quarter (warp % 4), column halves 0 and 1
+    constexpr int CW = BN / 2;                  // columns per thread
     const int e = warp - kWarpEpi0;             // 0..7
     const int et = tid - kWarpEpi0 * 32;        // 0..255
     const int quarter = warp & 3;
-    const int sub = SUB == 2 ? (e >> 2) : 0;
-    const int c_lo = SUB == 2 ? 0 : (e >> 2) * CW;
-    const int row = sub * 128 + quarter * 32 + lane;   // row of the tile
+    const int c_lo = (e >> 2) * CW;
+    const int row = quarter * 32 + lane;
     bool ok = true;   // after a timed-out wait, keep only the named barriers (uniform over the 8 warps)
 #pragma unroll 1
     for (int jt = 0; jt < n_local; ++jt) {
       const int t = (int)blockIdx.x + jt * G;
-      const int n0 = (t % args.nt) * BN;
-      const int m = (t / args.nt) * kRows + row;
+      const int mt = (int)fdiv((uint32_t)t, args.div_nt);
+      const int n0 = (t - mt * args.nt) * BN;
+      const int m = mt * kBM + row;
       const int tb = args.nt > 1 ? (jt & 1) : 0;
       if (jt == 0 || args.nt > 1) {
         for (int c = et; c < BN; c += 256) {
@@ -407,10 +403,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         named_bar(1, kEpiWarps * 32);
       }
       const int ab = jt & 1;
-      if (ok) ok = mbar_wait(acc_full(ab), (uint32_t)(jt >> 1) & 1u);
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(acc_full(ab), (uint32_t)(jt >> 1) & 1u));
       if (!ok) continue;
       tc_fence_after();
-      const uint32_t tacc = tmem + (uint32_t)((ab * SUB + sub) * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
+      const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
       const float4* th = sThr + tb * BN + c_lo;
       uint32_t packed[CW / 16];
 #pragma unroll

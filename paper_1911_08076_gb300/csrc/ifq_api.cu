@@ -76,41 +76,27 @@ cudaError_t launch_k(void (*kern)(Exp...), dim3 grid, dim3 block, size_t smem, c
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
 }
 
-// Tile variants of the tensor-core kernel: (BN, SUB) with their pipeline depths
-// (expanded A/B stages, raw packed-code stages) sized to the 227 KB of shared memory.
-template <int BN, int SUB>
-struct TcCfg;
-template <> struct TcCfg<256, 1> { static constexpr int st = 4, raw = 4; };
-template <> struct TcCfg<128, 2> { static constexpr int st = 3, raw = 6; };
-template <> struct TcCfg<128, 1> { static constexpr int st = 5, raw = 6; };
-template <> struct TcCfg<64, 2> { static constexpr int st = 4, raw = 6; };
-template <> struct TcCfg<64, 1> { static constexpr int st = 6, raw = 8; };
-template <> struct TcCfg<32, 2> { static constexpr int st = 4, raw = 6; };
-
-template <int BN, int SUB, int GB>
+template <int BN, int GB>
 struct TcInst {
-  static constexpr int ST = TcCfg<BN, SUB>::st;
-  static constexpr int RAW = GB >= 4 ? TcCfg<BN, SUB>::raw : 0;
-  using L = TcSmem<BN, SUB, ST, RAW>;
+  using L = TcSmem<BN>;
   static_assert(L::bytes <= 232448, "shared memory budget");
   static cudaError_t set_attr() {
-    return cudaFuncSetAttribute(conv_tc_kernel<BN, SUB, ST, RAW, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                L::bytes);
+    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
     const int grid = a.ntiles < nsm ? a.ntiles : nsm;
-    return launch_k(conv_tc_kernel<BN, SUB, ST, RAW, GB>, dim3(grid), dim3(kTcThreads), (size_t)L::bytes, st, tm, a);
+    return launch_k(conv_tc_kernel<BN, GB>, dim3(grid), dim3(kTcThreads), (size_t)L::bytes, st, tm, a);
   }
 };
 
-// The tile variants, in one list used for attribute setup and dispatch.
-#define IFQ_TC_VARIANTS(X, GB) X(256, 1, GB) X(128, 2, GB) X(128, 1, GB) X(64, 2, GB) X(64, 1, GB) X(32, 2, GB)
+// The output-channel tile widths of the tensor-core kernel.
+#define IFQ_TC_VARIANTS(X, GB) X(128, GB) X(64, GB) X(32, GB)
 
 template <int GB>
 cudaError_t set_attrs_gb() {
   cudaError_t e = cudaSuccess;
-#define IFQ_SET(BN, SUB, G) \
-  if (e == cudaSuccess) e = TcInst<BN, SUB, G>::set_attr();
+#define IFQ_SET(BN, G) \
+  if (e == cudaSuccess) e = TcInst<BN, G>::set_attr();
   IFQ_TC_VARIANTS(IFQ_SET, GB)
 #undef IFQ_SET
   return e;
@@ -137,6 +123,18 @@ int ensure_init(int* nsm_out) {
   }
   if (nsm_out) *nsm_out = d.nsm;
   return IFQ_OK;
+}
+
+// Multiply-high divisor for n / d with 0 <= n < 2^31 (d >= 1): shift = ceil(log2 d),
+// mul = floor(2^32 * (2^shift - d) / d) + 1, n / d = (umulhi(n, mul) + n) >> shift.
+FastDiv make_fastdiv(uint32_t d) {
+  FastDiv f;
+  f.d = d;
+  uint32_t l = 0;
+  while ((1ull << l) < d) ++l;
+  f.shift = l;
+  f.mul = (uint32_t)(((1ull << 32) * ((1ull << l) - d)) / d + 1ull);
+  return f;
 }
 
 int env_int(const char* name, int dflt) {
@@ -185,41 +183,33 @@ int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   return path;
 }
 
-// Tile of the persistent tensor-core kernel: BN output channels x SUB*128
-// pixels.  Cost model (cycles, measured on GB300): one 128 x BN x 32 e4m3 MMA
-// occupies the tensor pipe for max(53, 0.535*BN) cycles, and a chain of MMAs on
-// one accumulator advances one MMA per ~128 cycles; a K stage issues 4*SUB MMAs
-// as SUB independent chains, so it takes max(4*SUB*t(BN), 4*128).  The choice
-// minimises ceil(tiles / SMs) * stage time; ties go to the larger tile.
-struct TcTile {
-  int bn, sub;
-};
-
-TcTile choose_tile(const ConvGeom& g, int cout, int nsm) {
-  const int fbn = env_int("IFQ_TC_BN", 0), fsub = env_int("IFQ_TC_SUB", 0);
-  static const TcTile kTiles[] = {{256, 1}, {128, 2}, {128, 1}, {64, 2}, {64, 1}, {32, 2}};
-  TcTile best = {32, 2};
+// Output-channel tile BN of the persistent tensor-core kernel (128 pixels x BN).
+// Cost model: one 128 x BN x 32 e4m3 MMA takes t(BN) cycles on GB300 (measured
+// 52 / 54 / 72 at BN = 32 / 64 / 128, independent of whether consecutive MMAs
+// share an accumulator), a K stage issues 4 of them, and the makespan is
+// ceil(tiles / SMs) * nk * 4 * t(BN).  Ties go to the wider tile.
+int choose_bn(const ConvGeom& g, int cout, int nsm) {
+  const int forced = env_int("IFQ_TC_BN", 0);
+  if (forced == 32 || forced == 64 || forced == 128) return forced;
+  int best = 32;
   double best_cost = 1e300;
-  for (const TcTile& t : kTiles) {
-    if (fbn && t.bn != fbn) continue;
-    if (fsub && t.sub != fsub) continue;
-    if (!fbn && t.bn > 32 && t.bn / 2 >= cout) continue;   // no wider than needed to cover cout
-    const long long tiles = (long long)ceil_div(g.M, 128 * t.sub) * ceil_div(cout, t.bn);
-    const double mma = t.bn <= 64 ? 53.0 : 0.535 * t.bn;
-    const double stage = std::max(4.0 * t.sub * mma, 4.0 * 128.0);
-    const double cost = (double)((tiles + nsm - 1) / nsm) * stage;
-    if (cost < best_cost * (1.0 - 1e-9) || (cost <= best_cost * (1.0 + 1e-9) && t.bn * t.sub > best.bn * best.sub)) {
+  for (int bn = 32; bn <= 128; bn *= 2) {
+    if (bn > 32 && bn / 2 >= cout) break;   // no wider than needed to cover cout
+    const long long tiles = (long long)ceil_div(g.M, kBM) * ceil_div(cout, bn);
+    const double t = bn == 32 ? 52.0 : (bn == 64 ? 54.0 : 72.0);
+    const double cost = (double)((tiles + nsm - 1) / nsm) * t;
+    if (cost <= best_cost * (1.0 + 1e-9)) {
       best_cost = cost;
-      best = t;
+      best = bn;
     }
   }
   return best;
 }
 
 template <int GB>
-cudaError_t launch_tc_gb(TcTile t, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
-#define IFQ_LAUNCH(BN, SUB, G) \
-  if (t.bn == BN && t.sub == SUB) return TcInst<BN, SUB, G>::launch(tm, a, nsm, st);
+cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
+#define IFQ_LAUNCH(BN, G) \
+  if (bn == BN) return TcInst<BN, G>::launch(tm, a, nsm, st);
   IFQ_TC_VARIANTS(IFQ_LAUNCH, GB)
 #undef IFQ_LAUNCH
   return cudaErrorInvalidValue;
@@ -253,8 +243,7 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   cudaError_t e;
   if (path == IFQ_PATH_TC) {
     if (!get_encode()) return IFQ_ECUDA;
-    const TcTile tile = choose_tile(g, d->cout, nsm);
-    const int bn = tile.bn;
+    const int bn = choose_bn(g, d->cout, nsm);
     CUtensorMap tm;
     cuuint64_t gdim[2] = {(cuuint64_t)g.Kpad, (cuuint64_t)d->cout};
     cuuint64_t gstride[1] = {(cuuint64_t)g.Kpad};
@@ -276,12 +265,15 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     a.K = g.K;
     a.nk = g.Kpad / kBK;
     a.nt = ceil_div(d->cout, bn);
-    a.ntiles = ceil_div(g.M, 128 * tile.sub) * a.nt;
+    a.ntiles = ceil_div(g.M, kBM) * a.nt;
     const int gran = d->cin % 64 == 0 ? 64 : (d->cin % 16 == 0 ? 16 : 4);
     a.ntab = g.Kpad / gran;
-    if (gran == 64) e = launch_tc_gb<16>(tile, tm, a, nsm, st);
-    else if (gran == 16) e = launch_tc_gb<4>(tile, tm, a, nsm, st);
-    else e = launch_tc_gb<1>(tile, tm, a, nsm, st);
+    a.div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
+    a.div_wo = make_fastdiv((uint32_t)g.wo);
+    a.div_nt = make_fastdiv((uint32_t)a.nt);
+    if (gran == 64) e = launch_tc_gb<16>(bn, tm, a, nsm, st);
+    else if (gran == 16) e = launch_tc_gb<4>(bn, tm, a, nsm, st);
+    else e = launch_tc_gb<1>(bn, tm, a, nsm, st);
   } else {
     BsArgs a;
     a.x = (const uint8_t*)x;

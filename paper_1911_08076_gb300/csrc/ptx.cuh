@@ -14,8 +14,16 @@ __device__ int g_status;
 
 __device__ __forceinline__ void set_status(int s) { atomicCAS(&g_status, 0, s); }
 
-// ~2^22 polls of try_wait (each poll may itself suspend briefly): seconds at most.
-constexpr uint32_t kWaitLimit = 1u << 22;
+// A wait gives up after kWaitNs of wall time (read from %globaltimer) or
+// kWaitLimit polls, whichever comes first.
+constexpr uint32_t kWaitLimit = 1u << 24;
+constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+  return t;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -35,11 +43,23 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
 }
 
 // Wait until the phase with the given parity has completed; false on timeout.
+// The first poll is outside the loop: the common case (already complete) costs one try_wait.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-  for (uint32_t it = 0; it < kWaitLimit; ++it)
+  if (mbar_try(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (uint32_t it = 1; it < kWaitLimit; ++it) {
     if (mbar_try(bar, parity)) return true;
+    if ((it & 255u) == 0 && global_ns() - t0 > kWaitNs) break;
+  }
   set_status(IFQ_ETIMEOUT);
   return false;
+}
+
+// One lane of a converged warp, chosen by the hardware (all 32 lanes must execute this).
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred;
+  asm volatile("{.reg .pred p; elect.sync _|p, 0xffffffff; selp.u32 %0, 1, 0, p;}" : "=r"(pred));
+  return pred != 0;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
@@ -130,6 +150,16 @@ __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t adesc, uint64
       "{.reg .pred p; setp.ne.b32 p, %4, 0;"
       " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;}" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Same MMA with the A operand read from tensor memory (lane = row, 32-bit column = 4 K bytes).
+__device__ __forceinline__ void mma_e4m3_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                                uint32_t accumulate) {
+  asm volatile(
+      "{.reg .pred p; setp.ne.b32 p, %4, 0;"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
 
