@@ -199,7 +199,13 @@ typedef struct {
   int32_t* y_acc;
 } ifq_layer;
 
-/* Workspace that ifq_forward needs for `layers` (host, pure); may be 0. */
+/*
+ * Workspace that lets ifq_forward run `layers` as one persistent launch (host;
+ * reads the environment variable IFQ_STACK): 4 bytes per 128-output-row block
+ * of every layer, rounded up to 256; 0 when the persistent launch is not
+ * selected (IFQ_STACK is not "1") or the stack does not qualify (it then runs
+ * one launch per layer and needs no workspace).
+ */
 int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* bytes);
 
 /*
@@ -207,7 +213,16 @@ int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* by
  * quantized network is a chain of substructures; the codes of one are the
  * input of the next, and the output scale of one is the input step of the
  * next).  Shapes are checked along the chain before any launch.
- * x (device): the stack input codes; ws (device): workspace.
+ * x (device): the stack input codes; ws (device): workspace, or NULL.
+ * By default one launch per layer in stream order (consecutive launches
+ * overlap their prologues through programmatic dependent launch).  With
+ * IFQ_STACK=1 in the environment and a workspace of
+ * ifq_forward_workspace_bytes bytes, a stack of conv layers that all take the
+ * tensor-core path, whose written buffers overlap no other buffer of the
+ * stack, runs instead as one cooperative persistent launch: its completion
+ * counters (in ws, zeroed on `stream` by every call) let each output tile
+ * start as soon as the rows it reads exist.  Calls in flight at the same time
+ * must not share a workspace.  Results are identical either way.
  */
 int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream);
 

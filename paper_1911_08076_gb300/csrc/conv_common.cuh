@@ -1,0 +1,167 @@
+// Device helpers shared by the single-layer and the stack tensor-core conv
+// kernels: layer arguments, tile geometry, the packed-code gather and the
+// 2-bit -> e4m3 expansion into tensor memory.  See conv_tc.cuh for the data
+// path and the exactness argument.
+#pragma once
+#include <cuda.h>
+
+#include <cstdint>
+
+#include "ptx.cuh"
+
+namespace ifq {
+
+
+// n / d for 0 <= n < 2^31 by multiply-high (Granlund-Montgomery), set up on the host.
+struct FastDiv {
+  uint32_t d, mul, shift;
+};
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, FastDiv f) {
+  return (uint32_t)(((uint64_t)__umulhi(n, f.mul) + n) >> f.shift);
+}
+
+struct ConvArgs {
+  const uint8_t* x;      // packed input codes, NHWC
+  const int32_t* thr;    // [cout][3]
+  const int8_t* sign;    // [cout]
+  uint8_t* y_codes;      // packed output codes or nullptr
+  int32_t* y_acc;        // int32 accumulators or nullptr
+  int n, h, w, cin, cout, kh, kw, stride, pad, ho, wo;
+  int M;                 // n*ho*wo
+  int K;                 // kh*kw*cin
+  int nk;                // number of 128-wide K stages (Kpad / 128)
+  int nt;                // number of BN-wide output-channel tiles
+  int ntiles;            // M tiles * nt
+  int ntab;              // entries of the K-granule table (Kpad / codes per granule)
+  FastDiv div_hw, div_wo, div_nt;   // by ho*wo, wo, nt
+};
+
+constexpr int kBM = 128;         // output pixels per tile (MMA M)
+constexpr int kBK = 128;         // K elements (= bytes) per pipeline stage
+constexpr int kGatherGroups = 4;
+constexpr int kGatherWarps = 4 * kGatherGroups;
+constexpr int kEpiWarps = 8;
+constexpr int kTcThreads = 32 * (kGatherWarps + 2 + kEpiWarps);   // 832
+constexpr int kWarpTma = kGatherWarps, kWarpMma = kGatherWarps + 1, kWarpEpi0 = kGatherWarps + 2;
+constexpr int kMaxTab = 1024;    // K-granule table entries
+constexpr int kStages = 8;       // K stages in flight (A in tensor memory, B in shared memory)
+constexpr int kTmemA = 256;      // first tensor-memory column of the A stages
+constexpr int kAhead = 2;        // own K stages of packed codes a gather thread keeps in registers
+
+template <int BN>
+struct TcSmem {
+  static constexpr int kB = BN * kBK;
+  static constexpr int offB = 0;
+  static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN float4
+  static constexpr int offTab = offThr + 2 * BN * 16;      // kMaxTab x int2
+  static constexpr int offBar = offTab + kMaxTab * 8;
+  static constexpr int nBar = 2 * kStages + 5;             // full, empty, acc_full[2], acc_empty[2], done
+  static constexpr int offTmem = offBar + nBar * 8;
+  static constexpr int bytes = offTmem + 16 + 1024;        // + alignment slack
+};
+
+// The input row (output pixel) that a gather thread reads in one tile: a base
+// pointer for tap (0,0) (possibly outside the image; dereferenced only when
+// valid) and bitmasks of the taps dy / dx that fall inside the image.
+struct RowGeom {
+  const uint8_t* base;
+  uint32_t vy, vx;
+};
+
+// bits lo..hi-1 of a tap mask (empty when hi <= lo); hi - lo <= 32
+__device__ __forceinline__ uint32_t bit_range(int lo, int hi) {
+  return hi > lo ? (uint32_t)(((1ull << (hi - lo)) - 1ull) << lo) : 0u;
+}
+
+__device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
+  RowGeom g;
+  g.base = a.x;
+  g.vy = g.vx = 0;
+  if (m < a.M) {
+    const int b = (int)fdiv((uint32_t)m, a.div_hw), rem = m - b * a.ho * a.wo;
+    const int oy = (int)fdiv((uint32_t)rem, a.div_wo), ox = rem - oy * a.wo;
+    const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
+    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * (a.cin >> 2);
+    g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));
+    g.vx = bit_range(max(0, -ix0), min(a.kw, a.w - ix0));
+  }
+  return g;
+}
+
+__device__ __forceinline__ bool tap_ok(const RowGeom& g, int2 e) {
+  const int dy = e.y >> 8, dx = e.y & 0xFF;
+  return dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
+}
+
+// Loads of packed codes.  COHERENT = false: the codes were written by an earlier kernel and
+// stay read-only for this one, so they may take the non-coherent read-only path (ld.global.nc).
+// COHERENT = true: another CTA of the same kernel wrote them and this thread ordered itself
+// after those writes with an acquire load of a completion counter, so only ordinary weak loads
+// are allowed (the memory model makes them see the released writes; .nc loads carry no such
+// guarantee).  Plain dereferences keep the compiler from moving them above the acquire.
+template <bool COHERENT>
+__device__ __forceinline__ uint4 ld_codes16(const uint8_t* p) {
+  if constexpr (COHERENT) return *(const uint4*)p;
+  else return __ldg((const uint4*)p);
+}
+template <bool COHERENT>
+__device__ __forceinline__ uint32_t ld_codes4(const uint8_t* p) {
+  if constexpr (COHERENT) return *(const uint32_t*)p;
+  else return __ldg((const uint32_t*)p);
+}
+template <bool COHERENT>
+__device__ __forceinline__ uint32_t ld_codes1(const uint8_t* p) {
+  if constexpr (COHERENT) return (uint32_t)*p;
+  else return (uint32_t)__ldg(p);
+}
+
+// 16 bytes (64 codes) of row g at K positions stage*128 + half*64 .. +64, zero outside the image.
+template <int GB, bool COHERENT = false>
+__device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int stage, int half) {
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if constexpr (GB == 16) {
+    const int2 e = tab[stage * 2 + half];
+    if (tap_ok(g, e)) v = ld_codes16<COHERENT>(g.base + e.x);
+  } else if constexpr (GB == 4) {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const int2 e = tab[stage * 8 + half * 4 + q];
+      w[q] = tap_ok(g, e) ? ld_codes4<COHERENT>(g.base + e.x) : 0u;
+    }
+    v = make_uint4(w[0], w[1], w[2], w[3]);
+  } else {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint32_t u = 0;
+#pragma unroll
+      for (int bq = 0; bq < 4; ++bq) {
+        const int2 e = tab[stage * 32 + half * 16 + q * 4 + bq];
+        if (tap_ok(g, e)) u |= ld_codes1<COHERENT>(g.base + e.x) << (8 * bq);
+      }
+      w[q] = u;
+    }
+    v = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  return v;
+}
+
+// 64 packed codes -> 16 tensor-memory columns of e4m3 bytes (column 4j+q holds
+// byte t = code 4t + q of the 16 codes in word j).
+__device__ __forceinline__ void expand_tmem_store(uint32_t taddr, uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t o[16];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
+      "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
+      : "memory");
+}
+
+}  // namespace ifq

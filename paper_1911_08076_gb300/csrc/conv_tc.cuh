@@ -44,143 +44,9 @@
 // Tensor memory (512 columns): accumulators in [0, 2*BN), A stages in
 // [256, 256 + 32*STAGES).  The K-stage pipeline runs continuously across tiles.
 #pragma once
-#include <cuda.h>
-
-#include <cstdint>
-
-#include "ptx.cuh"
+#include "conv_common.cuh"
 
 namespace ifq {
-
-// n / d for 0 <= n < 2^31 by multiply-high (Granlund-Montgomery), set up on the host.
-struct FastDiv {
-  uint32_t d, mul, shift;
-};
-__device__ __forceinline__ uint32_t fdiv(uint32_t n, FastDiv f) {
-  return (uint32_t)(((uint64_t)__umulhi(n, f.mul) + n) >> f.shift);
-}
-
-struct ConvArgs {
-  const uint8_t* x;      // packed input codes, NHWC
-  const int32_t* thr;    // [cout][3]
-  const int8_t* sign;    // [cout]
-  uint8_t* y_codes;      // packed output codes or nullptr
-  int32_t* y_acc;        // int32 accumulators or nullptr
-  int n, h, w, cin, cout, kh, kw, stride, pad, ho, wo;
-  int M;                 // n*ho*wo
-  int K;                 // kh*kw*cin
-  int nk;                // number of 128-wide K stages (Kpad / 128)
-  int nt;                // number of BN-wide output-channel tiles
-  int ntiles;            // M tiles * nt
-  int ntab;              // entries of the K-granule table (Kpad / codes per granule)
-  FastDiv div_hw, div_wo, div_nt;   // by ho*wo, wo, nt
-};
-
-constexpr int kBM = 128;         // output pixels per tile (MMA M)
-constexpr int kBK = 128;         // K elements (= bytes) per pipeline stage
-constexpr int kGatherGroups = 4;
-constexpr int kGatherWarps = 4 * kGatherGroups;
-constexpr int kEpiWarps = 8;
-constexpr int kTcThreads = 32 * (kGatherWarps + 2 + kEpiWarps);   // 832
-constexpr int kWarpTma = kGatherWarps, kWarpMma = kGatherWarps + 1, kWarpEpi0 = kGatherWarps + 2;
-constexpr int kMaxTab = 1024;    // K-granule table entries
-constexpr int kStages = 8;       // K stages in flight (A in tensor memory, B in shared memory)
-constexpr int kTmemA = 256;      // first tensor-memory column of the A stages
-constexpr int kAhead = 2;        // own K stages of packed codes a gather thread keeps in registers
-
-template <int BN>
-struct TcSmem {
-  static constexpr int kB = BN * kBK;
-  static constexpr int offB = 0;
-  static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN float4
-  static constexpr int offTab = offThr + 2 * BN * 16;      // kMaxTab x int2
-  static constexpr int offBar = offTab + kMaxTab * 8;
-  static constexpr int nBar = 2 * kStages + 5;             // full, empty, acc_full[2], acc_empty[2], done
-  static constexpr int offTmem = offBar + nBar * 8;
-  static constexpr int bytes = offTmem + 16 + 1024;        // + alignment slack
-};
-
-// The input row (output pixel) that a gather thread reads in one tile: a base
-// pointer for tap (0,0) (possibly outside the image; dereferenced only when
-// valid) and bitmasks of the taps dy / dx that fall inside the image.
-struct RowGeom {
-  const uint8_t* base;
-  uint32_t vy, vx;
-};
-
-// bits lo..hi-1 of a tap mask (empty when hi <= lo); hi - lo <= 32
-__device__ __forceinline__ uint32_t bit_range(int lo, int hi) {
-  return hi > lo ? (uint32_t)(((1ull << (hi - lo)) - 1ull) << lo) : 0u;
-}
-
-__device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
-  RowGeom g;
-  g.base = a.x;
-  g.vy = g.vx = 0;
-  if (m < a.M) {
-    const int b = (int)fdiv((uint32_t)m, a.div_hw), rem = m - b * a.ho * a.wo;
-    const int oy = (int)fdiv((uint32_t)rem, a.div_wo), ox = rem - oy * a.wo;
-    const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
-    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * (a.cin >> 2);
-    g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));
-    g.vx = bit_range(max(0, -ix0), min(a.kw, a.w - ix0));
-  }
-  return g;
-}
-
-__device__ __forceinline__ bool tap_ok(const RowGeom& g, int2 e) {
-  const int dy = e.y >> 8, dx = e.y & 0xFF;
-  return dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
-}
-
-// 16 bytes (64 codes) of row g at K positions stage*128 + half*64 .. +64, zero outside the image.
-template <int GB>
-__device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int stage, int half) {
-  uint4 v = make_uint4(0u, 0u, 0u, 0u);
-  if constexpr (GB == 16) {
-    const int2 e = tab[stage * 2 + half];
-    if (tap_ok(g, e)) v = __ldg((const uint4*)(g.base + e.x));
-  } else if constexpr (GB == 4) {
-    uint32_t w[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int2 e = tab[stage * 8 + half * 4 + q];
-      w[q] = tap_ok(g, e) ? __ldg((const uint32_t*)(g.base + e.x)) : 0u;
-    }
-    v = make_uint4(w[0], w[1], w[2], w[3]);
-  } else {
-    uint32_t w[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      uint32_t u = 0;
-#pragma unroll
-      for (int bq = 0; bq < 4; ++bq) {
-        const int2 e = tab[stage * 32 + half * 16 + q * 4 + bq];
-        if (tap_ok(g, e)) u |= (uint32_t)__ldg(g.base + e.x) << (8 * bq);
-      }
-      w[q] = u;
-    }
-    v = make_uint4(w[0], w[1], w[2], w[3]);
-  }
-  return v;
-}
-
-// 64 packed codes -> 16 tensor-memory columns of e4m3 bytes (column 4j+q holds
-// byte t = code 4t + q of the 16 codes in word j).
-__device__ __forceinline__ void expand_tmem_store(uint32_t taddr, uint4 v) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  uint32_t o[16];
-#pragma unroll
-  for (int j = 0; j < 4; ++j)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
-      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
-      "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
-      : "memory");
-}
 
 // GB: bytes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1 (cin % 4 == 0).
 template <int BN, int GB>
@@ -289,7 +155,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const int it = group + kGatherGroups * j;
           const int s = it % kStages;
           const uint32_t ph = (uint32_t)(it / kStages) & 1u;
-          if (!__all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u))) { ok = false; break; }
+          if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
           tc_fence_after();
           expand_tmem_store(tA + (uint32_t)(s * 32), lo);
           expand_tmem_store(tA + (uint32_t)(s * 32 + 16), hi);
@@ -313,7 +179,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       for (int k = 0; k < nk; ++k, ++it) {
         const int s = it % kStages;
         const uint32_t ph = (uint32_t)(it / kStages) & 1u;
-        if (!__all_sync(0xffffffffu, mbar_wait(empty(s), ph ^ 1u))) { ok = false; break; }
+        if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
         if (elect_one()) {
           mbar_arrive_expect_tx(full(s), (uint32_t)L::kB);
           tma_load_2d(sB + (uint32_t)(s * L::kB), &tmap_w, full(s), k * kBK, n0);
@@ -403,7 +269,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         named_bar(1, kEpiWarps * 32);
       }
       const int ab = jt & 1;
-      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(acc_full(ab), (uint32_t)(jt >> 1) & 1u));
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait_backoff(acc_full(ab), (uint32_t)(jt >> 1) & 1u, 64));
       if (!ok) continue;
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);

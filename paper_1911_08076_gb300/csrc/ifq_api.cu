@@ -12,11 +12,13 @@
 #include <mutex>
 #include <algorithm>
 #include <utility>
+#include <vector>
 
 #include "conv_bitserial.cuh"
 #include "conv_tc.cuh"
 #include "ifq.h"
 #include "pool_pack.cuh"
+#include "stack_tc.cuh"
 
 namespace {
 
@@ -105,12 +107,13 @@ cudaError_t set_attrs_gb() {
 struct DevState {
   bool init = false;
   int nsm = 0;
+  bool stack_ok = false;   // the stack kernel fits one CTA per SM (cooperative launch possible)
 };
 DevState g_dev[kMaxDevices];
 std::mutex g_dev_mu;
 
 // Per-device one-time setup (shared-memory limits of the kernels, SM count).
-int ensure_init(int* nsm_out) {
+int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return IFQ_ECUDA;
   std::lock_guard<std::mutex> lk(g_dev_mu);
@@ -119,9 +122,19 @@ int ensure_init(int* nsm_out) {
     if (set_attrs_gb<16>() != cudaSuccess || set_attrs_gb<4>() != cudaSuccess || set_attrs_gb<1>() != cudaSuccess)
       return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
+    if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
+        cudaSuccess)
+      return IFQ_ECUDA;
+    int per_sm = 0, coop = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, conv_stack_kernel, kStackThreads, StackSmem::bytes) !=
+        cudaSuccess)
+      return IFQ_ECUDA;
+    if (cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev) != cudaSuccess) return IFQ_ECUDA;
+    d.stack_ok = per_sm >= 1 && coop != 0;
     d.init = true;
   }
   if (nsm_out) *nsm_out = d.nsm;
+  if (stack_ok) *stack_ok = d.stack_ok;
   return IFQ_OK;
 }
 
@@ -225,6 +238,41 @@ bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
   return span < (1LL << 31);
 }
 
+// Bytes of packed codes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1.
+int granule_bytes(const ifq_conv_desc* d) { return d->cin % 64 == 0 ? 16 : (d->cin % 16 == 0 ? 4 : 1); }
+
+// TMA descriptor of the prepared e4m3 filter rows: [cout][Kpad] bytes, box 128 x bn, 128B swizzle.
+bool encode_wmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, int bn, CUtensorMap* tm) {
+  if (!get_encode()) return false;
+  cuuint64_t gdim[2] = {(cuuint64_t)g.Kpad, (cuuint64_t)d->cout};
+  cuuint64_t gstride[1] = {(cuuint64_t)g.Kpad};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)bn};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(w_prep), gdim, gstride, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const void* x, const int32_t* thr,
+                    const int8_t* sign, uint8_t* yc, int32_t* ya, ConvArgs* a) {
+  a->x = (const uint8_t*)x;
+  a->thr = thr;
+  a->sign = sign;
+  a->y_codes = yc;
+  a->y_acc = ya;
+  a->n = d->n; a->h = d->h; a->w = d->w; a->cin = d->cin; a->cout = d->cout;
+  a->kh = d->kh; a->kw = d->kw; a->stride = d->stride; a->pad = d->pad; a->ho = g.ho; a->wo = g.wo;
+  a->M = g.M;
+  a->K = g.K;
+  a->nk = g.Kpad / kBK;
+  a->nt = ceil_div(d->cout, bn);
+  a->ntiles = ceil_div(g.M, kBM) * a->nt;
+  a->ntab = g.Kpad / (4 * granule_bytes(d));
+  a->div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
+  a->div_wo = make_fastdiv((uint32_t)g.wo);
+  a->div_nt = make_fastdiv((uint32_t)a->nt);
+}
+
 int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
              void* y_codes, int32_t* y_acc, cudaStream_t st) {
   ConvGeom g;
@@ -242,37 +290,14 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   const int path = choose_path(d, g);
   cudaError_t e;
   if (path == IFQ_PATH_TC) {
-    if (!get_encode()) return IFQ_ECUDA;
     const int bn = choose_bn(g, d->cout, nsm);
     CUtensorMap tm;
-    cuuint64_t gdim[2] = {(cuuint64_t)g.Kpad, (cuuint64_t)d->cout};
-    cuuint64_t gstride[1] = {(cuuint64_t)g.Kpad};
-    cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)bn};
-    cuuint32_t estr[2] = {1, 1};
-    if (g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(w_prep), gdim, gstride, box, estr,
-                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return IFQ_ECUDA;
+    if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
     ConvArgs a;
-    a.x = (const uint8_t*)x;
-    a.thr = thr;
-    a.sign = sign;
-    a.y_codes = yc;
-    a.y_acc = ya;
-    a.n = d->n; a.h = d->h; a.w = d->w; a.cin = d->cin; a.cout = d->cout;
-    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad; a.ho = g.ho; a.wo = g.wo;
-    a.M = g.M;
-    a.K = g.K;
-    a.nk = g.Kpad / kBK;
-    a.nt = ceil_div(d->cout, bn);
-    a.ntiles = ceil_div(g.M, kBM) * a.nt;
-    const int gran = d->cin % 64 == 0 ? 64 : (d->cin % 16 == 0 ? 16 : 4);
-    a.ntab = g.Kpad / gran;
-    a.div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
-    a.div_wo = make_fastdiv((uint32_t)g.wo);
-    a.div_nt = make_fastdiv((uint32_t)a.nt);
-    if (gran == 64) e = launch_tc_gb<16>(bn, tm, a, nsm, st);
-    else if (gran == 16) e = launch_tc_gb<4>(bn, tm, a, nsm, st);
+    fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
+    const int gb = granule_bytes(d);
+    if (gb == 16) e = launch_tc_gb<16>(bn, tm, a, nsm, st);
+    else if (gb == 4) e = launch_tc_gb<4>(bn, tm, a, nsm, st);
     else e = launch_tc_gb<1>(bn, tm, a, nsm, st);
   } else {
     BsArgs a;
@@ -377,6 +402,135 @@ int check_stack(const ifq_layer* layers, int nlayers, const void* x) {
   return IFQ_OK;
 }
 
+// Completion counters of the persistent stack kernel: one per 128-row block of every layer.
+size_t stack_counters(const ifq_layer* layers, int nlayers) {
+  size_t n = 0;
+  for (int i = 0; i < nlayers; ++i) {
+    ConvGeom g;
+    check_conv(&layers[i].conv, &g);
+    n += (size_t)ceil_div(g.M, kBM);
+  }
+  return n;
+}
+
+// Whether a (validated) stack can run as one persistent launch: conv layers only, each on the
+// tensor-core path, at most kMaxStackLayers, K tables that fit in shared memory.  `bytes` gets
+// the workspace it needs (the completion counters).
+bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
+  if (nlayers < 1 || nlayers > kMaxStackLayers) return false;
+  int tab = 0;
+  for (int i = 0; i < nlayers; ++i) {
+    if (layers[i].kind != IFQ_LAYER_CONV) return false;
+    ConvGeom g;
+    if (check_conv(&layers[i].conv, &g)) return false;
+    if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
+    tab += g.Kpad / (4 * granule_bytes(&layers[i].conv));
+  }
+  if (tab > kMaxStackTab) return false;
+  if (bytes) *bytes = round_up(stack_counters(layers, nlayers) * sizeof(unsigned int), 256);
+  return true;
+}
+
+// The persistent stack kernel is opt-in (IFQ_STACK=1, read on every call): on the stacks
+// measured so far one launch per layer, chained with programmatic dependent launch, is faster.
+bool stack_enabled() {
+  const char* v = getenv("IFQ_STACK");
+  return v && v[0] == '1';
+}
+
+// The persistent stack kernel orders a layer only after the layer it reads, so it needs every
+// buffer a layer writes to be disjoint from every other buffer of the stack (input, weights,
+// thresholds, signs, other outputs, counters).  Stacks that reuse buffers run layer by layer,
+// where stream order makes reuse safe.
+struct Span { uintptr_t lo, hi; bool written; };
+
+bool stack_buffers_disjoint(const ifq_layer* layers, int nlayers, const void* x, const void* ws, size_t ws_bytes) {
+  std::vector<Span> v;
+  auto add = [&](const void* p, size_t n, bool wr) {
+    if (p && n) v.push_back({(uintptr_t)p, (uintptr_t)p + n, wr});
+  };
+  size_t x_bytes = 0;
+  for (int i = 0; i < nlayers; ++i)
+    if (layers[i].src < 0) {
+      const ifq_conv_desc& d = layers[i].conv;
+      x_bytes = std::max(x_bytes, (size_t)d.n * d.h * d.w * d.cin / 4);
+    }
+  add(x, x_bytes, false);
+  add(ws, ws_bytes, true);
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_conv_desc& d = layers[i].conv;
+    ConvGeom g;
+    check_conv(&d, &g);
+    const size_t rows = (size_t)d.n * g.ho * g.wo;
+    add(layers[i].w_prep, prep_bits_offset(&d, g) + (size_t)d.cout * g.kwords * 4, false);
+    if (d.out_mode & IFQ_OUT_CODES) {
+      add(layers[i].thr, (size_t)d.cout * 3 * 4, false);
+      add(layers[i].sign, (size_t)d.cout, false);
+      add(layers[i].y_codes, rows * d.cout / 4, true);
+    }
+    if (d.out_mode & IFQ_OUT_ACC) add(layers[i].y_acc, rows * d.cout * 4, true);
+  }
+  for (size_t i = 0; i < v.size(); ++i)
+    for (size_t j = i + 1; j < v.size(); ++j)
+      if ((v[i].written || v[j].written) && v[i].lo < v[j].hi && v[j].lo < v[i].hi) return false;
+  return true;
+}
+
+int run_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes,
+                     cudaStream_t st) {
+  size_t need = 0;
+  if (!stack_enabled() || !stack_eligible(layers, nlayers, &need) || !ws || ws_bytes < need) return IFQ_EUNSUPPORTED;
+  int nsm = 0;
+  bool ok = false;
+  int rc = ensure_init(&nsm, &ok);
+  if (rc) return rc;
+  if (!ok) return IFQ_EUNSUPPORTED;
+  if (!stack_buffers_disjoint(layers, nlayers, x, ws, need)) return IFQ_EUNSUPPORTED;
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_layer& l = layers[i];
+    const void* in = l.src < 0 ? x : layers[l.src].y_codes;
+    if (!in || !l.w_prep || !aligned16(in) || !aligned16(l.w_prep)) return IFQ_EUNSUPPORTED;
+    if ((l.conv.out_mode & IFQ_OUT_CODES) && (!l.y_codes || !l.thr || !l.sign || !aligned16(l.y_codes)))
+      return IFQ_EUNSUPPORTED;
+    if ((l.conv.out_mode & IFQ_OUT_ACC) && (!l.y_acc || !aligned16(l.y_acc))) return IFQ_EUNSUPPORTED;
+  }
+  StackParams P;
+  memset(&P, 0, sizeof(P));
+  P.nlayers = nlayers;
+  P.cnt = (unsigned int*)ws;
+  int tab = 0, cnt = 0;
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_layer& l = layers[i];
+    ConvGeom g;
+    check_conv(&l.conv, &g);
+    const int bn = choose_bn(g, l.conv.cout, nsm);
+    if (!encode_wmap(&l.conv, g, l.w_prep, bn, &P.tm[i])) return IFQ_ECUDA;
+    uint8_t* yc = (l.conv.out_mode & IFQ_OUT_CODES) ? (uint8_t*)l.y_codes : nullptr;
+    int32_t* ya = (l.conv.out_mode & IFQ_OUT_ACC) ? l.y_acc : nullptr;
+    StackLayer& S = P.L[i];
+    fill_conv_args(&l.conv, g, bn, l.src < 0 ? x : layers[l.src].y_codes, l.thr, l.sign, yc, ya, &S.a);
+    S.bn = bn;
+    S.gb = granule_bytes(&l.conv);
+    S.tab_off = tab;
+    S.dep = l.src;
+    S.cnt_off = cnt;
+    tab += S.a.ntab;
+    cnt += ceil_div(g.M, kBM);
+  }
+  if (cudaMemsetAsync(ws, 0, need, st) != cudaSuccess) return IFQ_ECUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(nsm);
+  cfg.blockDim = dim3(kStackThreads);
+  cfg.dynamicSmemBytes = StackSmem::bytes;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeCooperative;
+  at[0].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, conv_stack_kernel, P) == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
 int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t st) {
   for (int i = 0; i < nlayers; ++i) {
     const ifq_layer& l = layers[i];
@@ -446,15 +600,16 @@ int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, v
 
 int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* bytes) {
   if (!layers || nlayers < 1 || !bytes) return IFQ_EINVAL;
-  *bytes = 0;
+  size_t need = 0;
+  *bytes = stack_enabled() && stack_eligible(layers, nlayers, &need) ? need : 0;
   return IFQ_OK;
 }
 
 int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream) {
-  (void)ws;
-  (void)ws_bytes;
   int rc = check_stack(layers, nlayers, x);
   if (rc) return rc;
+  rc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, S(stream));
+  if (rc != IFQ_EUNSUPPORTED) return rc;
   return run_stack(layers, nlayers, x, S(stream));
 }
 

@@ -55,6 +55,34 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return false;
 }
 
+// mbar_wait for waiters off the critical path (producers waiting for a free
+// ring slot, epilogue warps waiting for an accumulator): after a failed poll
+// the thread sleeps `ns` nanoseconds before polling again, so a dozen waiting
+// warps do not flood the shared-memory pipe with barrier polls that the
+// working warps' loads queue behind.
+__device__ __forceinline__ bool mbar_wait_backoff(uint32_t bar, uint32_t parity, uint32_t ns) {
+  if (mbar_try(bar, parity)) return true;
+  const unsigned long long t0 = global_ns();
+  for (uint32_t it = 1; it < kWaitLimit; ++it) {
+    __nanosleep(ns);
+    if (mbar_try(bar, parity)) return true;
+    if ((it & 15u) == 0 && global_ns() - t0 > kWaitNs) break;
+  }
+  set_status(IFQ_ETIMEOUT);
+  return false;
+}
+
+// Non-blocking check that the phase with the given parity has completed.
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{.reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p;}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // One lane of a converged warp, chosen by the hardware (all 32 lanes must execute this).
 __device__ __forceinline__ bool elect_one() {
   uint32_t pred;

@@ -153,3 +153,22 @@ def test_stack_validation_rejects_broken_chains():
     with pytest.raises(ifq.IfqError) as e:
         ifq.ifq_forward([L3, L4], fake, stream=0)
     assert e.value.status == ifq.IFQ_ESHAPE
+
+
+def test_forward_workspace_is_counters_only_for_the_persistent_launch(monkeypatch):
+    """ifq_forward_workspace_bytes: 0 for the default per-layer launches; with IFQ_STACK=1, one
+    4-byte completion counter per 128-output-row block of every layer, rounded up to 256 bytes."""
+    fake = 1 << 20
+    descs = [ifq.conv_desc(3, 20, 20, 64, 64, 3, 1, 1), ifq.conv_desc(3, 20, 20, 64, 128, 3, 2, 1),
+             ifq.conv_desc(3, 10, 10, 128, 128, 1, 1, 0)]
+    layers = [ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=i - 1, conv=d, w_prep=fake, thr=fake, sign=fake, y_codes=fake)
+              for i, d in enumerate(descs)]
+    monkeypatch.delenv("IFQ_STACK", raising=False)
+    assert ifq.ifq_forward_workspace_bytes(layers) == 0
+    monkeypatch.setenv("IFQ_STACK", "1")
+    rows = [3 * 20 * 20, 3 * 10 * 10, 3 * 10 * 10]
+    blocks = sum((m + 127) // 128 for m in rows)
+    assert ifq.ifq_forward_workspace_bytes(layers) == (4 * blocks + 255) // 256 * 256
+    # a pooling layer keeps the stack on per-layer launches
+    pool = ifq.Layer(kind=ifq.IFQ_LAYER_POOL, src=2, pool=ifq.PoolDesc(3, 10, 10, 128, 2, 2, 0), y_codes=fake)
+    assert ifq.ifq_forward_workspace_bytes(layers + [pool]) == 0

@@ -234,10 +234,13 @@ def test_workload_matches_oracle(name):
             assert (synth.unpack_codes(out["codes"][imgs], c) == r).all(), l.name
 
 
-def test_graph_replay_equals_forward():
+@pytest.mark.parametrize("persistent", ["0", "1"], ids=["per_layer", "persistent"])
+def test_graph_replay_equals_forward(persistent, monkeypatch):
+    monkeypatch.setenv("IFQ_STACK", persistent)
     wl = synth.get("resnet18", batch=3)
     x, params = synth.draw_workload(wl)
     st = DeviceStack(wl, params)
+    assert (st.ws_bytes > 0) == (persistent == "1")
     xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
     st.forward(xd)
     torch.cuda.synchronize()
@@ -253,3 +256,71 @@ def test_graph_replay_equals_forward():
             assert (v == direct[li][k]).all()
     st.release()
     assert ifq.ifq_device_status() == ifq.IFQ_OK
+
+
+def _stack_outputs(st):
+    return {li: {k: v.copy() for k, v in st.output(li).items()} for li in range(len(st.wl.layers))}
+
+
+@pytest.mark.parametrize("name", ["resnet18", "custom"])
+def test_persistent_stack_kernel_equals_per_layer_launches(name, monkeypatch):
+    """With IFQ_STACK=1 and its workspace, ifq_forward runs the whole conv stack as one persistent
+    launch; without a workspace it launches layer by layer.  Both must give identical codes and
+    accumulators, and the oracle must agree on sampled images."""
+    monkeypatch.setenv("IFQ_STACK", "1")
+    if name == "resnet18":
+        wl = synth.get("resnet18", batch=6)
+    else:
+        L = [synth.Conv("a", 16, 48, 3, 1, 1, 11, 11, 11, 11, -1),
+             synth.Conv("b", 48, 64, 1, 2, 0, 11, 11, 6, 6, 0),
+             synth.Conv("c", 48, 96, 3, 2, 1, 11, 11, 6, 6, 0, "both"),      # second reader of layer 0
+             synth.Conv("d", 96, 256, 3, 1, 1, 6, 6, 6, 6, 2),
+             synth.Conv("e", 256, 30, 1, 1, 0, 6, 6, 6, 6, 3, "acc")]
+        wl = synth.Workload("custom_stack", 7, 5, 11, 11, 16, L)
+    x, params = synth.draw_workload(wl)
+    st = DeviceStack(wl, params)
+    assert st.ws_bytes > 0, "the stack should qualify for the persistent kernel"
+    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    st.forward(xd)
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    fused = _stack_outputs(st)
+    for t in list(st.y_codes.values()) + list(st.y_acc.values()):
+        t.zero_()
+    ifq.ifq_forward(st.layers, xd)          # no workspace: one launch per layer
+    torch.cuda.synchronize()
+    per_layer = _stack_outputs(st)
+    for li in fused:
+        for k in fused[li]:
+            assert (fused[li][k] == per_layer[li][k]).all(), (wl.layers[li].name, k)
+    ref = O.forward(wl, x, params, images=[0, wl.batch - 1])
+    for li, l in enumerate(wl.layers):
+        out, r = fused[li], ref[li]
+        if l.out == "both":
+            assert (synth.unpack_codes(out["codes"][[0, -1]], l.cout) == r["codes"]).all()
+            assert (out["acc"][[0, -1]] == r["acc"]).all()
+        elif l.out == "acc":
+            assert (out["acc"][[0, -1]] == r).all()
+        else:
+            assert (synth.unpack_codes(out["codes"][[0, -1]], l.cout) == r).all(), l.name
+
+
+def test_stack_with_reused_output_buffer_runs_layer_by_layer(monkeypatch):
+    """A stack whose third layer writes into the first layer's output buffer (ping-pong reuse)
+    must not run as one persistent launch (layers there are ordered only after their source);
+    ifq_forward falls back to one launch per layer and the results follow stream order."""
+    monkeypatch.setenv("IFQ_STACK", "1")
+    L = [synth.Conv("a", 16, 64, 3, 1, 1, 9, 9, 9, 9, -1),
+         synth.Conv("b", 64, 64, 3, 1, 1, 9, 9, 9, 9, 0),
+         synth.Conv("c", 64, 64, 3, 1, 1, 9, 9, 9, 9, 1)]
+    wl = synth.Workload("pingpong", 3, 3, 9, 9, 16, L)
+    x, params = synth.draw_workload(wl)
+    st = DeviceStack(wl, params)
+    st.layers[2].y_codes = st.layers[0].y_codes          # c overwrites a's codes after b has read them
+    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    st.forward(xd)
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    ref = O.forward(wl, x, params, images=[0, 1, 2])
+    assert (synth.unpack_codes(st.y_codes[1].cpu().numpy(), 64) == ref[1]).all()
+    assert (synth.unpack_codes(st.y_codes[0].cpu().numpy(), 64) == ref[2]).all()
