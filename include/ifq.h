@@ -227,6 +227,27 @@ int ifq_forward_workspace_bytes(const ifq_layer* layers, int nlayers, size_t* by
 int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * ifq_forward_noalloc -- ifq_forward for callers that cannot hand the library
+ * device scratch: a plain C host that owns no device allocator, or a serving
+ * loop that must not call cudaMalloc (which can synchronize the whole device).
+ * The paper has no counterpart; this is a deployment convenience.  It
+ * allocates nothing.  A stack that qualifies for the persistent launch (see
+ * ifq_forward; IFQ_STACK is not consulted) keeps that launch's completion
+ * counters in a file-scope device array of 256 KiB: 65536 counters, one per
+ * 128-output-row block of every layer.  A stack that needs more counters is
+ * rejected with IFQ_EWORKSPACE before anything is launched.  The counters
+ * must be zero when the kernel starts: every call zeroes the part it uses, on
+ * `stream`, before the launch.  Other stacks run one launch per layer, which
+ * needs no scratch.  The first call on each device looks up the array's device
+ * address (cudaGetSymbolAddress with that device current, no allocation) and
+ * should come before any stream capture.  All calls on one device share the
+ * array, so calls whose executions overlap in time (on other streams or from
+ * other host threads) race on it and must be serialised by the caller.
+ * Results are identical to ifq_forward's.
+ */
+int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, void* stream);
+
+/*
  * CUDA-graph form of ifq_forward: ifq_graph_create captures the launches of
  * ifq_forward(layers, nlayers, x, ws, ws_bytes) on `stream` into a graph that
  * ifq_graph_launch replays on any stream with the same buffers.  The graph is

@@ -476,10 +476,19 @@ bool stack_buffers_disjoint(const ifq_layer* layers, int nlayers, const void* x,
   return true;
 }
 
+int launch_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t need,
+                        cudaStream_t st);
+
 int run_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes,
                      cudaStream_t st) {
   size_t need = 0;
   if (!stack_enabled() || !stack_eligible(layers, nlayers, &need) || !ws || ws_bytes < need) return IFQ_EUNSUPPORTED;
+  return launch_stack_kernel(layers, nlayers, x, ws, need, st);
+}
+
+// The launch itself, for an eligible stack with `need` bytes of counters at ws.
+int launch_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t need,
+                        cudaStream_t st) {
   int nsm = 0;
   bool ok = false;
   int rc = ensure_init(&nsm, &ok);
@@ -529,6 +538,30 @@ int run_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, void* 
   cfg.attrs = at;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, conv_stack_kernel, P) == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+// Counter scratch of ifq_forward_noalloc.  That entry point serves callers that cannot hand
+// the library device scratch (a plain C host without a device allocator, or a serving loop that
+// must not call cudaMalloc, which can synchronize the whole device), so its counters live in a
+// file-scope device array instead of a caller's workspace: 65536 counters, one per 128-row
+// output block, enough for the ResNet-18 body at batch 256.
+constexpr size_t kNoallocCounterBytes = 256 * 1024;
+static __device__ __align__(256) unsigned int g_noalloc_counters[kNoallocCounterBytes / sizeof(unsigned int)];
+void* g_noalloc_addr[kMaxDevices];   // device address of g_noalloc_counters per device (g_dev_mu)
+
+// Device address of the counter array on the current device: looked up once per device, with
+// that device current (cudaGetSymbolAddress allocates nothing).
+int noalloc_counters(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return IFQ_ECUDA;
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  if (!g_noalloc_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_counters) != cudaSuccess || !p) return IFQ_ECUDA;
+    g_noalloc_addr[dev] = p;
+  }
+  *out = g_noalloc_addr[dev];
+  return IFQ_OK;
 }
 
 int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t st) {
@@ -609,6 +642,19 @@ int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, s
   int rc = check_stack(layers, nlayers, x);
   if (rc) return rc;
   rc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, S(stream));
+  if (rc != IFQ_EUNSUPPORTED) return rc;
+  return run_stack(layers, nlayers, x, S(stream));
+}
+
+int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, void* stream) {
+  int rc = check_stack(layers, nlayers, x);
+  if (rc) return rc;
+  size_t need = 0;
+  if (!stack_eligible(layers, nlayers, &need)) return run_stack(layers, nlayers, x, S(stream));
+  if (need > kNoallocCounterBytes) return IFQ_EWORKSPACE;
+  void* ws = nullptr;
+  if ((rc = noalloc_counters(&ws))) return rc;
+  rc = launch_stack_kernel(layers, nlayers, x, ws, need, S(stream));
   if (rc != IFQ_EUNSUPPORTED) return rc;
   return run_stack(layers, nlayers, x, S(stream));
 }

@@ -65,6 +65,7 @@ _SIGS = {
     "ifq_maxpool2bit": ([ctypes.POINTER(PoolDesc), _P, _P, _P, _P], _I),
     "ifq_forward_workspace_bytes": ([ctypes.POINTER(Layer), _I, ctypes.POINTER(_SZ)], _I),
     "ifq_forward": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P], _I),
+    "ifq_forward_noalloc": ([ctypes.POINTER(Layer), _I, _P, _P], _I),
     "ifq_graph_create": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, ctypes.POINTER(_P)], _I),
     "ifq_graph_launch": ([_P, _P], _I),
     "ifq_graph_destroy": ([_P], _I),
@@ -212,6 +213,11 @@ def ifq_forward_workspace_bytes(layers: Sequence[Layer]) -> int:
 def ifq_forward(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=None):
     arr, n = _layer_array(layers)
     _ok(lib().ifq_forward(arr, n, _ptr(x), _ptr(ws), ws_bytes, _stream(stream)), "ifq_forward")
+
+
+def ifq_forward_noalloc(layers: Sequence[Layer], x, stream=None):
+    arr, n = _layer_array(layers)
+    _ok(lib().ifq_forward_noalloc(arr, n, _ptr(x), _stream(stream)), "ifq_forward_noalloc")
 
 
 def ifq_graph_create(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=None) -> int:
