@@ -42,7 +42,7 @@ INT8_PEAK_TOPS = 151.4
 FP8_PER_BF16 = 2.0          # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK_BF16_TFLOPS = 1900.0
 PROFILE = os.path.join(ROOT, "profiles", "conv_tc_resnet18_b32.md")
-KERNEL_SRC = os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", "conv_tc.cuh")
+KERNEL_SRC = [os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", f) for f in ("conv_tc.cuh", "conv_common.cuh", "ptx.cuh")]
 
 
 def log(*a):
@@ -81,8 +81,12 @@ def read_peaks():
 
 
 def kernel_sha():
-    with open(KERNEL_SRC, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """Hash of the sources the conv kernel compiles from (a stale ncu summary must not be reused)."""
+    h = hashlib.sha256()
+    for path in KERNEL_SRC:
+        with open(path, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def profiled_traffic():
