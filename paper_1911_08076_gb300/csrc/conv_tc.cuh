@@ -31,13 +31,14 @@
 // the 128B-swizzled K-major layout.
 //
 // Persistent, warp-specialized CTA (one per SM), tiles of 128 output pixels x
-// BN output channels (BN <= 128) handed out round-robin; 26 warps:
+// BN output channels (BN <= 128) handed out round-robin; 27 warps:
 //   warps 0-15   gather, in 4 groups of 4 warps; group g fills the K stages
 //                g, g+4, g+8, ... so four stages are filled concurrently; warp
 //                w writes rows 32*(w%4)..+31 (the tensor-memory lanes it may
 //                access), all 128 K positions of the stage;
 //   warp 16      TMA producer of the prepared filter tile;
-//   warp 17      TMEM allocation and the tcgen05.mma issue (one elected lane);
+//   warps 17, 26 TMEM allocation (17) and the tcgen05.mma issue, alternate pairs of K
+//                stages each (one elected lane per warp);
 //   warps 18-25  epilogue: tcgen05.ld of the finished accumulator (two
 //                buffers, so it overlaps the next tile's mainloop), thresholds,
 //                2-bit packing, stores.
@@ -48,12 +49,26 @@
 
 namespace ifq {
 
+// A second MMA-issuing warp after the epilogue warps (27 warps in all).
+constexpr int kWarpMma2 = kWarpEpi0 + kEpiWarps;
+constexpr int kConvThreads = kTcThreads + 32;
+
+// 16 columns of zeros into tensor memory (this warp's 32 lanes).
+__device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
+  const uint32_t z = 0u;
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};" ::"r"(taddr),
+      "r"(z)
+      : "memory");
+}
+
 // GB: bytes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1 (cin % 4 == 0).
 template <int BN, int GB>
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kConvThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
   static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
   using L = TcSmem<BN>;
+  constexpr int kS = kStages;
   extern __shared__ uint8_t smem_raw_[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
@@ -64,10 +79,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // full[s]: the arrivals of the 4 warps of the gather group that owns stage s, plus
   // the TMA producer's (with the B bytes)
   auto full = [&](int s) { return barBase + 8u * s; };
-  auto empty = [&](int s) { return barBase + 8u * (kStages + s); };
-  auto acc_full = [&](int b) { return barBase + 8u * (2 * kStages + b); };
-  auto acc_empty = [&](int b) { return barBase + 8u * (2 * kStages + 2 + b); };
-  const uint32_t done_bar = barBase + 8u * (2 * kStages + 4);
+  auto empty = [&](int s) { return barBase + 8u * (kS + s); };
+  auto acc_full = [&](int b) { return barBase + 8u * (2 * kS + b); };
+  auto acc_empty = [&](int b) { return barBase + 8u * (2 * kS + 2 + b); };
+  const uint32_t done_bar = barBase + 8u * (2 * kS + 4);
   uint32_t* tmem_slot = (uint32_t*)(smem + L::offTmem);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -82,15 +97,15 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tmem_relinquish();
   }
   if (tid == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kS; ++s) {
       mbar_init(full(s), 4 + 1);   // one gather group (4 warps) + the TMA producer
       mbar_init(empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(acc_full(b), 1);
-      mbar_init(acc_empty(b), kEpiWarps);
+      mbar_init(acc_full(b), 2);           // one commit from each MMA warp
+      mbar_init(acc_empty(b), kEpiWarps);  // drained and zeroed by every epilogue warp
     }
-    mbar_init(done_bar, 1);
+    mbar_init(done_bar, 2);
     fence_mbar_init();
   }
   if (warp == kWarpTma && lane == 0) prefetch_tmap(&tmap_w);
@@ -98,7 +113,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   // pointer, and its tap (dy, dx); dy = 0xFF past K.
   {
     const int cinb = args.cin >> 2;
-    for (int gk = tid; gk < args.ntab; gk += kTcThreads) {
+    for (int gk = tid; gk < args.ntab; gk += kConvThreads) {
       const int k0 = gk * 4 * GB;
       const int tap = k0 / args.cin, cc = k0 - tap * args.cin;
       int2 e = make_int2(0, 0xFF << 8);
@@ -153,8 +168,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const uint4 lo = ring_lo[d], hi = ring_hi[d];
           if (j + kAhead < own) next_load(ring_lo[d], ring_hi[d]);
           const int it = group + kGatherGroups * j;
-          const int s = it % kStages;
-          const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+          const int s = it % kS;
+          const uint32_t ph = (uint32_t)(it / kS) & 1u;
           if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
           tc_fence_after();
           expand_tmem_store(tA + (uint32_t)(s * 32), lo);
@@ -177,8 +192,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       const int n0 = (t - (int)fdiv((uint32_t)t, args.div_nt) * args.nt) * BN;
 #pragma unroll 1
       for (int k = 0; k < nk; ++k, ++it) {
-        const int s = it % kStages;
-        const uint32_t ph = (uint32_t)(it / kStages) & 1u;
+        const int s = it % kS;
+        const uint32_t ph = (uint32_t)(it / kS) & 1u;
         if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
         if (elect_one()) {
           mbar_arrive_expect_tx(full(s), (uint32_t)L::kB);
@@ -190,28 +205,37 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     // drain: every load issued into a slot has landed before the CTA may exit
     // (full(s) completes only when the gather warps and the bytes have arrived)
     if (!ok) {
-      for (int i = it - kStages < 0 ? 0 : it - kStages; i < it; ++i)
-        mbar_wait(full(i % kStages), (uint32_t)(i / kStages) & 1u);
+      for (int i = it - kS < 0 ? 0 : it - kS; i < it; ++i)
+        mbar_wait(full(i % kS), (uint32_t)(i / kS) & 1u);
     }
     __syncwarp();
-  } else if (warp == kWarpMma) {
+  } else if (warp == kWarpMma || warp == kWarpMma2) {
     // =================== MMA issue ===================
-    // the whole warp runs the loop; one elected lane issues the MMAs and commits
+    // Two MMA warps take alternate pairs of K stages of every tile into the same accumulator:
+    // one thread issuing tcgen05.mma costs more per instruction than an N <= 128 MMA takes on
+    // the tensor pipe.  Every MMA accumulates into a buffer that
+    // the epilogue left zeroed, so the order of the two warps' MMAs does not matter (the fp32
+    // sums are exact integers in any order).  Each warp runs its loop uniformly; one elected
+    // lane issues and commits.
+    const int mi = warp == kWarpMma2 ? 1 : 0;
     constexpr uint32_t idesc = idesc_e4m3_f32(kBM, BN);
-    int it = 0;
+    int gp = 0;   // pairs of K stages seen so far (pairs alternate between the two warps)
     bool ok = true;
 #pragma unroll 1
     for (int jt = 0; jt < n_local && ok; ++jt) {
       const int ab = jt & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait(acc_empty(ab), ((uint32_t)(jt >> 1) & 1u) ^ 1u))) break;
+      // buffer ab is zero once the epilogue has drained it (phase 0: the zeroing at start)
+      if (!__all_sync(0xffffffffu, mbar_wait(acc_empty(ab), (uint32_t)(jt >> 1) & 1u))) break;
       tc_fence_after();
       const uint32_t dacc = tmem + (uint32_t)(ab * BN);
-      // two K stages per round: one vote, fence and elect for 8 MMAs
+      // stages k, k+1 of this tile (one vote, fence and elect for up to 8 MMAs)
 #pragma unroll 1
-      for (int k = 0; k < nk; k += 2, it += 2) {
+      for (int k = 0; k < nk; k += 2, ++gp) {
+        if ((gp & 1) != mi) continue;
         const bool two = k + 1 < nk;
-        const int s0 = it % kStages, s1 = (it + 1) % kStages;
-        const uint32_t ph0 = (uint32_t)(it / kStages) & 1u, ph1 = (uint32_t)((it + 1) / kStages) & 1u;
+        const int it = jt * nk + k;   // position in the CTA's stage sequence
+        const int s0 = it % kS, s1 = (it + 1) % kS;
+        const uint32_t ph0 = (uint32_t)(it / kS) & 1u, ph1 = (uint32_t)((it + 1) / kS) & 1u;
         bool got = mbar_wait(full(s0), ph0);
         if (two) got = got && mbar_wait(full(s1), ph1);
         if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
@@ -220,7 +244,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           const uint32_t a0 = tmem + (uint32_t)(kTmemA + s0 * 32), b0 = sB + (uint32_t)(s0 * L::kB);
 #pragma unroll
           for (int kk = 0; kk < kBK / 32; ++kk)
-            mma_e4m3_tmem_a(dacc, a0 + (uint32_t)(8 * kk), sdesc_sw128(b0 + 32 * kk), idesc, (k | kk) != 0 ? 1u : 0u);
+            mma_e4m3_tmem_a(dacc, a0 + (uint32_t)(8 * kk), sdesc_sw128(b0 + 32 * kk), idesc, 1u);
           mma_commit(empty(s0));
           if (two) {
             const uint32_t a1 = tmem + (uint32_t)(kTmemA + s1 * 32), b1 = sB + (uint32_t)(s1 * L::kB);
@@ -232,11 +256,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
         __syncwarp();
       }
-      if (nk & 1) it -= 1;   // the last round covered a single stage
       if (ok && elect_one()) mma_commit(acc_full(ab));
       __syncwarp();
     }
-    if (elect_one()) mma_commit(done_bar);   // fires once every MMA issued above has completed
+    if (elect_one()) mma_commit(done_bar);   // fires once every MMA this warp issued has completed
     __syncwarp();
   } else {
     // =================== epilogue ===================
@@ -248,6 +271,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     const int c_lo = (e >> 2) * CW;
     const int row = quarter * 32 + lane;
     bool ok = true;   // after a timed-out wait, keep only the named barriers (uniform over the 8 warps)
+    // both accumulator buffers start at zero: every MMA accumulates
+    {
+      const uint32_t tz = tmem + (uint32_t)c_lo + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll
+      for (int b2 = 0; b2 < 2; ++b2)
+#pragma unroll
+        for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16(tz + (uint32_t)(b2 * BN + c0));
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(acc_empty(0));
+        mbar_arrive(acc_empty(1));
+      }
+    }
 #pragma unroll 1
     for (int jt = 0; jt < n_local; ++jt) {
       const int t = (int)blockIdx.x + jt * G;
@@ -311,7 +349,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
         }
       }
-      // the accumulator buffer may be refilled once every epilogue warp has read it
+      // the accumulator buffer may be refilled once every epilogue warp has read and zeroed it
+#pragma unroll
+      for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16(tacc + c0);
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty(ab));

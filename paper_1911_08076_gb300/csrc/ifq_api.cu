@@ -87,7 +87,7 @@ struct TcInst {
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
     const int grid = a.ntiles < nsm ? a.ntiles : nsm;
-    return launch_k(conv_tc_kernel<BN, GB>, dim3(grid), dim3(kTcThreads), (size_t)L::bytes, st, tm, a);
+    return launch_k(conv_tc_kernel<BN, GB>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
   }
 };
 
