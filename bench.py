@@ -60,11 +60,12 @@ def conv_ops(layer, batch):
 
 def alg_bytes(layer, batch):
     """Bytes the method must move for one conv launch: 2-bit input codes read once, 1-bit
-    filters, 13 B of thresholds+sign per channel, 2-bit output codes (int32 for accumulators)."""
+    filters, 13 B of thresholds+sign per channel, 2-bit output codes (int32 for accumulators),
+    after the fused pool when the launch has one."""
     inp = batch * layer.h * layer.w * layer.cin / 4
     wts = layer.cout * layer.k * layer.k * layer.cin / 8
     thr = 13 * layer.cout
-    out = batch * layer.ho * layer.wo * layer.cout
+    out = batch * layer.out_h * layer.out_w * layer.cout
     out = out / 4 if layer.out == "codes" else (out * 4 if layer.out == "acc" else out * 4.25)
     return inp + wts + thr + out
 

@@ -114,6 +114,12 @@ int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
  * IFQ_OUT_*; codes output needs cout % 4 == 0.  path selects a kernel path
  * (IFQ_PATH_AUTO lets the library choose).  Limits: all sizes >= 1,
  * K = kh*kw*cin <= 65536, cout <= 65536, n*ho*wo < 2^31.
+ * pool: 0 or 1 for none; p = 2 or 4 max-pools the convolution output over
+ * p x p windows with stride p before the thresholds (Sec. 2.1: the pool acts
+ * on Y^conv, before BN and the quantizer), so that the codes are those of the
+ * window maximum of A and the output is [n][ho/p][wo/p][cout].  Needs
+ * ho % p == 0, wo % p == 0, out_mode IFQ_OUT_CODES and the tensor-core path
+ * (IFQ_EUNSUPPORTED otherwise).
  */
 typedef struct {
   int n, h, w, cin;
@@ -121,10 +127,11 @@ typedef struct {
   int kh, kw, stride, pad;
   int out_mode;
   int path;
+  int pool;
 } ifq_conv_desc;
 
 /* Output spatial size of a conv descriptor (host, pure). */
-int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo);
+int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo);   /* after the pool, if any */
 
 /*
  * Size of the prepared-filter buffer that ifq_pack_weights fills for `d`

@@ -223,6 +223,8 @@ def forward(workload, x: np.ndarray, params: Sequence, images: Optional[Sequence
             if layer.kind == "conv":
                 p, T, s = folded[li]
                 A = conv_acc(src, params[li].w, layer.stride, layer.pad)
+                if getattr(layer, "pool", 0) > 1:   # pool on Y^conv, before BN and the quantizer (Sec. 2.1)
+                    A = maxpool_acc(A, layer.pool, layer.pool, 0)
                 if check_float:
                     codes, _ = check_chains(A, p, T, s)
                 else:

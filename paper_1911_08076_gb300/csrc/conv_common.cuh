@@ -34,6 +34,11 @@ struct ConvArgs {
   int ntiles;            // M tiles * nt
   int ntab;              // entries of the K-granule table (Kpad / codes per granule)
   FastDiv div_hw, div_wo, div_nt;   // by ho*wo, wo, nt
+  // Fused p x p / stride p pool (p = 1 << lpool, lpool = 0: none).  Tile rows are then ordered
+  // by pooled pixel and, within it, by window position (p*p consecutive rows, dy-major), so
+  // that a window's rows sit in consecutive lanes of one epilogue warp.
+  int lpool;
+  FastDiv div_phw, div_pwo;         // by (ho/p)*(wo/p), wo/p
 };
 
 constexpr int kBM = 128;         // output pixels per tile (MMA M)
@@ -78,8 +83,21 @@ __device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
   g.base = a.x;
   g.vy = g.vx = 0;
   if (m < a.M) {
-    const int b = (int)fdiv((uint32_t)m, a.div_hw), rem = m - b * a.ho * a.wo;
-    const int oy = (int)fdiv((uint32_t)rem, a.div_wo), ox = rem - oy * a.wo;
+    int b, oy, ox;
+    if (a.lpool == 0) {
+      b = (int)fdiv((uint32_t)m, a.div_hw);
+      const int rem = m - b * a.ho * a.wo;
+      oy = (int)fdiv((uint32_t)rem, a.div_wo);
+      ox = rem - oy * a.wo;
+    } else {   // row m = window position w of pooled pixel P
+      const int P = m >> (2 * a.lpool), wpos = m & ((1 << (2 * a.lpool)) - 1);
+      const int pwo = a.wo >> a.lpool;
+      b = (int)fdiv((uint32_t)P, a.div_phw);
+      const int rem = P - b * (a.ho >> a.lpool) * pwo;
+      const int py = (int)fdiv((uint32_t)rem, a.div_pwo), px = rem - py * pwo;
+      oy = (py << a.lpool) + (wpos >> a.lpool);
+      ox = (px << a.lpool) + (wpos & ((1 << a.lpool) - 1));
+    }
     const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
     g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * (a.cin >> 2);
     g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));

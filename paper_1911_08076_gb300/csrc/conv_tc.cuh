@@ -323,6 +323,44 @@ __global__ void __launch_bounds__(kConvThreads, 1)
             : "r"(tacc + c0)
             : "memory");
         tmem_ld_wait();
+        // Fused pool (Sec. 2.1: the pool acts on Y^conv, before BN and the quantizer): the window
+        // maximum of A over the window's consecutive lanes, then the thresholds.
+        if (args.lpool == 1) {
+          // 2x2: a reduce-scatter over the window's 4 lanes (columns 8 apart with lane ^ 2, then
+          // 4 apart with lane ^ 1) leaves this lane the maxima of 4 of the 16 columns,
+          // [sub, sub + 4); it thresholds those alone and stores their byte of codes
+          const bool h2 = (lane & 2) != 0, h1 = (lane & 1) != 0;
+          float a8[8], a4[4];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const float lo8 = __uint_as_float(v[j]), hi8 = __uint_as_float(v[j + 8]);
+            a8[j] = fmaxf(h2 ? hi8 : lo8, __shfl_xor_sync(0xffffffffu, h2 ? lo8 : hi8, 2));
+          }
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            a4[j] = fmaxf(h1 ? a8[j + 4] : a8[j], __shfl_xor_sync(0xffffffffu, h1 ? a8[j] : a8[j + 4], 1));
+          const int sub = (h2 ? 8 : 0) + (h1 ? 4 : 0);
+          uint32_t byte = 0;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const float4 tq = th[c0 + sub + j];
+            const float sv = a4[j] * tq.w;
+            byte |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
+          }
+          const int cabs = n0 + c_lo + c0 + sub;
+          if (args.y_codes && m < args.M && cabs < args.cout)
+            args.y_codes[(size_t)(m >> 2) * (args.cout >> 2) + (cabs >> 2)] = (uint8_t)byte;
+          continue;
+        }
+        if (args.lpool) {   // 4x4: every lane of the window gets the maxima of all 16 columns
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            float x = __uint_as_float(v[j]);
+            for (int off = 1; off < (1 << (2 * args.lpool)); off <<= 1)
+              x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, off));
+            v[j] = __float_as_uint(x);
+          }
+        }
         uint32_t wd = 0;
 #pragma unroll
         for (int j = 0; j < 16; ++j) {
@@ -356,10 +394,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty(ab));
-      if (args.y_codes && m < args.M) {
+      // (2x2 pools stored their codes above; with a 4x4 pool the first lane of each window stores
+      // the pooled pixel m >> 4)
+      const bool store = args.y_codes && m < args.M && args.lpool != 1 && (m & ((1 << (2 * args.lpool)) - 1)) == 0;
+      if (store) {
         const int rowb = args.cout >> 2;        // bytes per output pixel
         const int cb = n0 + c_lo;               // first channel of this thread
-        uint8_t* dst = args.y_codes + (size_t)m * rowb + (cb >> 2);
+        uint8_t* dst = args.y_codes + (size_t)(m >> (2 * args.lpool)) * rowb + (cb >> 2);
         if (cb + CW <= args.cout && CW >= 64 && (rowb & 15) == 0 && (cb & 63) == 0) {
 #pragma unroll
           for (int q = 0; q < CW / 64; ++q)

@@ -159,12 +159,17 @@ int env_int(const char* name, int dflt) {
 
 struct ConvGeom {
   int ho, wo, M, K, Kpad, kwords;
+  int pool, pho, pwo;   // fused pool window (1: none) and the output shape after it
 };
 
 int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if (!d) return IFQ_EINVAL;
-  int rc = ifq_conv_out_shape(d, &g->ho, &g->wo);
+  int rc = ifq_conv_out_shape(d, &g->pho, &g->pwo);   // output shape, after the fused pool if any
   if (rc) return rc;
+  g->pool = d->pool > 1 ? d->pool : 1;
+  g->ho = g->pho * g->pool;                            // the convolution's own output
+  g->wo = g->pwo * g->pool;
+  if (g->pool > 1 && d->out_mode != IFQ_OUT_CODES) return IFQ_EUNSUPPORTED;
   if (d->cin % 4 != 0) return IFQ_ESHAPE;
   if (d->out_mode < IFQ_OUT_CODES || d->out_mode > IFQ_OUT_BOTH) return IFQ_EINVAL;
   if ((d->out_mode & IFQ_OUT_CODES) && d->cout % 4 != 0) return IFQ_ESHAPE;
@@ -193,6 +198,8 @@ int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
     path = forced ? forced : IFQ_PATH_TC;
   }
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
+  // the fused pool exists on the tensor-core path only
+  if (g.pool > 1 && path != IFQ_PATH_TC) return -1;
   return path;
 }
 
@@ -271,6 +278,9 @@ void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const voi
   a->div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
   a->div_wo = make_fastdiv((uint32_t)g.wo);
   a->div_nt = make_fastdiv((uint32_t)a->nt);
+  a->lpool = g.pool == 4 ? 2 : (g.pool == 2 ? 1 : 0);
+  a->div_phw = make_fastdiv((uint32_t)(g.pho * g.pwo));
+  a->div_pwo = make_fastdiv((uint32_t)g.pwo);
 }
 
 int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
@@ -288,6 +298,7 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   uint8_t* yc = (d->out_mode & IFQ_OUT_CODES) ? (uint8_t*)y_codes : nullptr;
   int32_t* ya = (d->out_mode & IFQ_OUT_ACC) ? y_acc : nullptr;
   const int path = choose_path(d, g);
+  if (path < 0) return IFQ_EUNSUPPORTED;
   cudaError_t e;
   if (path == IFQ_PATH_TC) {
     const int bn = choose_bn(g, d->cout, nsm);
@@ -363,7 +374,7 @@ int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes) {
     ConvGeom g;
     int rc = check_conv(&l.conv, &g);
     if (rc) return rc;
-    *n = l.conv.n; *h = g.ho; *w = g.wo; *c = l.conv.cout;
+    *n = l.conv.n; *h = g.pho; *w = g.pwo; *c = l.conv.cout;
     *codes = (l.conv.out_mode & IFQ_OUT_CODES) != 0;
     return IFQ_OK;
   }
@@ -423,6 +434,7 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     if (layers[i].kind != IFQ_LAYER_CONV) return false;
     ConvGeom g;
     if (check_conv(&layers[i].conv, &g)) return false;
+    if (g.pool > 1) return false;   // the persistent kernel has no fused pool
     if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
     tab += g.Kpad / (4 * granule_bytes(&layers[i].conv));
   }
@@ -461,7 +473,7 @@ bool stack_buffers_disjoint(const ifq_layer* layers, int nlayers, const void* x,
     const ifq_conv_desc& d = layers[i].conv;
     ConvGeom g;
     check_conv(&d, &g);
-    const size_t rows = (size_t)d.n * g.ho * g.wo;
+    const size_t rows = (size_t)d.n * g.pho * g.pwo;
     add(layers[i].w_prep, prep_bits_offset(&d, g) + (size_t)d.cout * g.kwords * 4, false);
     if (d.out_mode & IFQ_OUT_CODES) {
       add(layers[i].thr, (size_t)d.cout * 3 * 4, false);

@@ -86,8 +86,17 @@ extern "C" int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo) {
     return IFQ_ESHAPE;
   const int a = d->h + 2 * d->pad - d->kh, b = d->w + 2 * d->pad - d->kw;
   if (a < 0 || b < 0) return IFQ_ESHAPE;
-  *ho = a / d->stride + 1;
-  *wo = b / d->stride + 1;
+  int oh = a / d->stride + 1, ow = b / d->stride + 1;
+  if (d->pool > 1) {   // fused p x p / stride p pool of the convolution output
+    if (d->pool != 2 && d->pool != 4) return IFQ_EUNSUPPORTED;
+    if (oh % d->pool != 0 || ow % d->pool != 0) return IFQ_ESHAPE;
+    oh /= d->pool;
+    ow /= d->pool;
+  } else if (d->pool < 0) {
+    return IFQ_EINVAL;
+  }
+  *ho = oh;
+  *wo = ow;
   return IFQ_OK;
 }
 

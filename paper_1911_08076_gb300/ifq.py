@@ -33,7 +33,7 @@ class IfqError(RuntimeError):
 
 class ConvDesc(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int) for f in
-                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path")]
+                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path", "pool")]
 
 
 class PoolDesc(ctypes.Structure):
@@ -156,8 +156,8 @@ def ifq_codes_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> int:
     return out.value
 
 
-def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None):
-    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path)
+def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None, pool=0):
+    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path, pool)
 
 
 def ifq_conv_out_shape(d: ConvDesc):

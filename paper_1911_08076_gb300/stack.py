@@ -38,7 +38,7 @@ class DeviceStack:
             if l.kind == "conv":
                 p = params[li]
                 mode = {"codes": ifq.IFQ_OUT_CODES, "acc": ifq.IFQ_OUT_ACC, "both": ifq.IFQ_OUT_BOTH}[l.out]
-                d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path)
+                d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path, pool=l.pool)
                 K = l.k * l.k * l.cin
                 T, s = ifq.ifq_fold_layer(K, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias, p.eps,
                                           p.q_base, p.q_offset, kbits)
@@ -52,8 +52,8 @@ class DeviceStack:
                 prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=self.device)
                 ifq.ifq_pack_weights(d, bits, prep)
                 self.w_prep[li] = prep
-                ho, wo = ifq.ifq_conv_out_shape(d)
-                assert (ho, wo) == (l.ho, l.wo), (l.name, ho, wo)
+                ho, wo = ifq.ifq_conv_out_shape(d)   # after the fused pool, if any
+                assert (ho, wo) == (l.out_h, l.out_w), (l.name, ho, wo)
                 if mode & ifq.IFQ_OUT_CODES:
                     self.y_codes[li] = torch.empty((B, ho, wo, l.cout // 4), dtype=torch.uint8, device=self.device)
                 if mode & ifq.IFQ_OUT_ACC:

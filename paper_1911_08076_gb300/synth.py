@@ -38,7 +38,9 @@ class Conv:
 
     `src` is the index of the layer whose output codes feed this one (-1 for
     the stack input).  `out` is "codes", "acc" (int32 accumulators, for a
-    layer whose substructure is not quantized) or "both".
+    layer whose substructure is not quantized) or "both".  `pool` = p >= 2
+    max-pools the accumulators over p x p windows with stride p before the
+    thresholds (Sec. 2.1), so the codes are [b][ho/p][wo/p][cout].
     """
     name: str
     cin: int
@@ -52,7 +54,16 @@ class Conv:
     wo: int
     src: int
     out: str = "codes"
+    pool: int = 0
     kind: str = field(default="conv", init=False)
+
+    @property
+    def out_h(self) -> int:
+        return self.ho // self.pool if self.pool > 1 else self.ho
+
+    @property
+    def out_w(self) -> int:
+        return self.wo // self.pool if self.pool > 1 else self.wo
 
 
 @dataclass
@@ -163,12 +174,51 @@ def roofline(batch: int = 256, which: str = "3x3") -> Workload:
                     [_c1("conv1x1", 512, 512, 28, 28, -1)])
 
 
+def fuse_pools(wl: Workload) -> Workload:
+    """The same stack with every convolution whose codes feed only a signed p x p / stride p pool
+    (p in {2, 4}, no padding, sizes divisible by p) computing that pool itself (Sec. 2.1 order:
+    pool on the accumulators, then BN and the quantizer).  Same index, so the same draws."""
+    consumers = {}
+    for i, l in enumerate(wl.layers):
+        consumers.setdefault(l.src, []).append(i)
+    fused_into = {}   # conv index -> pool index merged into it
+    for i, l in enumerate(wl.layers):
+        if l.kind != "pool" or l.src < 0:
+            continue
+        c = wl.layers[l.src]
+        if (c.kind == "conv" and c.out == "codes" and c.pool <= 1 and l.signed and l.pad == 0 and
+                l.k == l.stride and l.k in (2, 4) and c.ho % l.k == 0 and c.wo % l.k == 0 and
+                consumers.get(l.src) == [i]):
+            fused_into[l.src] = i
+    dropped = set(fused_into.values())
+    new_index, layers = {}, []
+    for i, l in enumerate(wl.layers):
+        if i in dropped:
+            continue
+        new_index[i] = len(layers)
+        layers.append(l)
+    for i in dropped:   # a dropped pool's consumers read the fused conv
+        new_index[i] = new_index[wl.layers[i].src]
+    out = []
+    for i, l in enumerate(layers):
+        src = -1 if l.src < 0 else new_index[l.src]
+        if l.kind == "conv":
+            old = [j for j, m in enumerate(wl.layers) if m is l][0]
+            p = wl.layers[fused_into[old]].k if old in fused_into else l.pool
+            out.append(Conv(l.name, l.cin, l.cout, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.out, p))
+        else:
+            out.append(Pool(l.name, l.c, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.signed))
+    return Workload(wl.name + "_fused", wl.index, wl.batch, wl.h, wl.w, wl.c, out)
+
+
 WORKLOADS = {
     "pr1": pr1,
     "resnet18": resnet18,
     "alexnet": alexnet,
     "tinyyolo": lambda batch=64: tiny_yolo(batch, False),
     "tinieryolo": lambda batch=64: tiny_yolo(batch, True),
+    "tinyyolo_fused": lambda batch=64: fuse_pools(tiny_yolo(batch, False)),
+    "tinieryolo_fused": lambda batch=64: fuse_pools(tiny_yolo(batch, True)),
     "roofline3x3": lambda batch=256: roofline(batch, "3x3"),
     "roofline1x1": lambda batch=256: roofline(batch, "1x1"),
 }

@@ -172,3 +172,27 @@ def test_forward_workspace_is_counters_only_for_the_persistent_launch(monkeypatc
     # a pooling layer keeps the stack on per-layer launches
     pool = ifq.Layer(kind=ifq.IFQ_LAYER_POOL, src=2, pool=ifq.PoolDesc(3, 10, 10, 128, 2, 2, 0), y_codes=fake)
     assert ifq.ifq_forward_workspace_bytes(layers + [pool]) == 0
+
+
+def test_fused_pool_shapes_and_refusals():
+    """pool = p in {2, 4}: the output shape is the convolution's divided by p; other windows,
+    sizes not divisible by p, and accumulator outputs are refused before any launch."""
+    d = ifq.conv_desc(2, 16, 12, 64, 64, 3, 1, 1, pool=2)
+    assert ifq.ifq_conv_out_shape(d) == (8, 6)
+    assert ifq.ifq_conv_out_shape(ifq.conv_desc(1, 16, 16, 64, 64, 3, 1, 1, pool=4)) == (4, 4)
+    assert ifq.ifq_conv_out_shape(ifq.conv_desc(1, 16, 16, 64, 64, 3, 1, 1, pool=1)) == (16, 16)
+
+    def status(**kw):
+        args = dict(n=1, h=16, w=16, cin=64, cout=64, k=3, stride=1, pad=1)
+        args.update(kw)
+        with pytest.raises(ifq.IfqError) as e:
+            ifq.ifq_conv_out_shape(ifq.conv_desc(**args))
+        return e.value.status
+
+    assert status(h=13, pool=2) == ifq.IFQ_ESHAPE        # 13 rows do not split into 2x2 windows
+    assert status(pool=3) == ifq.IFQ_EUNSUPPORTED
+    fake = 1 << 20
+    d = ifq.conv_desc(1, 16, 16, 64, 64, 3, 1, 1, out_mode=ifq.IFQ_OUT_BOTH, pool=2)
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_conv2bit(d, fake, fake, fake, fake, fake, fake, stream=0)
+    assert e.value.status == ifq.IFQ_EUNSUPPORTED        # pooled accumulators are not an output

@@ -34,11 +34,11 @@ def _fold_gpu(p, K):
     return T, s
 
 
-def _run_conv(x, w, T, s, stride, pad, out_mode, path, bn=None):
+def _run_conv(x, w, T, s, stride, pad, out_mode, path, bn=None, pool=0):
     B, H, W, C = x.shape
     cout, k, _, _ = w.shape
     K = k * k * C
-    d = ifq.conv_desc(B, H, W, C, cout, k, stride, pad, out_mode, path)
+    d = ifq.conv_desc(B, H, W, C, cout, k, stride, pad, out_mode, path, pool=pool)
     xp = torch.from_numpy(synth.pack_codes(x)).to(DEV)
     bits = torch.from_numpy(synth.pack_signs(w).view(np.int32)).to(DEV)
     prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=DEV)
@@ -108,6 +108,44 @@ def test_conv_matches_oracle(case, path):
         ref, _ = O.check_chains(A, prm, To, so)
         assert len(np.unique(ref)) >= 3
         assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
+
+
+POOL_FUSED_CASES = [
+    # B, H, W, C, cout, k, stride, pad, p, bn
+    (2, 16, 16, 64, 64, 3, 1, 1, 2, None),      # 64 pooled pixels, one tile
+    (3, 22, 26, 64, 96, 3, 1, 1, 2, None),      # ragged last tile, partial channel tile
+    (2, 20, 20, 16, 32, 3, 1, 1, 2, None),      # 4-byte granules
+    (2, 12, 12, 8, 16, 3, 1, 1, 2, None),       # 1-byte granules
+    (2, 16, 16, 128, 256, 3, 1, 1, 4, None),    # 4x4 windows, 16 lanes each
+    (1, 28, 28, 64, 128, 3, 2, 1, 2, None),     # strided convolution, then the pool
+    (2, 16, 16, 64, 200, 3, 1, 1, 2, 32),       # every channel-tile width
+    (2, 16, 16, 64, 200, 3, 1, 1, 2, 64),
+    (2, 16, 16, 64, 200, 3, 1, 1, 2, 128),
+]
+
+
+@pytest.mark.parametrize("case", POOL_FUSED_CASES, ids=[str(c) for c in POOL_FUSED_CASES])
+def test_fused_pool_matches_oracle(case):
+    """Convolution with the fused p x p pool: the codes are those of the window maximum of the
+    accumulators (Sec. 2.1, pool before BN and the quantizer), bit-exact, including channels with
+    a negative BN scale (there the code is the window minimum)."""
+    B, H, W, C, cout, k, s, p, pool, bn = case
+    rng = np.random.default_rng(abs(hash(case)) % (2 ** 32))
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, k, k, C)) == 1, 1, -1).astype(np.int8)
+    K = k * k * C
+    prm = _params(rng, cout, K)
+    prm.gamma[1::3] = -np.abs(prm.gamma[1::3])      # channels with a negative BN scale in every case
+    T, sg = _fold_gpu(prm, K)
+    assert (sg < 0).any() and (sg > 0).any()
+    codes, _ = _run_conv(x, w, T, sg, s, p, ifq.IFQ_OUT_CODES, ifq.IFQ_PATH_TC, bn=bn, pool=pool)
+    A = O.conv_acc(x, w, s, p)
+    ref = O.int_chain(O.maxpool_acc(A, pool, pool, 0), *O.fold(prm, K))
+    assert codes.shape == ref.shape
+    assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
+    # and it equals the separate sign-aware pool on the unpooled codes
+    full, _ = _run_conv(x, w, T, sg, s, p, ifq.IFQ_OUT_CODES, ifq.IFQ_PATH_TC, bn=bn)
+    assert (codes == O.maxpool_codes(full, pool, pool, 0, sg)).all()
 
 
 @pytest.mark.parametrize("bn", [32, 64, 128])
@@ -324,3 +362,38 @@ def test_stack_with_reused_output_buffer_runs_layer_by_layer(monkeypatch):
     ref = O.forward(wl, x, params, images=[0, 1, 2])
     assert (synth.unpack_codes(st.y_codes[1].cpu().numpy(), 64) == ref[1]).all()
     assert (synth.unpack_codes(st.y_codes[0].cpu().numpy(), 64) == ref[2]).all()
+
+
+@pytest.mark.parametrize("name", ["tinyyolo", "tinieryolo"])
+def test_fused_pool_stack_equals_separate_pools(name):
+    """The YOLO stacks with each conv + 2x2/s2 pool pair fused into one launch: every fused layer's
+    pooled codes equal the separate sign-aware pool's output, every other layer is unchanged, and
+    the oracle (pool on the accumulators) agrees on the first and last image."""
+    base = synth.get(name, batch=3)
+    fused = synth.fuse_pools(base)
+    assert len(fused.layers) < len(base.layers)
+    x, params = synth.draw_workload(base)
+    xf, params_f = synth.draw_workload(fused)
+    assert (x == xf).all()
+    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+    sb, sf = DeviceStack(base, params), DeviceStack(fused, params_f)
+    sb.forward(xd)
+    sf.forward(xd)
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    # map each fused layer to the base layer whose output it must equal (the pool, when fused)
+    bi = 0
+    ref = O.forward(fused, x, params_f, images=[0, base.batch - 1])
+    for fi, lf in enumerate(fused.layers):
+        while base.layers[bi].name != lf.name:
+            bi += 1
+        target = bi + 1 if (lf.kind == "conv" and lf.pool > 1) else bi
+        got, want = sf.output(fi), sb.output(target)
+        for k in got:
+            assert (got[k] == want[k]).all(), (lf.name, k)
+        r = ref[fi]
+        if lf.kind == "conv" and lf.out == "acc":
+            assert (got["acc"][[0, -1]] == r).all()
+        elif not (lf.kind == "conv" and lf.out == "both"):
+            c = lf.cout if lf.kind == "conv" else lf.c
+            assert (synth.unpack_codes(got["codes"][[0, -1]], c) == r).all(), lf.name
