@@ -105,6 +105,26 @@ int ifq_fold_layer(int cout, int K, int kbits, const float* alpha, float delta_i
                    const float* gamma, const float* beta, const float* mean, const float* var, float eps,
                    float q_base, float q_offset, int32_t* thr_out, int8_t* sign_out);
 
+/*
+ * ifq_fold_layer_separated -- the same thresholds for the SEPARATED fixed-point
+ * conversion of Sec. 2.2 (Fig. 3a), the baseline the paper compares against:
+ * with Q = 2^m each float is floored at its own scale, a = floor(alpha*Q),
+ * d = floor(delta_in*Q), bq = floor(bias*Q^2), theta = floor(mean*Q),
+ * sigma = floor(sqrt(var + eps)/gamma * Q) (the affine BN's divisor),
+ * be = floor(beta*Q), t_i = floor(thr_i*Q), and the substructure computes
+ *   Y^conv = (a*d*A + bq)/Q^2,  Y^BN = (Y^conv - theta/Q)/(sigma/Q) + be/Q,
+ *   code = #{ i : Y^BN > t_i/Q }.
+ * That is monotone in A, so it too is code = #{ i : sign*A > T_i }; this
+ * returns those exact integer thresholds (64-bit integer arithmetic, no
+ * rounding), to run the separated conversion on the same kernels.
+ * Same arguments as ifq_fold_layer plus m (1..20); IFQ_EINVAL also when some
+ * channel's sigma floors to 0 (no fixed-point divisor).
+ */
+int ifq_fold_layer_separated(int cout, int K, int kbits, int m, const float* alpha, float delta_in,
+                             const float* bias, const float* gamma, const float* beta, const float* mean,
+                             const float* var, float eps, float q_base, float q_offset, int32_t* thr_out,
+                             int8_t* sign_out);
+
 /* Packed size in bytes of an n x h x w x c map of kbits-bit codes, 1 <= kbits <= 32 (host, pure). */
 int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
 

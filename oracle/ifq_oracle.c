@@ -22,6 +22,8 @@
  *   ifqo_maxpool_acc  Sec. 2.1: max pooling on Y^conv, before BN / quantizer.
  *   ifqo_maxpool_codes  pooling on codes: plain max, or with a per-channel sign
  *                     the max/min that equals quantize(max over Y^conv).
+ *   ifqo_separated_chain  the separated fixed-point conversion of Sec. 2.2 (each
+ *                     float floored at scale Q_m = 2^m on its own), for comparison.
  *
  * Readings of the paper used here (where it is silent or assumes more):
  *   - BN is the general affine form z = gamma*(y - mean)/sqrt(var + eps) + beta;
@@ -39,6 +41,8 @@
 
 #define ORC_OK 0
 #define ORC_EINVAL 1
+
+static int64_t floor_scaled(double x, double q) { return (int64_t)floor(x * q); }
 
 /* Uniform quantizer level i (1-based), Sec. 3.2: thr_i = i*base + offset. */
 static double level(int i, double q_base, double q_offset) { return (double)i * q_base + q_offset; }
@@ -226,5 +230,54 @@ int ifqo_maxpool_codes(int nb, int h, int w, int c, int k, int stride, int pad, 
             }
           out[(((long)b * ho + oy) * wo + ox) * c + ch] = (uint8_t)best;
         }
+  return ORC_OK;
+}
+
+/*
+ * Separated fixed-point conversion, Sec. 2.2 (Fig. 3a), for comparison with the
+ * integrated conversion.  With Q = 2^m, every float is floored at its own scale:
+ *   a = floor(alpha*Q), d = floor(delta_in*Q), bq = floor(bias*Q^2)
+ *   Y^conv = (a*d*A + bq) / Q^2                         (the paper's separated conv)
+ *   BN, Eq. (2) with the paper's theta = mean and sigma = sqrt(var + eps)/gamma (the
+ *   divisor of the affine BN), plus the shift beta: th = floor(mean*Q),
+ *   sg = floor(sigma*Q), be = floor(beta*Q):
+ *   Y^BN = (Y^conv - th/Q) / (sg/Q) + be/Q
+ *   code = #{ i : Y^BN > floor(thr_i*Q)/Q }             Eq. (3)
+ * evaluated exactly in 64-bit integers: with N = a*d*A + bq (= Y^conv * Q^2) and
+ * t_i = floor(thr_i*Q),  Y^BN > t_i/Q  <=>  (N - th*Q) / sg > t_i - be, i.e.
+ * N - th*Q > (t_i - be)*sg for sg > 0 and N - th*Q < (t_i - be)*sg for sg < 0.
+ * gamma = 0 (sigma infinite) gives Y^BN = be/Q for every A.  sg = 0 (|sigma| < 1/Q)
+ * has no fixed-point divisor and is rejected, as is m outside 1..20 (int64 range).
+ */
+int ifqo_separated_chain(long M, int cout, const int32_t* A, int L, int m, const double* alpha, double delta_in,
+                         const double* bias, const double* gamma, const double* beta, const double* mean,
+                         const double* var, double eps, double q_base, double q_offset, uint8_t* codes) {
+  if (M < 0 || cout <= 0 || L <= 0 || L > 255 || m < 1 || m > 20) return ORC_EINVAL;
+  const double Q = ldexp(1.0, m);
+  const int64_t Qi = (int64_t)1 << m;
+  const int64_t d = floor_scaled(delta_in, Q);
+  for (int n = 0; n < cout; ++n) {
+    const int64_t a = floor_scaled(alpha[n], Q);
+    const int64_t bq = (int64_t)floor((bias ? bias[n] : 0.0) * Q * Q);
+    const int64_t th = floor_scaled(mean[n], Q), be = floor_scaled(beta[n], Q);
+    int64_t sg = 0;
+    if (gamma[n] != 0.0) {
+      sg = floor_scaled(sqrt(var[n] + eps) / gamma[n], Q);
+      if (sg == 0) return ORC_EINVAL;
+    }
+    for (long r = 0; r < M; ++r) {
+      const int64_t N = a * d * (int64_t)A[r * cout + n] + bq;
+      int code = 0;
+      for (int i = 1; i <= L; ++i) {
+        const int64_t t = floor_scaled(level(i, q_base, q_offset), Q);
+        int above;
+        if (gamma[n] == 0.0) above = be > t;                          /* Y^BN = be/Q */
+        else if (sg > 0) above = N - th * Qi > (t - be) * sg;
+        else above = N - th * Qi < (t - be) * sg;
+        code += above;
+      }
+      codes[r * cout + n] = (uint8_t)code;
+    }
+  }
   return ORC_OK;
 }

@@ -57,8 +57,9 @@ def lib():
             L.ifqo_conv_acc.argtypes = [i, i, i, i, i, i, i, i, i, P, P, P]
             L.ifqo_maxpool_acc.argtypes = [i, i, i, i, i, i, i, P, P]
             L.ifqo_maxpool_codes.argtypes = [i, i, i, i, i, i, i, P, P, P]
+            L.ifqo_separated_chain.argtypes = [l, i, P, i, i, P, d, P, P, P, P, P, d, d, d, P]
             for f in ("ifqo_float_chain", "ifqo_fold", "ifqo_int_chain", "ifqo_conv_acc",
-                      "ifqo_maxpool_acc", "ifqo_maxpool_codes"):
+                      "ifqo_maxpool_acc", "ifqo_maxpool_codes", "ifqo_separated_chain"):
                 getattr(L, f).restype = ctypes.c_int
             _lib = L
     return _lib
@@ -137,6 +138,18 @@ def int_chain(A: np.ndarray, T: np.ndarray, sign: np.ndarray) -> np.ndarray:
 
 def conv_out(h: int, k: int, stride: int, pad: int) -> int:
     return (h + 2 * pad - k) // stride + 1
+
+
+def separated_chain(A: np.ndarray, p: "Params", m: int) -> np.ndarray:
+    """Codes of the separated fixed-point conversion (Sec. 2.2) at Q_m = 2^m, exact integers."""
+    cout = p.alpha.shape[0]
+    A2 = np.ascontiguousarray(A, dtype=np.int32).reshape(-1, cout)
+    codes = np.empty(A2.shape, dtype=np.uint8)
+    _check(lib().ifqo_separated_chain(A2.shape[0], cout, _p(A2), p.levels, m, _p(p.alpha), p.delta_in,
+                                      _p(p.bias) if p.bias is not None else None, _p(p.gamma), _p(p.beta),
+                                      _p(p.mean), _p(p.var), p.eps, p.q_base, p.q_offset, _p(codes)),
+           "separated_chain")
+    return codes.reshape(A.shape)
 
 
 def conv_acc(x: np.ndarray, w: np.ndarray, stride: int, pad: int) -> np.ndarray:

@@ -72,6 +72,68 @@ extern "C" int ifq_fold_layer(int cout, int K, int kbits, const float* alpha, fl
   return IFQ_OK;
 }
 
+// Floor division of 64-bit integers (toward -infinity), d > 0.
+static int64_t floor_div64(int64_t x, int64_t d) {
+  int64_t q = x / d;
+  if ((x % d != 0) && (x < 0)) --q;
+  return q;
+}
+
+extern "C" int ifq_fold_layer_separated(int cout, int K, int kbits, int m, const float* alpha, float delta_in,
+                                        const float* bias, const float* gamma, const float* beta, const float* mean,
+                                        const float* var, float eps, float q_base, float q_offset, int32_t* thr_out,
+                                        int8_t* sign_out) {
+  if (cout < 1 || K < 1 || kbits < 1 || kbits > 8 || m < 1 || m > 20) return IFQ_EINVAL;
+  if (!alpha || !gamma || !beta || !mean || !var || !thr_out || !sign_out) return IFQ_EINVAL;
+  const double din = delta_in, qb = q_base, qo = q_offset, ep = eps;
+  if (!(din > 0.0) || !std::isfinite(din) || !(qb > 0.0) || !std::isfinite(qb) || !std::isfinite(qo) ||
+      !std::isfinite(ep))
+    return IFQ_EINVAL;
+  const int L = (1 << kbits) - 1;
+  const int64_t amax = (int64_t)L * K;
+  const double Q = std::ldexp(1.0, m);
+  const int64_t Qi = (int64_t)1 << m;
+  // the fixed-point constants, each floored at its own scale (Sec. 2.2)
+  auto fx = [&](double x) { return (int64_t)std::floor(x * Q); };
+  for (int n = 0; n < cout; ++n) {
+    const double a = alpha[n], g = gamma[n], v = var[n], b = bias ? (double)bias[n] : 0.0;
+    if (!(a > 0.0) || !std::isfinite(a) || !std::isfinite(g) || !std::isfinite((double)beta[n]) ||
+        !std::isfinite((double)mean[n]) || !std::isfinite(v) || !std::isfinite(b) || !(v + ep > 0.0))
+      return IFQ_EINVAL;
+    if (g != 0.0 && fx(std::sqrt(v + ep) / g) == 0) return IFQ_EINVAL;   // no fixed-point BN divisor
+  }
+  const int64_t d = fx(din);
+  for (int n = 0; n < cout; ++n) {
+    const double g = gamma[n];
+    const int64_t ad = fx(alpha[n]) * d;                                  // Y^conv = (ad*A + bq) / Q^2
+    const int64_t bq = (int64_t)std::floor((bias ? (double)bias[n] : 0.0) * Q * Q);
+    const int64_t th = fx(mean[n]), be = fx(beta[n]);
+    const int64_t sg = g != 0.0 ? fx(std::sqrt((double)var[n] + ep) / g) : 0;   // sigma = sqrt(var+eps)/gamma
+    sign_out[n] = (int8_t)(sg < 0 ? -1 : 1);
+    for (int i = 1; i <= L; ++i) {
+      const int64_t t = fx(level(i, qb, qo));
+      int64_t T;
+      if (g == 0.0) {
+        T = be > t ? -amax - 1 : amax;   // Y^BN = be/Q for every A
+      } else {
+        // Y^BN > t/Q  <=>  (ad*A + bq - th*Q) / sg > t - be
+        //   sg > 0:  ad*A > X;   sg < 0:  ad*A < X,  X = (t - be)*sg + th*Q - bq
+        const int64_t X = (t - be) * sg + th * Qi - bq;
+        if (ad == 0) {
+          const bool above = sg > 0 ? 0 > X : 0 < X;
+          T = above ? -amax - 1 : amax;
+        } else {
+          T = sg > 0 ? floor_div64(X, ad) : floor_div64(-X, ad);   // -A > floor(-X/ad) for sg < 0
+        }
+        if (T < -amax - 1) T = -amax - 1;
+        if (T > amax) T = amax;
+      }
+      thr_out[(size_t)n * L + (i - 1)] = (int32_t)T;
+    }
+  }
+  return IFQ_OK;
+}
+
 extern "C" int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes) {
   if (!bytes || n < 0 || h < 0 || w < 0 || c < 0 || kbits < 1 || kbits > 32) return IFQ_EINVAL;
   const unsigned long long bits = (unsigned long long)n * h * w * c * (unsigned long long)kbits;

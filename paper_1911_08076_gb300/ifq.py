@@ -55,6 +55,7 @@ _SIGS = {
     "ifq_status_str": ([_I], ctypes.c_char_p),
     "ifq_version": ([], _I),
     "ifq_fold_layer": ([_I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
+    "ifq_fold_layer_separated": ([_I, _I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
     "ifq_codes_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
     "ifq_conv_out_shape": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
     "ifq_weights_prep_bytes": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_SZ)], _I),
@@ -147,6 +148,21 @@ def ifq_fold_layer(K: int, alpha, gamma, beta, mean, var, delta_in: float = 0.5,
     s = np.empty(cout, np.int8)
     _ok(lib().ifq_fold_layer(cout, int(K), kbits, _ptr(al), delta_in, _ptr(bi), _ptr(ga), _ptr(be), _ptr(mu),
                              _ptr(va), eps, q_base, q_offset, _ptr(T), _ptr(s)), "ifq_fold_layer")
+    return T, s
+
+
+def ifq_fold_layer_separated(K: int, m: int, alpha, gamma, beta, mean, var, delta_in: float = 0.5, bias=None,
+                             eps: float = 1e-5, q_base: float = 0.5, q_offset: float = -0.25, kbits: int = 2):
+    """Thresholds of the separated fixed-point conversion at Q = 2^m (host): (T, sign)."""
+    f32 = lambda a: None if a is None else np.ascontiguousarray(a, dtype=np.float32)
+    al, ga, be, mu, va, bi = map(f32, (alpha, gamma, beta, mean, var, bias))
+    cout = al.shape[0]
+    L = (1 << kbits) - 1
+    T = np.empty((cout, L), np.int32)
+    s = np.empty(cout, np.int8)
+    _ok(lib().ifq_fold_layer_separated(cout, int(K), kbits, int(m), _ptr(al), delta_in, _ptr(bi), _ptr(ga), _ptr(be),
+                                       _ptr(mu), _ptr(va), eps, q_base, q_offset, _ptr(T), _ptr(s)),
+        "ifq_fold_layer_separated")
     return T, s
 
 

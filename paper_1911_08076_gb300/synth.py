@@ -18,7 +18,9 @@ Sec. 4.1), Tiny-YOLO / Tinier-YOLO backbones (Sec. 4.2) and a ResNet-18 stack;
 the datasets and trained weights are not used.  Distributions: codes uniform
 on {0..3}, weights uniform +-1, alpha ~ U(0.5, 1.5), gamma ~ N(1, 0.3),
 beta ~ N(0, 0.5), mean ~ N(0, 2), var ~ U(0.5, 2), quantizer step 0.5,
-bias 0, eps 1e-5, seed 1911_08076 + config index.
+bias 0, eps 1e-5, seed 1911_08076 + config index.  For the separated-conversion
+study, draw_conv_params_calibrated gives trained-layer ranges instead (small
+alpha, BN statistics matched to the layer's pre-BN spread).
 """
 from __future__ import annotations
 
@@ -255,6 +257,23 @@ def draw_conv_params(rng: np.random.Generator, layer: Conv) -> ConvParams:
     beta = rng.normal(0.0, 0.5, cout).astype(np.float32)
     mean = rng.normal(0.0, 2.0, cout).astype(np.float32)
     var = rng.uniform(0.5, 2.0, cout).astype(np.float32)
+    return ConvParams(w, alpha, gamma, beta, mean, var)
+
+
+def draw_conv_params_calibrated(rng: np.random.Generator, layer: Conv) -> ConvParams:
+    """Parameters in the ranges of a trained HWGQ layer, for the separated-conversion study:
+    small filter scales alpha ~ U(0.005, 0.05) (the paper's loss case is small alpha), and BN
+    statistics of the layer's own pre-BN output y = alpha*STEP*A, whose spread for uniform codes
+    and +-1 filters is alpha*STEP*sqrt(3.5 K): mean ~ N(0, 0.1 sd), var = sd^2 * U(0.8, 1.25),
+    gamma ~ N(1, 0.3), beta ~ N(0, 0.5), so that the codes spread over every level."""
+    cout, k, cin = layer.cout, layer.k, layer.cin
+    w = np.where(rng.integers(0, 2, size=(cout, k, k, cin), dtype=np.int8) == 1, 1, -1).astype(np.int8)
+    alpha = rng.uniform(0.005, 0.05, cout).astype(np.float32)
+    sd = alpha.astype(np.float64) * STEP * np.sqrt(3.5 * k * k * cin)
+    gamma = rng.normal(1.0, 0.3, cout).astype(np.float32)
+    beta = rng.normal(0.0, 0.5, cout).astype(np.float32)
+    mean = (rng.normal(0.0, 0.1, cout) * sd).astype(np.float32)
+    var = (sd * sd * rng.uniform(0.8, 1.25, cout)).astype(np.float32)
     return ConvParams(w, alpha, gamma, beta, mean, var)
 
 

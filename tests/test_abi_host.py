@@ -196,3 +196,30 @@ def test_fused_pool_shapes_and_refusals():
     with pytest.raises(ifq.IfqError) as e:
         ifq.ifq_conv2bit(d, fake, fake, fake, fake, fake, fake, stream=0)
     assert e.value.status == ifq.IFQ_EUNSUPPORTED        # pooled accumulators are not an output
+
+
+@pytest.mark.parametrize("m", [6, 8, 10, 12, 16])
+def test_separated_fold_matches_oracle_chain_everywhere(m):
+    """ifq_fold_layer_separated solves the separated conversion's inequalities for integer
+    thresholds; on every achievable accumulator A in [-3K, 3K] its codes equal the oracle's
+    element-by-element evaluation of the separated chain (Sec. 2.2), for calibrated parameters with
+    both BN-scale signs."""
+    rng = np.random.default_rng(100 + m)
+    layer = synth.Conv("x", 64, 40, 3, 1, 1, 8, 8, 8, 8, -1)
+    cp = synth.draw_conv_params_calibrated(rng, layer)
+    cp.gamma[1::4] *= -1
+    cp.gamma[3] = 0.0
+    K = 9 * 64
+    T, s = ifq.ifq_fold_layer_separated(K, m, cp.alpha, cp.gamma, cp.beta, cp.mean, cp.var, synth.STEP, None,
+                                        synth.EPS)
+    p = O.Params.from_synth(cp)
+    A = np.arange(-3 * K, 3 * K + 1, dtype=np.int32)[:, None].repeat(40, 1)
+    assert (O.int_chain(A, T, s) == O.separated_chain(A, p, m)).all()
+
+
+def test_separated_fold_refusals():
+    one = np.ones(4, np.float32)
+    with pytest.raises(ifq.IfqError):
+        ifq.ifq_fold_layer_separated(64, 21, one, one, one * 0, one * 0, one)      # m beyond 20
+    with pytest.raises(ifq.IfqError):                                                # sigma floors to 0
+        ifq.ifq_fold_layer_separated(64, 4, one, one * 1e4, one * 0, one * 0, one)

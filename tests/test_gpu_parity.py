@@ -397,3 +397,28 @@ def test_fused_pool_stack_equals_separate_pools(name):
         elif not (lf.kind == "conv" and lf.out == "both"):
             c = lf.cout if lf.kind == "conv" else lf.c
             assert (synth.unpack_codes(got["codes"][[0, -1]], c) == r).all(), lf.name
+
+
+@pytest.mark.parametrize("m", [6, 8, 12])
+def test_separated_conversion_on_the_kernel(m):
+    """The separated fixed-point conversion (Sec. 2.2) is also a per-channel integer threshold test;
+    with ifq_fold_layer_separated's thresholds the tensor-core kernel reproduces the oracle's
+    element-by-element separated chain bit-exactly, and (with calibrated, small filter scales) it
+    differs from the integrated codes while the integrated codes equal the float chain."""
+    rng = np.random.default_rng(300 + m)
+    B, H, W, C, cout, k = 2, 14, 14, 64, 96, 3
+    layer = synth.Conv("x", C, cout, k, 1, 1, H, W, H, W, -1)
+    cp = synth.draw_conv_params_calibrated(rng, layer)
+    x = synth.draw_codes(rng, (B, H, W, C))
+    K = k * k * C
+    Ts, ss = ifq.ifq_fold_layer_separated(K, m, cp.alpha, cp.gamma, cp.beta, cp.mean, cp.var, synth.STEP, None,
+                                          synth.EPS)
+    codes, acc = _run_conv(x, cp.w, Ts, ss, 1, 1, ifq.IFQ_OUT_BOTH, ifq.IFQ_PATH_TC)
+    A = O.conv_acc(x, cp.w, 1, 1)
+    assert (acc == A).all()
+    p = O.Params.from_synth(cp)
+    sep = O.separated_chain(A, p, m)
+    assert (codes == sep).all()
+    integ, _ = O.check_chains(A, p, *O.fold(p, K))
+    if m <= 8:
+        assert (sep != integ).any()

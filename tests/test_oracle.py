@@ -302,3 +302,57 @@ def test_code_and_sign_packing_formats():
     assert int(words[0, 0]) == (0b1001 | (((1 << 28) - 1) << 4)) and int(words[0, 1]) == 0b11
     W = np.where(rng.integers(0, 2, (5, 3, 3, 20)) == 1, 1, -1).astype(np.int8)
     assert (synth.unpack_signs(synth.pack_signs(W), 180) == W.reshape(5, -1)).all()
+
+
+# ---------------------------------------------------------------- separated conversion (Sec. 2.2)
+
+def _sep_params(alpha, gamma, beta, mean, var, eps=0.0):
+    c = len(alpha)
+    return O.Params(np.array(alpha, float), np.array(gamma, float), np.array(beta, float), np.array(mean, float),
+                    np.array(var, float), None, 0.5, 0.5, -0.25, eps)
+
+
+def test_separated_equals_float_when_every_constant_is_exact():
+    """alpha = 3/4, delta = 1/2, mean = 1/4, sigma = 1, beta = 0 and the levels 1/4, 3/4, 5/4 are all
+    multiples of 1/16, so at Q = 16 no floor loses anything: the separated chain reproduces the float
+    chain for every achievable accumulator."""
+    p = _sep_params([0.75, 0.75], [1.0, -1.0], [0.0, 0.0], [0.25, 0.25], [1.0, 1.0])
+    K = 64
+    A = np.arange(-3 * K, 3 * K + 1, dtype=np.int32)[:, None].repeat(2, 1)
+    fc = O.float_chain(A, p)
+    assert (O.separated_chain(A, p, 4) == fc).all()
+
+
+def test_separated_hand_case_floor_loss():
+    """alpha = 0.3 at Q = 4 (m = 2): floor(1.2) = 1, so the separated conv scale is 1*2/16 = 0.125
+    per unit of A instead of 0.3*0.5 = 0.15 (delta 0.5 -> d = 2; sigma = 1 -> 4; mean = beta = 0;
+    levels 0.25/0.75/1.25 -> 1/3/5 quarters).  Float: z = 0.15 A; separated: Y = 0.125 A, and the
+    strict comparisons give, for A = 0..10,
+      float      0 0 1 1 1 1 2 2 2 3 3
+      separated  0 0 0 1 1 1 1 2 2 2 2   (A = 2: 0.25 is not above 0.25; A = 10: 1.25 not above 1.25)"""
+    p = _sep_params([0.3], [1.0], [0.0], [0.0], [1.0])
+    A = np.arange(0, 11, dtype=np.int32)[:, None]
+    fc = O.float_chain(A, p)
+    assert fc[:, 0].tolist() == [0, 0, 1, 1, 1, 1, 2, 2, 2, 3, 3]
+    assert O.separated_chain(A, p, 2)[:, 0].tolist() == [0, 0, 0, 1, 1, 1, 1, 2, 2, 2, 2]
+
+
+def test_separated_converges_and_is_monotone():
+    """Calibrated parameters: at m = 20 the separated codes equal the float chain's except within
+    rounding distance of a level; at every m the codes are monotone in A (non-decreasing for a
+    positive BN scale, non-increasing for a negative one)."""
+    rng = np.random.default_rng(7)
+    layer = synth.Conv("x", 64, 48, 3, 1, 1, 8, 8, 8, 8, -1)
+    cp = synth.draw_conv_params_calibrated(rng, layer)
+    cp.gamma[::5] *= -1
+    p = O.Params.from_synth(cp)
+    K = 576
+    A = np.arange(-3 * K, 3 * K + 1, dtype=np.int32)[:, None].repeat(48, 1)
+    fc, gap = O.float_chain(A, p, return_gap=True)
+    s20 = O.separated_chain(A, p, 20)
+    assert ((s20 != fc) <= (gap < 1e-4)).all()
+    for m in (4, 8, 12):
+        sc = O.separated_chain(A, p, m).astype(int)
+        d = np.diff(sc, axis=0)
+        up = p.gamma > 0
+        assert (d[:, up] >= 0).all() and (d[:, ~up] <= 0).all()
