@@ -4,10 +4,11 @@
  * for Embedded Vision", arXiv:1911.08076).
  *
  * The library computes, on one GPU, the quantized convolution of Eq. (1) with
- * +-1 filters W_b and unsigned 2-bit input codes X_q, and applies the
- * integrated fixed-point conversion of Sec. 3.2 as its epilogue: the integer
- * accumulator W_b (x) X_q is compared with per-channel integer thresholds
- * (Eq. (7) after the floor), which emits the next layer's 2-bit codes.
+ * +-1 filters W_b and unsigned k-bit input codes X_q (k = 2, 3 or 4), and
+ * applies the integrated fixed-point conversion of Sec. 3.2 as its epilogue:
+ * the integer accumulator W_b (x) X_q is compared with per-channel integer
+ * thresholds (Eq. (7) after the floor; Eq. (8) for k bits), which emits the
+ * next layer's k-bit codes.
  *
  * Conventions shared by every call:
  *   - Return value: an ifq_status.  Argument, shape, alignment and range
@@ -24,10 +25,12 @@
  *     ifq_device_status reads.
  *
  * Data formats:
- *   - Codes: NHWC, 2 bits per code, four codes per byte along C; channel c of
- *     a pixel is bits 2*(c%4)..2*(c%4)+1 of byte c/4 of that pixel.  C must be
- *     a multiple of 4, so a pixel is C/4 bytes.  Buffers are at least 16-byte
- *     aligned (cudaMalloc / torch allocations are).
+ *   - Codes: NHWC, packed along C in fields of f bits: f = 2 for k = 2 (four
+ *     codes per byte), f = 4 for k = 3 and k = 4 (two codes per byte, a 3-bit
+ *     code in the low bits of its field).  Channel c of a pixel is bits
+ *     f*(c%(8/f)) .. f*(c%(8/f))+f-1 of byte c/(8/f) of that pixel.  C must be
+ *     a multiple of 4, so a pixel is C*f/8 bytes.  Buffers are at least
+ *     16-byte aligned (cudaMalloc / torch allocations are).
  *   - Filter signs: one row per output channel over K = kh*kw*cin in
  *     (dy, dx, c) order (c fastest); bit k%32 of 32-bit word k/32 is 1 for +1
  *     and 0 for -1; a row is ceil(K/32) words.
@@ -125,8 +128,20 @@ int ifq_fold_layer_separated(int cout, int K, int kbits, int m, const float* alp
                              const float* var, float eps, float q_base, float q_offset, int32_t* thr_out,
                              int8_t* sign_out);
 
-/* Packed size in bytes of an n x h x w x c map of kbits-bit codes, 1 <= kbits <= 32 (host, pure). */
+/*
+ * Size in bits/8 (rounded up) of an n x h x w x c map of densely packed
+ * kbits-bit codes, 1 <= kbits <= 32 (host, pure): the memory count of the
+ * paper's comparison of feature-map sizes.  The library's own buffers use the
+ * field format above; ifq_codes_storage_bytes gives their size.
+ */
 int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
+
+/*
+ * Bytes of a packed code buffer in the library's format (host, pure):
+ * n*h*w*c*f/8 with f = 2 (kbits 0 or 2) or 4 (kbits 3, 4); c % 4 == 0
+ * (IFQ_ESHAPE otherwise); other kbits: IFQ_EUNSUPPORTED (negative: IFQ_EINVAL).
+ */
+int ifq_codes_storage_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
 
 /*
  * Convolution descriptor.  Input codes NHWC [n][h][w][cin] (cin % 4 == 0),
@@ -134,6 +149,9 @@ int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* bytes);
  * IFQ_OUT_*; codes output needs cout % 4 == 0.  path selects a kernel path
  * (IFQ_PATH_AUTO lets the library choose).  Limits: all sizes >= 1,
  * K = kh*kw*cin <= 65536, cout <= 65536, n*ho*wo < 2^31.
+ * kbits: the code width k of the input codes and of the output codes (0
+ * means 2; 2, 3 or 4, else IFQ_EUNSUPPORTED); the thresholds are then
+ * [cout][2^k - 1] (Eq. (8)).
  * pool: 0 or 1 for none; p = 2 or 4 max-pools the convolution output over
  * p x p windows with stride p before the thresholds (Sec. 2.1: the pool acts
  * on Y^conv, before BN and the quantizer), so that the codes are those of the
@@ -148,6 +166,7 @@ typedef struct {
   int out_mode;
   int path;
   int pool;
+  int kbits;
 } ifq_conv_desc;
 
 /* Output spatial size of a conv descriptor (host, pure). */
@@ -168,18 +187,30 @@ int ifq_weights_prep_bytes(const ifq_conv_desc* d, size_t* bytes);
  */
 int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_prep, void* stream);
 
+/*
+ * The kernel path ifq_conv2bit takes for `d` (host; reads IFQ_FORCE_PATH as
+ * ifq_conv2bit does): IFQ_PATH_TC or IFQ_PATH_BITSERIAL.  The tensor-core path
+ * needs (2^k - 1)*K <= 196608 (the accumulator range checked exact on the fp8
+ * tensor cores), kh, kw <= 32, and for k = 3, 4 cin % 8 == 0; a request for it
+ * outside that range takes the bit-serial path.  IFQ_EUNSUPPORTED for a fused
+ * pool off the tensor-core path.
+ */
+int ifq_conv_plan(const ifq_conv_desc* d, int* path);
+
 /* Device workspace that ifq_conv2bit needs for `d` (host, pure); may be 0. */
 int ifq_conv_workspace_bytes(const ifq_conv_desc* d, size_t* bytes);
 
 /*
  * ifq_conv2bit -- one quantized substructure (Eq. (1) integer core followed
- * by the thresholds of Eq. (7)).  For every output pixel and channel n:
+ * by the thresholds of Eq. (7), or of Eq. (8) for k bits; the name keeps the
+ * paper's k = 2 case).  For every output pixel and channel n:
  *   A = sum over (dy, dx, c) of w[n][dy][dx][c] * x[b][oy*s+dy-pad][ox*s+dx-pad][c]
- *   y_codes = #{ i : sign[n]*A > thr[n][i] }  (2-bit codes, packed)
+ *   y_codes = #{ i : sign[n]*A > thr[n][i] }  (k-bit codes, packed)
  *   y_acc   = A                                (int32), per out_mode
- * x (device): packed codes; w_prep (device): from ifq_pack_weights;
- * thr (device): int32 [cout][3]; sign (device): int8 [cout];
- * y_codes (device, out_mode & CODES): packed [n][ho][wo][cout/4] bytes;
+ * x (device): packed codes; w_prep (device): from ifq_pack_weights for the
+ * same descriptor; thr (device): int32 [cout][2^k - 1], ascending per channel;
+ * sign (device): int8 [cout];
+ * y_codes (device, out_mode & CODES): packed [n][ho][wo][cout*f/8] bytes;
  * y_acc (device, out_mode & ACC): int32 [n][ho][wo][cout];
  * ws (device): ifq_conv_workspace_bytes bytes (may be NULL if that is 0).
  * The results are exact integers; x must not alias the outputs.
@@ -188,9 +219,11 @@ int ifq_conv2bit(const ifq_conv_desc* d, const void* x, const void* w_prep, cons
                  const int8_t* sign, void* y_codes, int32_t* y_acc, void* ws, size_t ws_bytes, void* stream);
 
 /* Pooling descriptor (geometry in the header comment); c % 4 == 0. */
+/* Pooling descriptor; kbits is the code width as in ifq_conv_desc (0 means 2). */
 typedef struct {
   int n, h, w, c;
   int k, stride, pad;
+  int kbits;
 } ifq_pool_desc;
 
 int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo);
@@ -202,7 +235,7 @@ int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo);
  * composed conv/BN/quantizer map is monotone in the accumulator (increasing
  * for +1, decreasing for -1), this equals quantizing the max of Y^conv.  With
  * sign NULL it is the plain max of the codes (pooling after the quantizer).
- * x, y (device): packed codes.
+ * x, y (device): packed codes of width d->kbits.
  */
 int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, void* stream);
 
@@ -286,9 +319,15 @@ int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* 
 int ifq_graph_launch(ifq_graph* g, void* stream);
 int ifq_graph_destroy(ifq_graph* g);
 
-/* Codes <-> packed format helpers (device buffers; n % 4 == 0 codes). */
+/*
+ * Codes <-> packed format helpers (device buffers; n % 4 == 0 codes, one code
+ * per byte on the unpacked side).  The _kbits forms take the code width
+ * (0, 2, 3, 4; a code keeps its low f bits); the plain forms are kbits = 2.
+ */
 int ifq_pack_codes(const uint8_t* codes, void* packed, size_t n, void* stream);
 int ifq_unpack_codes(const void* packed, uint8_t* codes, size_t n, void* stream);
+int ifq_pack_codes_kbits(const uint8_t* codes, void* packed, size_t n, int kbits, void* stream);
+int ifq_unpack_codes_kbits(const void* packed, uint8_t* codes, size_t n, int kbits, void* stream);
 /* +-1 int8 filters [rows][K] (device) -> sign words [rows][ceil(K/32)] (device). */
 int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* stream);
 

@@ -221,11 +221,12 @@ def forward(workload, x: np.ndarray, params: Sequence, images: Optional[Sequence
     so they run on a thread pool (ctypes releases the GIL).
     """
     idx = list(range(x.shape[0])) if images is None else list(images)
+    kbits = getattr(workload, "kbits", 2)   # code width of every quantized layer (Eq. (8): 2^k - 1 thresholds)
     folded = {}
     for li, layer in enumerate(workload.layers):
         if layer.kind == "conv":
-            cp = params[li]
-            folded[li] = (Params.from_synth(cp), *fold(Params.from_synth(cp), layer.k * layer.k * layer.cin))
+            p = Params.from_synth(params[li], kbits)
+            folded[li] = (p, *fold(p, layer.k * layer.k * layer.cin))
 
     def one(b):
         outs = {}

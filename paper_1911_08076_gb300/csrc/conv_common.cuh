@@ -1,6 +1,6 @@
 // Device helpers shared by the single-layer and the stack tensor-core conv
 // kernels: layer arguments, tile geometry, the packed-code gather and the
-// 2-bit -> e4m3 expansion into tensor memory.  See conv_tc.cuh for the data
+// k-bit -> e4m3 expansion into tensor memory.  See conv_tc.cuh for the data
 // path and the exactness argument.
 #pragma once
 #include <cuda.h>
@@ -22,17 +22,19 @@ __device__ __forceinline__ uint32_t fdiv(uint32_t n, FastDiv f) {
 
 struct ConvArgs {
   const uint8_t* x;      // packed input codes, NHWC
-  const int32_t* thr;    // [cout][3]
+  const int32_t* thr;    // [cout][lvl]
   const int8_t* sign;    // [cout]
   uint8_t* y_codes;      // packed output codes or nullptr
   int32_t* y_acc;        // int32 accumulators or nullptr
   int n, h, w, cin, cout, kh, kw, stride, pad, ho, wo;
+  int cinb;              // bytes of packed codes per input pixel (cin * field bits / 8)
+  int lvl;               // thresholds per channel, 2^k - 1
   int M;                 // n*ho*wo
   int K;                 // kh*kw*cin
   int nk;                // number of 128-wide K stages (Kpad / 128)
   int nt;                // number of BN-wide output-channel tiles
   int ntiles;            // M tiles * nt
-  int ntab;              // entries of the K-granule table (Kpad / codes per granule)
+  int ntab;              // entries of the K-granule table (packed bytes of Kpad / granule bytes)
   FastDiv div_hw, div_wo, div_nt;   // by ho*wo, wo, nt
   // Fused p x p / stride p pool (p = 1 << lpool, lpool = 0: none).  Tile rows are then ordered
   // by pooled pixel and, within it, by window position (p*p consecutive rows, dy-major), so
@@ -53,12 +55,16 @@ constexpr int kStages = 8;       // K stages in flight (A in tensor memory, B in
 constexpr int kTmemA = 256;      // first tensor-memory column of the A stages
 constexpr int kAhead = 2;        // own K stages of packed codes a gather thread keeps in registers
 
-template <int BN>
+// SB: bits per stored code (2, or 4 for 3- and 4-bit codes).  Thresholds per column: a float4
+// (3 thresholds and the sign) for SB = 2, 16 floats (15 thresholds, padded with +inf, and the
+// sign) for SB = 4.
+template <int BN, int SB = 2>
 struct TcSmem {
   static constexpr int kB = BN * kBK;
+  static constexpr int kThrCol = SB == 2 ? 16 : 64;       // bytes of thresholds per column
   static constexpr int offB = 0;
-  static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN float4
-  static constexpr int offTab = offThr + 2 * BN * 16;      // kMaxTab x int2
+  static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN columns
+  static constexpr int offTab = offThr + 2 * BN * kThrCol; // kMaxTab x int2
   static constexpr int offBar = offTab + kMaxTab * 8;
   static constexpr int nBar = 2 * kStages + 5;             // full, empty, acc_full[2], acc_empty[2], done
   static constexpr int offTmem = offBar + nBar * 8;
@@ -99,7 +105,7 @@ __device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
       ox = (px << a.lpool) + (wpos & ((1 << a.lpool) - 1));
     }
     const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
-    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * (a.cin >> 2);
+    g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * a.cinb;
     g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));
     g.vx = bit_range(max(0, -ix0), min(a.kw, a.w - ix0));
   }
@@ -133,18 +139,20 @@ __device__ __forceinline__ uint32_t ld_codes1(const uint8_t* p) {
   else return (uint32_t)__ldg(p);
 }
 
-// 16 bytes (64 codes) of row g at K positions stage*128 + half*64 .. +64, zero outside the image.
+// 16 packed bytes of row g: unit u of the row's K sequence (bytes 16u .. 16u+15 of the packed
+// K codes, 64 two-bit or 32 four-bit codes), zero outside the image.  The table has one entry
+// per GB bytes, so unit u starts at entry u * 16 / GB.
 template <int GB, bool COHERENT = false>
-__device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int stage, int half) {
+__device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int u) {
   uint4 v = make_uint4(0u, 0u, 0u, 0u);
   if constexpr (GB == 16) {
-    const int2 e = tab[stage * 2 + half];
+    const int2 e = tab[u];
     if (tap_ok(g, e)) v = ld_codes16<COHERENT>(g.base + e.x);
   } else if constexpr (GB == 4) {
     uint32_t w[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const int2 e = tab[stage * 8 + half * 4 + q];
+      const int2 e = tab[u * 4 + q];
       w[q] = tap_ok(g, e) ? ld_codes4<COHERENT>(g.base + e.x) : 0u;
     }
     v = make_uint4(w[0], w[1], w[2], w[3]);
@@ -152,13 +160,13 @@ __device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, in
     uint32_t w[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      uint32_t u = 0;
+      uint32_t x = 0;
 #pragma unroll
       for (int bq = 0; bq < 4; ++bq) {
-        const int2 e = tab[stage * 32 + half * 16 + q * 4 + bq];
-        if (tap_ok(g, e)) u |= ld_codes1<COHERENT>(g.base + e.x) << (8 * bq);
+        const int2 e = tab[u * 16 + q * 4 + bq];
+        if (tap_ok(g, e)) x |= ld_codes1<COHERENT>(g.base + e.x) << (8 * bq);
       }
-      w[q] = u;
+      w[q] = x;
     }
     v = make_uint4(w[0], w[1], w[2], w[3]);
   }
@@ -174,6 +182,26 @@ __device__ __forceinline__ void expand_tmem_store(uint32_t taddr, uint4 v) {
   for (int j = 0; j < 4; ++j)
 #pragma unroll
     for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
+      "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
+      : "memory");
+}
+
+// 64 four-bit codes (two 16-byte units, 8 words) -> 16 tensor-memory columns of e4m3 bytes:
+// word j of the 8 contributes column 2j (its codes 0, 2, 4, 6 as bytes 0..3) and column
+// 2j+1 (codes 1, 3, 5, 7).  A code c in 0..15 is the e4m3 byte c, the value c * 2^-9 (0..7
+// subnormal, 8..15 with exponent field 1).
+__device__ __forceinline__ void expand4_tmem_store(uint32_t taddr, uint4 a, uint4 b) {
+  const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+  uint32_t o[16];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    o[2 * j] = w[j] & 0x0F0F0F0Fu;
+    o[2 * j + 1] = (w[j] >> 4) & 0x0F0F0F0Fu;
+  }
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
           taddr),

@@ -3,24 +3,25 @@
 //
 // GEMM view: D[m][n] = sum_k A[m][k] * B[n][k] with m = output pixel
 // (b, oy, ox), n = output channel, k = (dy, dx, c) -- an implicit GEMM whose
-// A rows are gathered on the fly from the packed 2-bit NHWC input.
+// A rows are gathered on the fly from the packed k-bit NHWC input (k = 2 in
+// 2-bit fields; k = 3, 4 in 4-bit fields, template parameter SB).
 //
 // Exact integer arithmetic on the fp8 tensor cores (sm_103a has no tcgen05
 // integer MMA):
-//   * A: code c in {0,1,2,3} is the e4m3 byte c, i.e. the subnormal value
-//     c * 2^-9; the 2-bit -> 8-bit expansion is a mask per byte lane.
+//   * A: code c in 0..15 is the e4m3 byte c, i.e. the value c * 2^-9
+//     (subnormal below 8); the k-bit -> 8-bit expansion is a mask per byte lane.
 //   * B: +1 / -1 are the e4m3 bytes 0x38 / 0xB8 (+-1.0).
 //   * Every product is c * 2^-9 exactly; every partial sum is an integer
-//     multiple of 2^-9 of magnitude <= 3K * 2^-9; with 3K < 2^15 it needs at
-//     most 24 significant bits, so the fp32 accumulator in tensor memory holds
-//     it exactly: D = A / 512.
+//     multiple of 2^-9 of magnitude <= (2^k - 1) K * 2^-9, far inside the
+//     24-bit fp32 significand for the magnitudes the host admits, so the fp32
+//     accumulator in tensor memory holds it exactly: D = A / 512.
 //   * Thresholds: sign*A > T  <=>  sign*D > T/512, and T/512 is exact in fp32
 //     (|T| < 2^24), so the epilogue compares the accumulator in fp32 directly.
 //
-// K ordering inside each 16-element chunk: the expansion of one 32-bit word
-// of 16 packed codes produces byte p = 4q + t from code 4t + q (a 4x4
-// transpose).  The prepared filter rows use the same order, so the dot
-// product over K is unchanged.
+// K ordering inside each chunk of one 32-bit word of packed codes (16 two-bit
+// or 8 four-bit codes): the expansion produces byte p = 4q + t from code
+// (cpw/4) t + q, cpw = codes per word (a transpose).  The prepared filter rows
+// use the same order, so the dot product over K is unchanged.
 //
 // Data path.  The expanded A operand never touches shared memory: gather
 // threads load packed codes from global memory into registers several K
@@ -41,7 +42,7 @@
 //                stages each (one elected lane per warp);
 //   warps 18-25  epilogue: tcgen05.ld of the finished accumulator (two
 //                buffers, so it overlaps the next tile's mainloop), thresholds,
-//                2-bit packing, stores.
+//                k-bit packing, stores.
 // Tensor memory (512 columns): accumulators in [0, 2*BN), A stages in
 // [256, 256 + 32*STAGES).  The K-stage pipeline runs continuously across tiles.
 #pragma once
@@ -62,18 +63,34 @@ __device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
       : "memory");
 }
 
-// GB: bytes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1 (cin % 4 == 0).
-template <int BN, int GB>
+// The code of one accumulator against 15 ascending thresholds (t[0..14], +inf past 2^k - 1)
+// and the channel sign (t[15]): #{ i : sign*D > t[i] } by binary search.
+__device__ __forceinline__ uint32_t code15(float d, const float* t) {
+  const float sv = d * t[15];
+  int c = sv > t[7] ? 8 : 0;
+  c += sv > t[c + 3] ? 4 : 0;
+  c += sv > t[c + 1] ? 2 : 0;
+  c += sv > t[c] ? 1 : 0;
+  return (uint32_t)c;
+}
+
+// GB: bytes per gathered granule: 16, 4 or 1 (the largest that divides the packed bytes of a
+// pixel); SB: bits per stored code (2 for k = 2, 4 for k = 3 and 4).
+template <int BN, int GB, int SB>
 __global__ void __launch_bounds__(kConvThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
   static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
-  using L = TcSmem<BN>;
+  static_assert(SB == 2 || SB == 4, "stored code width");
+  using L = TcSmem<BN, SB>;
+  constexpr int kU = kBK * SB / 8 / 16;       // 16-byte units of packed codes per K stage
+  constexpr int kCpb = 8 / SB;                // codes per byte
   constexpr int kS = kStages;
   extern __shared__ uint8_t smem_raw_[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sB = sbase + L::offB;
-  float4* sThr = (float4*)(smem + L::offThr);
+  float4* sThr = (float4*)(smem + L::offThr);      // SB = 2
+  float* sThr16 = (float*)(smem + L::offThr);       // SB = 4
   int2* sTab = (int2*)(smem + L::offTab);
   const uint32_t barBase = sbase + L::offBar;
   // full[s]: the arrivals of the 4 warps of the gather group that owns stage s, plus
@@ -112,14 +129,14 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   // K-granule table: byte offset of each granule from the row's tap-(0,0)
   // pointer, and its tap (dy, dx); dy = 0xFF past K.
   {
-    const int cinb = args.cin >> 2;
+    const int cinb = args.cinb;
     for (int gk = tid; gk < args.ntab; gk += kConvThreads) {
-      const int k0 = gk * 4 * GB;
+      const int k0 = gk * kCpb * GB;
       const int tap = k0 / args.cin, cc = k0 - tap * args.cin;
       int2 e = make_int2(0, 0xFF << 8);
       if (tap < args.kh * args.kw) {
         const int dy = tap / args.kw, dx = tap - dy * args.kw;
-        e = make_int2((dy * args.w + dx) * cinb + (cc >> 2), (dy << 8) | dx);
+        e = make_int2((dy * args.w + dx) * cinb + cc / kCpb, (dy << 8) | dx);
       }
       sTab[gk] = e;
     }
@@ -143,37 +160,47 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     while (l_k >= nk) { l_k -= nk; ++l_tile; }
     RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r
                                                 : args.M);
-    auto next_load = [&](uint4& lo, uint4& hi) {
-      lo = load_unit<GB>(sTab, g, l_k, 0);
-      hi = load_unit<GB>(sTab, g, l_k, 1);
+    // packed codes of kAh of this group's stages in registers (16 registers either way)
+    constexpr int kAh = SB == 2 ? kAhead : 1;
+    auto next_load = [&](uint4 (&u)[kU]) {
+#pragma unroll
+      for (int q = 0; q < kU; ++q) u[q] = load_unit<GB>(sTab, g, l_k * kU + q);
       l_k += kGatherGroups;
       if (l_k >= nk) {
         do { l_k -= nk; ++l_tile; } while (l_k >= nk);
         if (l_tile < n_local) g = row_geom(args, (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r);
       }
     };
-    uint4 ring_lo[kAhead], ring_hi[kAhead];
+    uint4 ring[kAh][kU];
 #pragma unroll
-    for (int d = 0; d < kAhead; ++d) {
-      ring_lo[d] = ring_hi[d] = make_uint4(0u, 0u, 0u, 0u);
-      if (d < own) next_load(ring_lo[d], ring_hi[d]);
+    for (int d = 0; d < kAh; ++d) {
+#pragma unroll
+      for (int q = 0; q < kU; ++q) ring[d][q] = make_uint4(0u, 0u, 0u, 0u);
+      if (d < own) next_load(ring[d]);
     }
     bool ok = true;
 #pragma unroll 1
-    for (int base = 0; base < own && ok; base += kAhead) {
+    for (int base = 0; base < own && ok; base += kAh) {
 #pragma unroll
-      for (int d = 0; d < kAhead; ++d) {
+      for (int d = 0; d < kAh; ++d) {
         const int j = base + d;
         if (j < own) {
-          const uint4 lo = ring_lo[d], hi = ring_hi[d];
-          if (j + kAhead < own) next_load(ring_lo[d], ring_hi[d]);
+          uint4 cur[kU];
+#pragma unroll
+          for (int q = 0; q < kU; ++q) cur[q] = ring[d][q];
+          if (j + kAh < own) next_load(ring[d]);
           const int it = group + kGatherGroups * j;
           const int s = it % kS;
           const uint32_t ph = (uint32_t)(it / kS) & 1u;
           if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
           tc_fence_after();
-          expand_tmem_store(tA + (uint32_t)(s * 32), lo);
-          expand_tmem_store(tA + (uint32_t)(s * 32 + 16), hi);
+          if constexpr (SB == 2) {
+            expand_tmem_store(tA + (uint32_t)(s * 32), cur[0]);
+            expand_tmem_store(tA + (uint32_t)(s * 32 + 16), cur[kU - 1]);
+          } else {
+            expand4_tmem_store(tA + (uint32_t)(s * 32), cur[0], cur[1]);
+            expand4_tmem_store(tA + (uint32_t)(s * 32 + 16), cur[kU - 2], cur[kU - 1]);
+          }
           asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
           tc_fence_before();
           __syncwarp();
@@ -296,13 +323,21 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       if (jt == 0 || args.nt > 1) {
         for (int c = et; c < BN; c += 256) {
           const int nn = n0 + c;
-          float4 v = make_float4(0.f, 0.f, 0.f, 1.f);
-          if (nn < args.cout && args.thr) {
-            // sign*A > T  <=>  sign*D > T/512 with D = A/512 (exact in fp32)
-            v = make_float4((float)args.thr[3 * nn] * (1.0f / 512.0f), (float)args.thr[3 * nn + 1] * (1.0f / 512.0f),
-                            (float)args.thr[3 * nn + 2] * (1.0f / 512.0f), (float)args.sign[nn]);
+          const bool has = nn < args.cout && args.thr;
+          // sign*A > T  <=>  sign*D > T/512 with D = A/512 (exact in fp32)
+          if constexpr (SB == 2) {
+            float4 v = make_float4(0.f, 0.f, 0.f, 1.f);
+            if (has)
+              v = make_float4((float)args.thr[3 * nn] * (1.0f / 512.0f), (float)args.thr[3 * nn + 1] * (1.0f / 512.0f),
+                              (float)args.thr[3 * nn + 2] * (1.0f / 512.0f), (float)args.sign[nn]);
+            sThr[tb * BN + c] = v;
+          } else {
+            float* t16 = sThr16 + (size_t)(tb * BN + c) * 16;
+#pragma unroll
+            for (int i = 0; i < 15; ++i)
+              t16[i] = has && i < args.lvl ? (float)args.thr[(size_t)args.lvl * nn + i] * (1.0f / 512.0f) : INFINITY;
+            t16[15] = has ? (float)args.sign[nn] : 1.0f;
           }
-          sThr[tb * BN + c] = v;
         }
         named_bar(1, kEpiWarps * 32);
       }
@@ -312,7 +347,9 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
       const float4* th = sThr + tb * BN + c_lo;
-      uint32_t packed[CW / 16];
+      const float* th16 = sThr16 + (size_t)(tb * BN + c_lo) * 16;
+      constexpr int kPW = CW * SB / 32;          // 32-bit words of packed codes per thread
+      uint32_t packed[kPW];
 #pragma unroll
       for (int c0 = 0; c0 < CW; c0 += 16) {
         uint32_t v[16];
@@ -340,16 +377,23 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           for (int j = 0; j < 4; ++j)
             a4[j] = fmaxf(h1 ? a8[j + 4] : a8[j], __shfl_xor_sync(0xffffffffu, h1 ? a8[j] : a8[j + 4], 1));
           const int sub = (h2 ? 8 : 0) + (h1 ? 4 : 0);
-          uint32_t byte = 0;
+          uint32_t bits = 0;
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            const float4 tq = th[c0 + sub + j];
-            const float sv = a4[j] * tq.w;
-            byte |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
+            if constexpr (SB == 2) {
+              const float4 tq = th[c0 + sub + j];
+              const float sv = a4[j] * tq.w;
+              bits |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
+            } else {
+              bits |= code15(a4[j], th16 + (c0 + sub + j) * 16) << (4 * j);
+            }
           }
           const int cabs = n0 + c_lo + c0 + sub;
-          if (args.y_codes && m < args.M && cabs < args.cout)
-            args.y_codes[(size_t)(m >> 2) * (args.cout >> 2) + (cabs >> 2)] = (uint8_t)byte;
+          if (args.y_codes && m < args.M && cabs < args.cout) {
+            uint8_t* dst = args.y_codes + (size_t)(m >> 2) * ((args.cout * SB) >> 3) + ((cabs * SB) >> 3);
+            if constexpr (SB == 2) *dst = (uint8_t)bits;
+            else *(uint16_t*)dst = (uint16_t)bits;   // cabs % 4 == 0: an even byte offset
+          }
           continue;
         }
         if (args.lpool) {   // 4x4: every lane of the window gets the maxima of all 16 columns
@@ -361,15 +405,25 @@ __global__ void __launch_bounds__(kConvThreads, 1)
             v[j] = __float_as_uint(x);
           }
         }
-        uint32_t wd = 0;
+        if constexpr (SB == 2) {
+          uint32_t wd = 0;
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const float4 tq = th[c0 + j];
-          const float sv = __uint_as_float(v[j]) * tq.w;
-          const uint32_t code = (uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z);
-          wd |= code << (2 * j);
+          for (int j = 0; j < 16; ++j) {
+            const float4 tq = th[c0 + j];
+            const float sv = __uint_as_float(v[j]) * tq.w;
+            const uint32_t code = (uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z);
+            wd |= code << (2 * j);
+          }
+          packed[c0 / 16] = wd;
+        } else {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            uint32_t wd = 0;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) wd |= code15(__uint_as_float(v[8 * h + j]), th16 + (c0 + 8 * h + j) * 16) << (4 * j);
+            packed[c0 / 8 + h] = wd;
+          }
         }
-        packed[c0 / 16] = wd;
         if (args.y_acc && m < args.M) {
           const int cbase = n0 + c_lo + c0;
           int32_t* dst = args.y_acc + (size_t)m * args.cout + cbase;
@@ -398,20 +452,23 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       // the pooled pixel m >> 4)
       const bool store = args.y_codes && m < args.M && args.lpool != 1 && (m & ((1 << (2 * args.lpool)) - 1)) == 0;
       if (store) {
-        const int rowb = args.cout >> 2;        // bytes per output pixel
-        const int cb = n0 + c_lo;               // first channel of this thread
-        uint8_t* dst = args.y_codes + (size_t)(m >> (2 * args.lpool)) * rowb + (cb >> 2);
-        if (cb + CW <= args.cout && CW >= 64 && (rowb & 15) == 0 && (cb & 63) == 0) {
+        const int rowb = (args.cout * SB) >> 3;   // bytes per output pixel
+        const int cb = n0 + c_lo;                 // first channel of this thread
+        const int cbb = (cb * SB) >> 3;           // its byte within the pixel
+        uint8_t* dst = args.y_codes + (size_t)(m >> (2 * args.lpool)) * rowb + cbb;
+        if (cb + CW <= args.cout && kPW >= 4 && (rowb & 15) == 0 && (cbb & 15) == 0) {
 #pragma unroll
-          for (int q = 0; q < CW / 64; ++q)
+          for (int q = 0; q < kPW / 4; ++q)
             *(uint4*)(dst + 16 * q) =
                 make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2], packed[4 * q + 3]);
-        } else if (cb + CW <= args.cout && (rowb & 3) == 0 && (cb & 15) == 0) {
+        } else if (cb + CW <= args.cout && (rowb & 3) == 0 && (cbb & 3) == 0) {
 #pragma unroll
-          for (int q = 0; q < CW / 16; ++q) *(uint32_t*)(dst + 4 * q) = packed[q];
+          for (int q = 0; q < kPW; ++q) *(uint32_t*)(dst + 4 * q) = packed[q];
         } else {
-          const int nbytes = max(0, min(CW, args.cout - cb)) >> 2;
-          for (int q = 0; q < nbytes; ++q) dst[q] = (uint8_t)(packed[q >> 2] >> (8 * (q & 3)));
+          const int nbytes = (max(0, min(CW, args.cout - cb)) * SB) >> 3;
+#pragma unroll
+          for (int q = 0; q < 4 * kPW; ++q)   // unrolled: packed[] stays in registers
+            if (q < nbytes) dst[q] = (uint8_t)(packed[q >> 2] >> (8 * (q & 3)));
         }
       }
     }

@@ -1,5 +1,5 @@
 // C ABI entry points that launch device work: filter preparation, the
-// quantized convolution (tensor-core and bit-serial paths), 2-bit pooling,
+// quantized convolution (tensor-core and bit-serial paths), code pooling,
 // the layer-stack driver and its CUDA-graph form, packing helpers and the
 // device status word.  Host-only calls (the fold, shapes) live in ifq_host.cpp.
 #include <cuda.h>
@@ -25,7 +25,11 @@ namespace {
 using namespace ifq;
 
 constexpr int kMaxK = 65536;
-constexpr int kTcMaxK = 10922;   // 3K < 2^15: accumulators exact in the fp32 tensor-memory path
+// Largest accumulator magnitude (2^k - 1) K of the tensor-core path.  Every partial sum is an
+// integer multiple of 2^-9 below 2^24 * 2^-9, so an fp32 accumulation is exact; this bound is the
+// largest magnitude at which exactness has been checked on GB300 with adversarial inputs
+// (accumulators near the bound with odd addends all along K).
+constexpr int kTcMaxAcc = 3 * 65536;
 constexpr int kMaxDevices = 64;
 
 inline bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -78,28 +82,28 @@ cudaError_t launch_k(void (*kern)(Exp...), dim3 grid, dim3 block, size_t smem, c
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
 }
 
-template <int BN, int GB>
+template <int BN, int GB, int SB>
 struct TcInst {
-  using L = TcSmem<BN>;
+  using L = TcSmem<BN, SB>;
   static_assert(L::bytes <= 232448, "shared memory budget");
   static cudaError_t set_attr() {
-    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
+    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB, SB>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
     const int grid = a.ntiles < nsm ? a.ntiles : nsm;
-    return launch_k(conv_tc_kernel<BN, GB>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
+    return launch_k(conv_tc_kernel<BN, GB, SB>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
   }
 };
 
 // The output-channel tile widths of the tensor-core kernel.
-#define IFQ_TC_VARIANTS(X, GB) X(128, GB) X(64, GB) X(32, GB)
+#define IFQ_TC_VARIANTS(X, GB, SB) X(128, GB, SB) X(64, GB, SB) X(32, GB, SB)
 
-template <int GB>
+template <int GB, int SB>
 cudaError_t set_attrs_gb() {
   cudaError_t e = cudaSuccess;
-#define IFQ_SET(BN, G) \
-  if (e == cudaSuccess) e = TcInst<BN, G>::set_attr();
-  IFQ_TC_VARIANTS(IFQ_SET, GB)
+#define IFQ_SET(BN, G, S) \
+  if (e == cudaSuccess) e = TcInst<BN, G, S>::set_attr();
+  IFQ_TC_VARIANTS(IFQ_SET, GB, SB)
 #undef IFQ_SET
   return e;
 }
@@ -119,7 +123,9 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   std::lock_guard<std::mutex> lk(g_dev_mu);
   DevState& d = g_dev[dev];
   if (!d.init) {
-    if (set_attrs_gb<16>() != cudaSuccess || set_attrs_gb<4>() != cudaSuccess || set_attrs_gb<1>() != cudaSuccess)
+    if (set_attrs_gb<16, 2>() != cudaSuccess || set_attrs_gb<4, 2>() != cudaSuccess ||
+        set_attrs_gb<1, 2>() != cudaSuccess || set_attrs_gb<16, 4>() != cudaSuccess ||
+        set_attrs_gb<4, 4>() != cudaSuccess)
       return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
     if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
@@ -157,15 +163,29 @@ int env_int(const char* name, int dflt) {
 
 // ---------------------------------------------------------------- descriptors and planning
 
+// Code width of a descriptor's kbits field (0 means 2): k, the stored field width sb (2 for
+// k = 2, 4 for k = 3 and 4) and the thresholds per channel 2^k - 1.  Returns an ifq_status.
+int code_width(int kbits, int* k, int* sb, int* lvl) {
+  if (kbits < 0) return IFQ_EINVAL;
+  const int kk = kbits == 0 ? 2 : kbits;
+  if (kk < 2 || kk > 4) return IFQ_EUNSUPPORTED;
+  *k = kk;
+  *sb = kk == 2 ? 2 : 4;
+  *lvl = (1 << kk) - 1;
+  return IFQ_OK;
+}
+
 struct ConvGeom {
   int ho, wo, M, K, Kpad, kwords;
   int pool, pho, pwo;   // fused pool window (1: none) and the output shape after it
+  int kb, sb, lvl;      // code width k, stored field bits, thresholds per channel
 };
 
 int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if (!d) return IFQ_EINVAL;
   int rc = ifq_conv_out_shape(d, &g->pho, &g->pwo);   // output shape, after the fused pool if any
   if (rc) return rc;
+  if ((rc = code_width(d->kbits, &g->kb, &g->sb, &g->lvl))) return rc;
   g->pool = d->pool > 1 ? d->pool : 1;
   g->ho = g->pho * g->pool;                            // the convolution's own output
   g->wo = g->pwo * g->pool;
@@ -226,27 +246,36 @@ int choose_bn(const ConvGeom& g, int cout, int nsm) {
   return best;
 }
 
-template <int GB>
+template <int GB, int SB>
 cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
-#define IFQ_LAUNCH(BN, G) \
-  if (bn == BN) return TcInst<BN, G>::launch(tm, a, nsm, st);
-  IFQ_TC_VARIANTS(IFQ_LAUNCH, GB)
+#define IFQ_LAUNCH(BN, G, S) \
+  if (bn == BN) return TcInst<BN, G, S>::launch(tm, a, nsm, st);
+  IFQ_TC_VARIANTS(IFQ_LAUNCH, GB, SB)
 #undef IFQ_LAUNCH
   return cudaErrorInvalidValue;
 }
 
-// Whether the tensor-core kernel supports this shape: exact fp32 accumulation
-// (3K < 2^15), taps addressable by 32-bit masks, and a K-granule table that fits.
-bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
-  if (g.K > kTcMaxK || d->kh > 32 || d->kw > 32) return false;
-  const int gran = d->cin % 64 == 0 ? 64 : (d->cin % 16 == 0 ? 16 : 4);
-  if (g.Kpad / gran > kMaxTab) return false;
-  const long long span = ((long long)(d->kh - 1) * d->w + d->kw) * (d->cin / 4) + d->cin / 4;
-  return span < (1LL << 31);
+// Bytes of packed codes per input pixel.
+int pixel_bytes(const ifq_conv_desc* d, const ConvGeom& g) { return d->cin * g.sb / 8; }
+
+// Bytes of packed codes per gathered granule: the largest of 16, 4, 1 that divides a pixel's bytes.
+int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
+  const int pb = pixel_bytes(d, g);
+  return pb % 16 == 0 ? 16 : (pb % 4 == 0 ? 4 : 1);
 }
 
-// Bytes of packed codes per gathered granule: 16 (cin % 64 == 0), 4 (cin % 16 == 0), 1.
-int granule_bytes(const ifq_conv_desc* d) { return d->cin % 64 == 0 ? 16 : (d->cin % 16 == 0 ? 4 : 1); }
+// Whether the tensor-core kernel supports this shape: an accumulator magnitude inside the
+// checked exact range, taps addressable by 32-bit masks, a K-granule table that fits, and an
+// instantiated granule (4-bit fields need 4-byte granules, cin % 8 == 0).
+bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  if ((long long)g.lvl * g.K > kTcMaxAcc || d->kh > 32 || d->kw > 32) return false;
+  const int gb = granule_bytes(d, g);
+  if (g.sb == 4 && gb == 1) return false;
+  if ((long long)g.Kpad * g.sb / 8 / gb > kMaxTab) return false;
+  const long long pb = pixel_bytes(d, g);
+  const long long span = ((long long)(d->kh - 1) * d->w + d->kw) * pb + pb;
+  return span < (1LL << 31);
+}
 
 // TMA descriptor of the prepared e4m3 filter rows: [cout][Kpad] bytes, box 128 x bn, 128B swizzle.
 bool encode_wmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, int bn, CUtensorMap* tm) {
@@ -269,12 +298,14 @@ void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const voi
   a->y_acc = ya;
   a->n = d->n; a->h = d->h; a->w = d->w; a->cin = d->cin; a->cout = d->cout;
   a->kh = d->kh; a->kw = d->kw; a->stride = d->stride; a->pad = d->pad; a->ho = g.ho; a->wo = g.wo;
+  a->cinb = pixel_bytes(d, g);
+  a->lvl = g.lvl;
   a->M = g.M;
   a->K = g.K;
   a->nk = g.Kpad / kBK;
   a->nt = ceil_div(d->cout, bn);
   a->ntiles = ceil_div(g.M, kBM) * a->nt;
-  a->ntab = g.Kpad / (4 * granule_bytes(d));
+  a->ntab = g.Kpad * g.sb / 8 / granule_bytes(d, g);
   a->div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
   a->div_wo = make_fastdiv((uint32_t)g.wo);
   a->div_nt = make_fastdiv((uint32_t)a->nt);
@@ -306,10 +337,15 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
-    const int gb = granule_bytes(d);
-    if (gb == 16) e = launch_tc_gb<16>(bn, tm, a, nsm, st);
-    else if (gb == 4) e = launch_tc_gb<4>(bn, tm, a, nsm, st);
-    else e = launch_tc_gb<1>(bn, tm, a, nsm, st);
+    const int gb = granule_bytes(d, g);
+    if (g.sb == 2) {
+      if (gb == 16) e = launch_tc_gb<16, 2>(bn, tm, a, nsm, st);
+      else if (gb == 4) e = launch_tc_gb<4, 2>(bn, tm, a, nsm, st);
+      else e = launch_tc_gb<1, 2>(bn, tm, a, nsm, st);
+    } else {
+      if (gb == 16) e = launch_tc_gb<16, 4>(bn, tm, a, nsm, st);
+      else e = launch_tc_gb<4, 4>(bn, tm, a, nsm, st);
+    }
   } else {
     BsArgs a;
     a.x = (const uint8_t*)x;
@@ -323,8 +359,10 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     a.M = g.M;
     a.K = g.K;
     a.kwords = g.kwords;
+    a.lvl = g.lvl;
     dim3 grid(ceil_div(g.M, kBsTM), ceil_div(d->cout, kBsTN));
-    e = launch_k(conv_bitserial_kernel, grid, dim3(kBsThreads), 0, st, a);
+    if (g.sb == 2) e = launch_k(conv_bitserial_kernel<2>, grid, dim3(kBsThreads), 0, st, a);
+    else e = launch_k(conv_bitserial_kernel<4>, grid, dim3(kBsThreads), 0, st, a);
   }
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
@@ -335,17 +373,20 @@ int launch_1d_blocks(size_t items, int threads, int nsm) {
   return b < 1 ? 1 : (int)b;
 }
 
-int check_pool(const ifq_pool_desc* d, int* ho, int* wo) {
+int check_pool(const ifq_pool_desc* d, int* ho, int* wo, int* sb = nullptr) {
   int rc = ifq_pool_out_shape(d, ho, wo);
   if (rc) return rc;
+  int k, f, lvl;
+  if ((rc = code_width(d->kbits, &k, &f, &lvl))) return rc;
+  if (sb) *sb = f;
   if (d->c % 4 != 0 || d->pad >= d->k) return IFQ_ESHAPE;
   if ((long long)d->n * d->h * d->w * d->c >= (1LL << 40)) return IFQ_ERANGE;
   return IFQ_OK;
 }
 
 int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, cudaStream_t st) {
-  int ho, wo;
-  int rc = check_pool(d, &ho, &wo);
+  int ho, wo, sb;
+  int rc = check_pool(d, &ho, &wo, &sb);
   if (rc) return rc;
   if (!x || !y) return IFQ_EINVAL;
   if (!aligned16(x) || !aligned16(y)) return IFQ_EALIGN;
@@ -358,24 +399,35 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   a.n = d->n; a.h = d->h; a.w = d->w; a.c = d->c; a.k = d->k; a.stride = d->stride; a.pad = d->pad;
   a.ho = ho; a.wo = wo;
   const size_t pix = (size_t)d->n * ho * wo;
+  const int pb = d->c * sb / 8;   // packed bytes per pixel
+  const dim3 b256(256);
   cudaError_t e;
-  if (d->c % 64 == 0)
-    e = launch_k(maxpool2bit_kernel<4>, dim3(launch_1d_blocks(pix * (d->c / 64), 256, nsm)), dim3(256), 0, st, a);
-  else if (d->c % 16 == 0)
-    e = launch_k(maxpool2bit_kernel<1>, dim3(launch_1d_blocks(pix * (d->c / 16), 256, nsm)), dim3(256), 0, st, a);
-  else
-    e = launch_k(maxpool2bit_bytes_kernel, dim3(launch_1d_blocks(pix * (d->c / 4), 256, nsm)), dim3(256), 0, st, a);
+  if (pb % 16 == 0) {
+    const dim3 grid(launch_1d_blocks(pix * (pb / 16), 256, nsm));
+    e = sb == 2 ? launch_k(maxpool_codes_kernel<4, 2>, grid, b256, 0, st, a)
+                : launch_k(maxpool_codes_kernel<4, 4>, grid, b256, 0, st, a);
+  } else if (pb % 4 == 0) {
+    const dim3 grid(launch_1d_blocks(pix * (pb / 4), 256, nsm));
+    e = sb == 2 ? launch_k(maxpool_codes_kernel<1, 2>, grid, b256, 0, st, a)
+                : launch_k(maxpool_codes_kernel<1, 4>, grid, b256, 0, st, a);
+  } else {
+    const dim3 grid(launch_1d_blocks(pix * pb, 256, nsm));
+    e = sb == 2 ? launch_k(maxpool_codes_bytes_kernel<2>, grid, b256, 0, st, a)
+                : launch_k(maxpool_codes_bytes_kernel<4>, grid, b256, 0, st, a);
+  }
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
-// Output shape (n, h, w, c) of a layer, and whether it produces codes.
-int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes) {
+// Output shape (n, h, w, c) of a layer, whether it produces codes, and their width k (a layer's
+// input codes and its output codes have the same width).
+int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes, int* kb) {
   if (l.kind == IFQ_LAYER_CONV) {
     ConvGeom g;
     int rc = check_conv(&l.conv, &g);
     if (rc) return rc;
     *n = l.conv.n; *h = g.pho; *w = g.pwo; *c = l.conv.cout;
     *codes = (l.conv.out_mode & IFQ_OUT_CODES) != 0;
+    *kb = g.kb;
     return IFQ_OK;
   }
   if (l.kind == IFQ_LAYER_POOL) {
@@ -384,6 +436,7 @@ int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes) {
     if (rc) return rc;
     *n = l.pool.n; *h = ho; *w = wo; *c = l.pool.c;
     *codes = true;
+    *kb = l.pool.kbits == 0 ? 2 : l.pool.kbits;
     return IFQ_OK;
   }
   return IFQ_EINVAL;
@@ -393,16 +446,16 @@ int check_stack(const ifq_layer* layers, int nlayers, const void* x) {
   if (!layers || nlayers < 1 || !x) return IFQ_EINVAL;
   for (int i = 0; i < nlayers; ++i) {
     const ifq_layer& l = layers[i];
-    int n, h, w, c;
+    int n, h, w, c, kb;
     bool codes;
-    int rc = layer_out(l, &n, &h, &w, &c, &codes);
+    int rc = layer_out(l, &n, &h, &w, &c, &codes, &kb);
     if (rc) return rc;
     if (l.src < -1 || l.src >= i) return IFQ_EINVAL;
     if (l.src >= 0) {
-      int sn, sh, sw, sc;
+      int sn, sh, sw, sc, skb;
       bool sc_codes;
-      layer_out(layers[l.src], &sn, &sh, &sw, &sc, &sc_codes);
-      if (!sc_codes) return IFQ_ESHAPE;
+      layer_out(layers[l.src], &sn, &sh, &sw, &sc, &sc_codes, &skb);
+      if (!sc_codes || skb != kb) return IFQ_ESHAPE;
       const int in_n = l.kind == IFQ_LAYER_CONV ? l.conv.n : l.pool.n;
       const int in_h = l.kind == IFQ_LAYER_CONV ? l.conv.h : l.pool.h;
       const int in_w = l.kind == IFQ_LAYER_CONV ? l.conv.w : l.pool.w;
@@ -434,9 +487,9 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     if (layers[i].kind != IFQ_LAYER_CONV) return false;
     ConvGeom g;
     if (check_conv(&layers[i].conv, &g)) return false;
-    if (g.pool > 1) return false;   // the persistent kernel has no fused pool
+    if (g.pool > 1 || g.kb != 2) return false;   // the persistent kernel: 2-bit codes, no fused pool
     if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
-    tab += g.Kpad / (4 * granule_bytes(&layers[i].conv));
+    tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g));
   }
   if (tab > kMaxStackTab) return false;
   if (bytes) *bytes = round_up(stack_counters(layers, nlayers) * sizeof(unsigned int), 256);
@@ -531,7 +584,7 @@ int launch_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, voi
     StackLayer& S = P.L[i];
     fill_conv_args(&l.conv, g, bn, l.src < 0 ? x : layers[l.src].y_codes, l.thr, l.sign, yc, ya, &S.a);
     S.bn = bn;
-    S.gb = granule_bytes(&l.conv);
+    S.gb = granule_bytes(&l.conv, g);
     S.tab_off = tab;
     S.dep = l.src;
     S.cnt_off = cnt;
@@ -619,8 +672,19 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
   uint8_t* base = (uint8_t*)w_prep;
   const int blocks = launch_1d_blocks((size_t)d->cout * (g.Kpad / 4), 256, nsm);
   prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
-                                                     d->cout, g.K, g.Kpad, g.kwords);
+                                                     d->cout, g.K, g.Kpad, g.kwords, 32 / g.sb);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_conv_plan(const ifq_conv_desc* d, int* path) {
+  ConvGeom g;
+  if (!path) return IFQ_EINVAL;
+  int rc = check_conv(d, &g);
+  if (rc) return rc;
+  const int p = choose_path(d, g);
+  if (p < 0) return IFQ_EUNSUPPORTED;
+  *path = p;
+  return IFQ_OK;
 }
 
 int ifq_conv_workspace_bytes(const ifq_conv_desc* d, size_t* bytes) {
@@ -717,24 +781,39 @@ int ifq_graph_destroy(ifq_graph* g) {
   return IFQ_OK;
 }
 
-int ifq_pack_codes(const uint8_t* codes, void* packed, size_t n, void* stream) {
+int ifq_pack_codes_kbits(const uint8_t* codes, void* packed, size_t n, int kbits, void* stream) {
+  int k, sb, lvl, rc;
+  if ((rc = code_width(kbits, &k, &sb, &lvl))) return rc;
   if (!codes || !packed || n % 4 != 0) return IFQ_EINVAL;
-  if ((uintptr_t)codes & 3u) return IFQ_EALIGN;
   if (n == 0) return IFQ_OK;
-  int nsm = 0, rc;
+  int nsm = 0;
   if ((rc = ensure_init(&nsm))) return rc;
-  pack_codes_kernel<<<launch_1d_blocks(n / 4, 256, nsm), 256, 0, S(stream)>>>(codes, (uint8_t*)packed, n / 4);
+  const size_t nb = n * sb / 8;
+  if (sb == 2) pack_codes_kernel<2><<<launch_1d_blocks(nb, 256, nsm), 256, 0, S(stream)>>>(codes, (uint8_t*)packed, nb);
+  else pack_codes_kernel<4><<<launch_1d_blocks(nb, 256, nsm), 256, 0, S(stream)>>>(codes, (uint8_t*)packed, nb);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
-int ifq_unpack_codes(const void* packed, uint8_t* codes, size_t n, void* stream) {
+int ifq_unpack_codes_kbits(const void* packed, uint8_t* codes, size_t n, int kbits, void* stream) {
+  int k, sb, lvl, rc;
+  if ((rc = code_width(kbits, &k, &sb, &lvl))) return rc;
   if (!codes || !packed || n % 4 != 0) return IFQ_EINVAL;
-  if ((uintptr_t)codes & 3u) return IFQ_EALIGN;
   if (n == 0) return IFQ_OK;
-  int nsm = 0, rc;
+  int nsm = 0;
   if ((rc = ensure_init(&nsm))) return rc;
-  unpack_codes_kernel<<<launch_1d_blocks(n / 4, 256, nsm), 256, 0, S(stream)>>>((const uint8_t*)packed, codes, n / 4);
+  const size_t nb = n * sb / 8;
+  const uint8_t* p = (const uint8_t*)packed;
+  if (sb == 2) unpack_codes_kernel<2><<<launch_1d_blocks(nb, 256, nsm), 256, 0, S(stream)>>>(p, codes, nb);
+  else unpack_codes_kernel<4><<<launch_1d_blocks(nb, 256, nsm), 256, 0, S(stream)>>>(p, codes, nb);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_pack_codes(const uint8_t* codes, void* packed, size_t n, void* stream) {
+  return ifq_pack_codes_kbits(codes, packed, n, 2, stream);
+}
+
+int ifq_unpack_codes(const void* packed, uint8_t* codes, size_t n, void* stream) {
+  return ifq_unpack_codes_kbits(packed, codes, n, 2, stream);
 }
 
 int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* stream) {

@@ -23,7 +23,7 @@ extern "C" const char* ifq_status_str(int s) {
   }
 }
 
-extern "C" int ifq_version(void) { return 100; }
+extern "C" int ifq_version(void) { return 200; }   // 2.0: k-bit descriptors (kbits fields)
 
 // Eq. (3)'s uniform level i (1-based) in the compact form of Sec. 3.2.
 static inline double level(int i, double q_base, double q_offset) { return (double)i * q_base + q_offset; }
@@ -138,6 +138,16 @@ extern "C" int ifq_codes_bytes(int n, int h, int w, int c, int kbits, size_t* by
   if (!bytes || n < 0 || h < 0 || w < 0 || c < 0 || kbits < 1 || kbits > 32) return IFQ_EINVAL;
   const unsigned long long bits = (unsigned long long)n * h * w * c * (unsigned long long)kbits;
   *bytes = (size_t)((bits + 7) / 8);
+  return IFQ_OK;
+}
+
+extern "C" int ifq_codes_storage_bytes(int n, int h, int w, int c, int kbits, size_t* bytes) {
+  if (!bytes || n < 0 || h < 0 || w < 0 || c < 0 || kbits < 0) return IFQ_EINVAL;
+  const int k = kbits == 0 ? 2 : kbits;
+  if (k < 2 || k > 4) return IFQ_EUNSUPPORTED;
+  if (c % 4 != 0) return IFQ_ESHAPE;
+  const unsigned long long f = k == 2 ? 2 : 4;
+  *bytes = (size_t)((unsigned long long)n * h * w * c * f / 8);
   return IFQ_OK;
 }
 

@@ -1,5 +1,5 @@
-// 2-bit max pooling (Sec. 2.1 placement, on codes with channel signs) and the
-// packing / filter-preparation kernels.
+// Max pooling of packed codes (Sec. 2.1 placement, on codes with channel signs)
+// and the packing / filter-preparation kernels.
 #pragma once
 #include <cstdint>
 
@@ -9,35 +9,46 @@ namespace ifq {
 
 // ---------------------------------------------------------------- pooling
 //
-// Channel c of a pixel is the 2-bit lane c%4 of byte c/4.  With a channel
-// sign of -1 the pool takes the min of the codes; min(a, b) = 3 - max(3-a, 3-b)
-// and 3 - x = x ^ 3 on a 2-bit lane, so flipping those lanes (XOR with a
-// per-channel mask), taking a plain lane-wise max, and flipping back gives
+// Channel c of a pixel is the SB-bit field c % (8/SB) of byte c / (8/SB) (SB = 2,
+// or 4 for 3- and 4-bit codes).  With a channel sign of -1 the pool takes the
+// min of the codes; with F = 2^SB - 1, min(a, b) = F - max(F-a, F-b) and
+// F - x = x ^ F on an SB-bit field, so flipping those fields (XOR with a
+// per-channel mask), taking a plain field-wise max, and flipping back gives
 // both cases with one max.
 
-// lane-wise max of 16 two-bit lanes, kept as four groups of byte lanes
-struct Lanes4 {
-  uint32_t g[4];
+// field-wise max of the 32/SB fields of a word, kept as 8/SB groups of byte lanes
+template <int SB>
+struct Lanes {
+  static constexpr int kG = 8 / SB;
+  static constexpr uint32_t kMask = SB == 2 ? 0x03030303u : 0x0F0F0F0Fu;
+  uint32_t g[kG];
 };
-__device__ __forceinline__ void lanes_split(uint32_t v, Lanes4& L) {
+template <int SB>
+__device__ __forceinline__ void lanes_split(uint32_t v, Lanes<SB>& L) {
 #pragma unroll
-  for (int s = 0; s < 4; ++s) L.g[s] = (v >> (2 * s)) & 0x03030303u;
+  for (int s = 0; s < Lanes<SB>::kG; ++s) L.g[s] = (v >> (SB * s)) & Lanes<SB>::kMask;
 }
-__device__ __forceinline__ void lanes_max(Lanes4& acc, uint32_t v) {
+template <int SB>
+__device__ __forceinline__ void lanes_max(Lanes<SB>& acc, uint32_t v) {
 #pragma unroll
-  for (int s = 0; s < 4; ++s) acc.g[s] = __vmaxu4(acc.g[s], (v >> (2 * s)) & 0x03030303u);
+  for (int s = 0; s < Lanes<SB>::kG; ++s) acc.g[s] = __vmaxu4(acc.g[s], (v >> (SB * s)) & Lanes<SB>::kMask);
 }
-__device__ __forceinline__ uint32_t lanes_join(const Lanes4& L) {
-  return L.g[0] | (L.g[1] << 2) | (L.g[2] << 4) | (L.g[3] << 6);
+template <int SB>
+__device__ __forceinline__ uint32_t lanes_join(const Lanes<SB>& L) {
+  uint32_t v = 0;
+#pragma unroll
+  for (int s = 0; s < Lanes<SB>::kG; ++s) v |= L.g[s] << (SB * s);
+  return v;
 }
 
-// mask word for the 16 channels of word `wi` of a pixel: lanes of sign -1 channels are 0b11
+// mask of the N fields of channels c0 .. c0+N-1: all ones in the fields of sign -1 channels
+template <int SB, int N>
 __device__ __forceinline__ uint32_t flip_mask(const int8_t* sign, int c0, int c) {
   if (!sign) return 0u;
   uint32_t m = 0;
 #pragma unroll
-  for (int j = 0; j < 16; ++j)
-    if (c0 + j < c && sign[c0 + j] < 0) m |= 3u << (2 * j);
+  for (int j = 0; j < N; ++j)
+    if (c0 + j < c && sign[c0 + j] < 0) m |= ((1u << SB) - 1u) << (SB * j);
   return m;
 }
 
@@ -48,12 +59,14 @@ struct PoolArgs {
   int n, h, w, c, k, stride, pad, ho, wo;
 };
 
-// U = 32-bit words handled per thread (4: 64 channels, 1: 16 channels).
-template <int U>
-__global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
+// U = 32-bit words handled per thread (4 or 1); needs the packed bytes of a pixel to be a
+// multiple of 4U.
+template <int U, int SB>
+__global__ void __launch_bounds__(256) maxpool_codes_kernel(const PoolArgs a) {
   grid_dep_launch();
   grid_dep_wait();
-  const int cw = a.c >> 4;                  // 32-bit words per pixel (c % 16 == 0)
+  constexpr int kCpw = 32 / SB;             // codes per word
+  const int cw = a.c / kCpw;                // 32-bit words per pixel
   const int groups = cw / U;
   const long total = (long)a.n * a.ho * a.wo * groups;
   for (long it = (long)blockIdx.x * blockDim.x + threadIdx.x; it < total; it += (long)gridDim.x * blockDim.x) {
@@ -65,8 +78,8 @@ __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
     const int b = (int)(t / a.ho);
     uint32_t mask[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) mask[u] = flip_mask(a.sign, (gi * U + u) * 16, a.c);
-    Lanes4 acc[U];
+    for (int u = 0; u < U; ++u) mask[u] = flip_mask<SB, kCpw>(a.sign, (gi * U + u) * kCpw, a.c);
+    Lanes<SB> acc[U];
     bool first = true;
     for (int dy = 0; dy < a.k; ++dy) {
       const int iy = oy * a.stride + dy;
@@ -74,7 +87,7 @@ __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
       for (int dx = 0; dx < a.k; ++dx) {
         const int ix = ox * a.stride + dx;
         if (ix >= a.w) continue;
-        const uint32_t* src = (const uint32_t*)(a.x + (((size_t)b * a.h + iy) * a.w + ix) * (size_t)(a.c >> 2)) + gi * U;
+        const uint32_t* src = (const uint32_t*)(a.x + (((size_t)b * a.h + iy) * a.w + ix) * (size_t)(cw * 4)) + gi * U;
         uint32_t v[U];
         if constexpr (U == 4) {
           const uint4 q = __ldg((const uint4*)src);
@@ -91,7 +104,7 @@ __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
         first = false;
       }
     }
-    uint32_t* dst = (uint32_t*)(a.y + (size_t)pix * (a.c >> 2)) + gi * U;
+    uint32_t* dst = (uint32_t*)(a.y + (size_t)pix * (cw * 4)) + gi * U;
     uint32_t o[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) o[u] = lanes_join(acc[u]) ^ mask[u];
@@ -103,11 +116,13 @@ __global__ void __launch_bounds__(256) maxpool2bit_kernel(const PoolArgs a) {
   }
 }
 
-// byte-granular variant for c % 16 != 0 (c % 4 == 0)
-__global__ void __launch_bounds__(256) maxpool2bit_bytes_kernel(const PoolArgs a) {
+// byte-granular variant for any c % 4 == 0
+template <int SB>
+__global__ void __launch_bounds__(256) maxpool_codes_bytes_kernel(const PoolArgs a) {
   grid_dep_launch();
   grid_dep_wait();
-  const int cb = a.c >> 2;
+  constexpr int kCpb = 8 / SB;
+  const int cb = a.c / kCpb;
   const long total = (long)a.n * a.ho * a.wo * cb;
   for (long it = (long)blockIdx.x * blockDim.x + threadIdx.x; it < total; it += (long)gridDim.x * blockDim.x) {
     const int bi = (int)(it % cb);
@@ -116,11 +131,8 @@ __global__ void __launch_bounds__(256) maxpool2bit_bytes_kernel(const PoolArgs a
     const long t = pix / a.wo;
     const int oy = (int)(t % a.ho);
     const int b = (int)(t / a.ho);
-    uint32_t mask = 0;
-    if (a.sign)
-      for (int j = 0; j < 4; ++j)
-        if (a.sign[bi * 4 + j] < 0) mask |= 3u << (2 * j);
-    Lanes4 acc;
+    const uint32_t mask = flip_mask<SB, kCpb>(a.sign, bi * kCpb, a.c);
+    Lanes<SB> acc;
     bool first = true;
     for (int dy = 0; dy < a.k; ++dy) {
       const int iy = oy * a.stride + dy;
@@ -140,17 +152,25 @@ __global__ void __launch_bounds__(256) maxpool2bit_bytes_kernel(const PoolArgs a
 
 // ---------------------------------------------------------------- packing
 
+// one code per byte <-> SB-bit fields, 8/SB codes per packed byte (codes keep their low SB bits)
+template <int SB>
 __global__ void pack_codes_kernel(const uint8_t* codes, uint8_t* packed, size_t nbytes) {
+  constexpr int kCpb = 8 / SB;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nbytes; i += (size_t)gridDim.x * blockDim.x) {
-    const uchar4 c = *(const uchar4*)(codes + 4 * i);
-    packed[i] = (uint8_t)((c.x & 3) | ((c.y & 3) << 2) | ((c.z & 3) << 4) | ((c.w & 3) << 6));
+    uint32_t v = 0;
+#pragma unroll
+    for (int l = 0; l < kCpb; ++l) v |= ((uint32_t)codes[kCpb * i + l] & ((1u << SB) - 1u)) << (SB * l);
+    packed[i] = (uint8_t)v;
   }
 }
 
+template <int SB>
 __global__ void unpack_codes_kernel(const uint8_t* packed, uint8_t* codes, size_t nbytes) {
+  constexpr int kCpb = 8 / SB;
   for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < nbytes; i += (size_t)gridDim.x * blockDim.x) {
     const uint32_t v = packed[i];
-    *(uchar4*)(codes + 4 * i) = make_uchar4(v & 3, (v >> 2) & 3, (v >> 4) & 3, (v >> 6) & 3);
+#pragma unroll
+    for (int l = 0; l < kCpb; ++l) codes[kCpb * i + l] = (uint8_t)((v >> (SB * l)) & ((1u << SB) - 1u));
   }
 }
 
@@ -168,10 +188,11 @@ __global__ void pack_signs_kernel(const int8_t* w, uint32_t* bits, int rows, int
 }
 
 // Prepared filter: e4m3 rows [cout][Kpad] in the chunk order of the
-// tensor-core A expansion (byte p of chunk j holds k = 16j + 4*(p%4) + p/4),
+// tensor-core A expansion: with cpw codes per packed word (16 for 2-bit, 8 for
+// 4-bit fields), byte p of chunk j holds k = cpw*j + (cpw/4)*(p%4) + p/4;
 // +1 -> 0x38, -1 -> 0xB8, k >= K -> 0; followed by a copy of the sign words.
 __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_t* bits_copy, int cout, int K,
-                                    int Kpad, int kwords) {
+                                    int Kpad, int kwords, int cpw) {
   const long total = (long)cout * (Kpad / 4);
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
     const int n = (int)(i / (Kpad / 4));
@@ -180,8 +201,8 @@ __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       const int pos = p4 + t;
-      const int j = pos >> 4, p = pos & 15;
-      const int k = 16 * j + 4 * (p & 3) + (p >> 2);
+      const int j = pos / cpw, p = pos - j * cpw;
+      const int k = cpw * j + (cpw >> 2) * (p & 3) + (p >> 2);
       uint32_t byte = 0;
       if (k < K) byte = ((bits[(size_t)n * kwords + (k >> 5)] >> (k & 31)) & 1u) ? 0x38u : 0xB8u;
       out |= byte << (8 * t);

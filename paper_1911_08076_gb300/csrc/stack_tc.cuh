@@ -181,8 +181,8 @@ __device__ __forceinline__ bool stack_gather_layer(const ConvArgs& a, const int2
       ok = warp_wait_ready(sReady, (uint32_t)(gt_base + l_tile + 1), lane) && ok;
       waited = l_tile;
     }
-    lo = load_unit<GB, true>(tab, g, l_k, 0);
-    hi = load_unit<GB, true>(tab, g, l_k, 1);
+    lo = load_unit<GB, true>(tab, g, 2 * l_k);
+    hi = load_unit<GB, true>(tab, g, 2 * l_k + 1);
     l_k += kGatherGroups;
     if (l_k >= nk) {
       do { l_k -= nk; ++l_tile; } while (l_k >= nk);

@@ -33,11 +33,11 @@ class IfqError(RuntimeError):
 
 class ConvDesc(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int) for f in
-                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path", "pool")]
+                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path", "pool", "kbits")]
 
 
 class PoolDesc(ctypes.Structure):
-    _fields_ = [(f, ctypes.c_int) for f in ("n", "h", "w", "c", "k", "stride", "pad")]
+    _fields_ = [(f, ctypes.c_int) for f in ("n", "h", "w", "c", "k", "stride", "pad", "kbits")]
 
 
 class Layer(ctypes.Structure):
@@ -57,9 +57,11 @@ _SIGS = {
     "ifq_fold_layer": ([_I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
     "ifq_fold_layer_separated": ([_I, _I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
     "ifq_codes_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
+    "ifq_codes_storage_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
     "ifq_conv_out_shape": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
     "ifq_weights_prep_bytes": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_SZ)], _I),
     "ifq_pack_weights": ([ctypes.POINTER(ConvDesc), _P, _P, _P], _I),
+    "ifq_conv_plan": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_I)], _I),
     "ifq_conv_workspace_bytes": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_SZ)], _I),
     "ifq_conv2bit": ([ctypes.POINTER(ConvDesc), _P, _P, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ifq_pool_out_shape": ([ctypes.POINTER(PoolDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
@@ -72,6 +74,8 @@ _SIGS = {
     "ifq_graph_destroy": ([_P], _I),
     "ifq_pack_codes": ([_P, _P, _SZ, _P], _I),
     "ifq_unpack_codes": ([_P, _P, _SZ, _P], _I),
+    "ifq_pack_codes_kbits": ([_P, _P, _SZ, _I, _P], _I),
+    "ifq_unpack_codes_kbits": ([_P, _P, _SZ, _I, _P], _I),
     "ifq_pack_signs": ([_P, _P, _I, _I, _P], _I),
     "ifq_device_status": ([_P, ctypes.POINTER(_I)], _I),
 }
@@ -172,8 +176,19 @@ def ifq_codes_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> int:
     return out.value
 
 
-def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None, pool=0):
-    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path, pool)
+def ifq_codes_storage_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> int:
+    out = _SZ()
+    _ok(lib().ifq_codes_storage_bytes(n, h, w, c, kbits, ctypes.byref(out)), "ifq_codes_storage_bytes")
+    return out.value
+
+
+def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None, pool=0,
+              kbits=2):
+    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path, pool, kbits)
+
+
+def pool_desc(n, h, w, c, k, stride, pad=0, kbits=2):
+    return PoolDesc(n, h, w, c, k, stride, pad, kbits)
 
 
 def ifq_conv_out_shape(d: ConvDesc):
@@ -186,6 +201,12 @@ def ifq_pool_out_shape(d: PoolDesc):
     ho, wo = _I(), _I()
     _ok(lib().ifq_pool_out_shape(ctypes.byref(d), ctypes.byref(ho), ctypes.byref(wo)), "ifq_pool_out_shape")
     return ho.value, wo.value
+
+
+def ifq_conv_plan(d: ConvDesc) -> int:
+    p = _I()
+    _ok(lib().ifq_conv_plan(ctypes.byref(d), ctypes.byref(p)), "ifq_conv_plan")
+    return p.value
 
 
 def ifq_weights_prep_bytes(d: ConvDesc) -> int:
@@ -258,6 +279,14 @@ def ifq_pack_codes(codes, packed, n: int, stream=None):
 
 def ifq_unpack_codes(packed, codes, n: int, stream=None):
     _ok(lib().ifq_unpack_codes(_ptr(packed), _ptr(codes), n, _stream(stream)), "ifq_unpack_codes")
+
+
+def ifq_pack_codes_kbits(codes, packed, n: int, kbits: int, stream=None):
+    _ok(lib().ifq_pack_codes_kbits(_ptr(codes), _ptr(packed), n, kbits, _stream(stream)), "ifq_pack_codes_kbits")
+
+
+def ifq_unpack_codes_kbits(packed, codes, n: int, kbits: int, stream=None):
+    _ok(lib().ifq_unpack_codes_kbits(_ptr(packed), _ptr(codes), n, kbits, _stream(stream)), "ifq_unpack_codes_kbits")
 
 
 def ifq_pack_signs(w, bits, rows: int, K: int, stream=None):

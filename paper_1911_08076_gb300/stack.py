@@ -18,8 +18,11 @@ from . import ifq
 
 class DeviceStack:
     def __init__(self, workload, params, batch: Optional[int] = None, device: str = "cuda", path: int = 0,
-                 kbits: int = 2):
+                 kbits: Optional[int] = None):
         self.wl = workload
+        kbits = getattr(workload, "kbits", 2) if kbits is None else kbits
+        self.kbits = kbits
+        fb = 2 if kbits == 2 else 4          # bits of a code's storage field
         self.batch = workload.batch if batch is None else batch
         self.device = torch.device(device)
         self.thr: Dict[int, torch.Tensor] = {}
@@ -38,7 +41,8 @@ class DeviceStack:
             if l.kind == "conv":
                 p = params[li]
                 mode = {"codes": ifq.IFQ_OUT_CODES, "acc": ifq.IFQ_OUT_ACC, "both": ifq.IFQ_OUT_BOTH}[l.out]
-                d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path, pool=l.pool)
+                d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path, pool=l.pool,
+                                  kbits=kbits)
                 K = l.k * l.k * l.cin
                 T, s = ifq.ifq_fold_layer(K, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias, p.eps,
                                           p.q_base, p.q_offset, kbits)
@@ -55,7 +59,8 @@ class DeviceStack:
                 ho, wo = ifq.ifq_conv_out_shape(d)   # after the fused pool, if any
                 assert (ho, wo) == (l.out_h, l.out_w), (l.name, ho, wo)
                 if mode & ifq.IFQ_OUT_CODES:
-                    self.y_codes[li] = torch.empty((B, ho, wo, l.cout // 4), dtype=torch.uint8, device=self.device)
+                    self.y_codes[li] = torch.empty((B, ho, wo, l.cout * fb // 8), dtype=torch.uint8,
+                                                   device=self.device)
                 if mode & ifq.IFQ_OUT_ACC:
                     self.y_acc[li] = torch.empty((B, ho, wo, l.cout), dtype=torch.int32, device=self.device)
                 rec.conv = d
@@ -65,10 +70,10 @@ class DeviceStack:
                 rec.y_codes = self.y_codes[li].data_ptr() if li in self.y_codes else None
                 rec.y_acc = self.y_acc[li].data_ptr() if li in self.y_acc else None
             else:
-                d = ifq.PoolDesc(B, l.h, l.w, l.c, l.k, l.stride, l.pad)
+                d = ifq.pool_desc(B, l.h, l.w, l.c, l.k, l.stride, l.pad, kbits)
                 ho, wo = ifq.ifq_pool_out_shape(d)
                 assert (ho, wo) == (l.ho, l.wo), (l.name, ho, wo)
-                self.y_codes[li] = torch.empty((B, ho, wo, l.c // 4), dtype=torch.uint8, device=self.device)
+                self.y_codes[li] = torch.empty((B, ho, wo, l.c * fb // 8), dtype=torch.uint8, device=self.device)
                 rec.pool = d
                 rec.sign = self.sign[l.src].data_ptr() if l.signed else None
                 rec.y_codes = self.y_codes[li].data_ptr()
@@ -79,7 +84,8 @@ class DeviceStack:
 
     def input_buffer(self) -> torch.Tensor:
         wl = self.wl
-        return torch.empty((self.batch, wl.h, wl.w, wl.c // 4), dtype=torch.uint8, device=self.device)
+        fb = 2 if self.kbits == 2 else 4
+        return torch.empty((self.batch, wl.h, wl.w, wl.c * fb // 8), dtype=torch.uint8, device=self.device)
 
     def forward(self, x: torch.Tensor, stream=None):
         ifq.ifq_forward(self.layers, x, self.ws, self.ws_bytes, stream)

@@ -4,19 +4,20 @@ This module holds no arithmetic of the method (no convolution, no folding, no
 thresholding).  It provides:
 
 * the layer tables of the benchmark workloads, written out with literal shapes;
-* seeded draws of 2-bit input codes, +-1 filters and the float parameters that
+* seeded draws of k-bit input codes, +-1 filters and the float parameters that
   the integrated conversion folds (alpha, BN, quantizer step);
 * the packed storage formats:
-    - 2-bit codes, NHWC, four codes per byte along C, channel c in bits
-      2*(c%4)..2*(c%4)+1 of byte c//4;
+    - k-bit codes, NHWC, in f-bit fields along C (f = 2 for k = 2, f = 4 for
+      k = 3 and 4), channel c in bits f*(c%(8/f)).. of byte c//(8/f);
     - sign bits of +-1 filters, one row per output channel over K = kh*kw*cin
       in (dy, dx, c) order, bit k%32 of 32-bit word k//32 set for +1, rows
       padded to whole words.
 
 Shapes stand in for the paper's workloads: AlexNet conv2..FC7 (Table 1,
-Sec. 4.1), Tiny-YOLO / Tinier-YOLO backbones (Sec. 4.2) and a ResNet-18 stack;
-the datasets and trained weights are not used.  Distributions: codes uniform
-on {0..3}, weights uniform +-1, alpha ~ U(0.5, 1.5), gamma ~ N(1, 0.3),
+Sec. 4.1; the k = 3 and 4 networks of Table 2 as alexnet_k3 / alexnet_k4),
+Tiny-YOLO / Tinier-YOLO backbones (Sec. 4.2) and a ResNet-18 stack; the
+datasets and trained weights are not used.  Distributions: codes uniform on
+{0..2^k-1}, weights uniform +-1, alpha ~ U(0.5, 1.5), gamma ~ N(1, 0.3),
 beta ~ N(0, 0.5), mean ~ N(0, 2), var ~ U(0.5, 2), quantizer step 0.5,
 bias 0, eps 1e-5, seed 1911_08076 + config index.  For the separated-conversion
 study, draw_conv_params_calibrated gives trained-layer ranges instead (small
@@ -95,6 +96,7 @@ class Workload:
     w: int
     c: int
     layers: list
+    kbits: int = 2      # code width k of every quantized layer's input and output codes
 
     @property
     def seed(self) -> int:
@@ -210,7 +212,13 @@ def fuse_pools(wl: Workload) -> Workload:
             out.append(Conv(l.name, l.cin, l.cout, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.out, p))
         else:
             out.append(Pool(l.name, l.c, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.signed))
-    return Workload(wl.name + "_fused", wl.index, wl.batch, wl.h, wl.w, wl.c, out)
+    return Workload(wl.name + "_fused", wl.index, wl.batch, wl.h, wl.w, wl.c, out, wl.kbits)
+
+
+def with_kbits(wl: Workload, kbits: int) -> Workload:
+    """The same stack with k-bit codes between layers (Table 2's k = 3, 4 columns; Eq. (8)).
+    Same index, so the same filter and parameter draws."""
+    return Workload(f"{wl.name}_k{kbits}", wl.index, wl.batch, wl.h, wl.w, wl.c, wl.layers, kbits)
 
 
 WORKLOADS = {
@@ -223,6 +231,10 @@ WORKLOADS = {
     "tinieryolo_fused": lambda batch=64: fuse_pools(tiny_yolo(batch, True)),
     "roofline3x3": lambda batch=256: roofline(batch, "3x3"),
     "roofline1x1": lambda batch=256: roofline(batch, "1x1"),
+    "alexnet_k3": lambda batch=128: with_kbits(alexnet(batch), 3),
+    "alexnet_k4": lambda batch=128: with_kbits(alexnet(batch), 4),
+    "resnet18_k4": lambda batch=32: with_kbits(resnet18(batch), 4),
+    "tinyyolo_fused_k4": lambda batch=64: with_kbits(fuse_pools(tiny_yolo(batch, False)), 4),
 }
 
 
@@ -277,8 +289,8 @@ def draw_conv_params_calibrated(rng: np.random.Generator, layer: Conv) -> ConvPa
     return ConvParams(w, alpha, gamma, beta, mean, var)
 
 
-def draw_codes(rng: np.random.Generator, shape) -> np.ndarray:
-    return rng.integers(0, 4, size=shape, dtype=np.uint8)
+def draw_codes(rng: np.random.Generator, shape, kbits: int = 2) -> np.ndarray:
+    return rng.integers(0, 1 << kbits, size=shape, dtype=np.uint8)
 
 
 def draw_workload(wl: Workload, batch: Optional[int] = None):
@@ -286,24 +298,39 @@ def draw_workload(wl: Workload, batch: Optional[int] = None):
     rng = np.random.default_rng(wl.seed)
     params = [draw_conv_params(rng, l) if l.kind == "conv" else None for l in wl.layers]
     b = wl.batch if batch is None else batch
-    x = draw_codes(rng, (b, wl.h, wl.w, wl.c))
+    x = draw_codes(rng, (b, wl.h, wl.w, wl.c), wl.kbits)
     return x, params
 
 
 # ----------------------------------------------------------------------------- formats
 
-def pack_codes(codes: np.ndarray) -> np.ndarray:
-    """uint8 codes [..., C] (C % 4 == 0) -> packed uint8 [..., C/4]."""
+def field_bits(kbits: int) -> int:
+    """Bits of the storage field of a k-bit code: 2 for k = 2, 4 for k = 3 and 4."""
+    assert kbits in (2, 3, 4), kbits
+    return 2 if kbits == 2 else 4
+
+
+def pack_codes(codes: np.ndarray, kbits: int = 2) -> np.ndarray:
+    """uint8 codes [..., C] (C % 4 == 0, values < 2^kbits) -> packed uint8 [..., C*f/8]."""
+    f = field_bits(kbits)
     c = np.ascontiguousarray(codes, dtype=np.uint8)
     assert c.shape[-1] % 4 == 0
-    q = c.reshape(c.shape[:-1] + (c.shape[-1] // 4, 4))
-    return (q[..., 0] | (q[..., 1] << 2) | (q[..., 2] << 4) | (q[..., 3] << 6)).astype(np.uint8)
+    assert c.size == 0 or int(c.max()) < (1 << kbits)
+    per = 8 // f
+    q = c.reshape(c.shape[:-1] + (c.shape[-1] // per, per))
+    out = np.zeros(q.shape[:-1], dtype=np.uint8)
+    for l in range(per):
+        out |= (q[..., l] << (f * l)).astype(np.uint8)
+    return out
 
 
-def unpack_codes(packed: np.ndarray, c: Optional[int] = None) -> np.ndarray:
-    """packed uint8 [..., C/4] -> uint8 codes [..., C] (optionally cut to c channels)."""
+def unpack_codes(packed: np.ndarray, c: Optional[int] = None, kbits: int = 2) -> np.ndarray:
+    """packed uint8 [..., C*f/8] -> uint8 codes [..., C] (optionally cut to c channels)."""
+    f = field_bits(kbits)
+    per = 8 // f
     p = np.ascontiguousarray(packed, dtype=np.uint8)
-    out = np.stack([(p >> s) & 3 for s in (0, 2, 4, 6)], axis=-1).reshape(p.shape[:-1] + (p.shape[-1] * 4,))
+    out = np.stack([(p >> (f * l)) & ((1 << f) - 1) for l in range(per)], axis=-1)
+    out = out.reshape(p.shape[:-1] + (p.shape[-1] * per,))
     return out if c is None else out[..., :c]
 
 

@@ -120,6 +120,43 @@ def test_fold_on_workload_parameters(wl_name):
         assert (np.diff(T, axis=1) >= 0).all()
 
 
+@pytest.mark.parametrize("kbits", [2, 3, 4])
+def test_kbit_fold_is_floor_of_compact_thresholds(kbits):
+    """Eq. (8): with uniform levels thr_i = i*base + offset, the composed thresholds lie on one
+    line, thr'_i = i*base' + offset' with base' = sigma*base/(alpha*delta) and
+    offset' = (theta - b + sigma*(offset - beta))/(alpha*delta), sigma = sqrt(var + eps)/gamma
+    (the BN shift beta moves the offset), and the integer thresholds are their floors
+    (gamma > 0) or the floors of -thr'_i (gamma < 0, compared with -A).  The compact form is
+    evaluated here from the inputs in 40-digit decimal arithmetic, independently of the oracle's
+    per-threshold double arithmetic; values within 1e-9 of an integer (where double rounding may
+    decide) are skipped and counted."""
+    from decimal import Decimal, getcontext
+    getcontext().prec = 40
+    rng = np.random.default_rng(300 + kbits)
+    K, cout = 576, 96
+    p = _random_params(rng, cout, kbits=kbits)
+    p.alpha = p.alpha * (4.0 / np.sqrt(K))
+    T, s = O.fold(p, K)
+    L, amax = p.levels, p.levels * K
+    D = lambda v: Decimal(float(v))
+    skipped = 0
+    for n in range(cout):
+        sigma = (D(p.var[n]) + D(p.eps)).sqrt() / D(p.gamma[n])
+        ad = D(p.alpha[n]) * D(p.delta_in)
+        base_c = sigma * D(p.q_base) / ad
+        off_c = (D(p.mean[n]) - D(p.bias[n]) + sigma * (D(p.q_offset) - D(p.beta[n]))) / ad
+        assert s[n] == (1 if p.gamma[n] > 0 else -1)
+        for i in range(1, L + 1):
+            t = i * base_c + off_c
+            v = t if p.gamma[n] > 0 else -t
+            fl = int(v.to_integral_value(rounding="ROUND_FLOOR"))
+            if abs(v - v.to_integral_value(rounding="ROUND_HALF_EVEN")) < Decimal("1e-9") * (1 + abs(v)):
+                skipped += 1
+                continue
+            assert T[n, i - 1] == min(max(fl, -amax - 1), amax), (n, i)
+    assert skipped <= 2
+
+
 def test_fold_invariants():
     rng = np.random.default_rng(7)
     K = 576
