@@ -58,15 +58,17 @@ def conv_ops(layer, batch):
     return 2.0 * batch * layer.ho * layer.wo * layer.cout * layer.k * layer.k * layer.cin
 
 
-def alg_bytes(layer, batch):
-    """Bytes the method must move for one conv launch: 2-bit input codes read once, 1-bit
-    filters, 13 B of thresholds+sign per channel, 2-bit output codes (int32 for accumulators),
-    after the fused pool when the launch has one."""
-    inp = batch * layer.h * layer.w * layer.cin / 4
+def alg_bytes(layer, batch, kbits=2):
+    """Bytes the method must move for one conv launch: input codes read once (f/8 bytes per code,
+    f = 2 for k = 2 and 4 for k = 3, 4), 1-bit filters, 4 (2^k - 1) + 1 bytes of thresholds and
+    sign per channel, output codes at f bits (int32 for accumulators), after the fused pool when
+    the launch has one."""
+    cb = synth.field_bits(kbits) / 8
+    inp = batch * layer.h * layer.w * layer.cin * cb
     wts = layer.cout * layer.k * layer.k * layer.cin / 8
-    thr = 13 * layer.cout
+    thr = (4 * ((1 << kbits) - 1) + 1) * layer.cout
     out = batch * layer.out_h * layer.out_w * layer.cout
-    out = out / 4 if layer.out == "codes" else (out * 4 if layer.out == "acc" else out * 4.25)
+    out = out * cb if layer.out == "codes" else (out * 4 if layer.out == "acc" else out * (4 + cb))
     return inp + wts + thr + out
 
 
@@ -192,7 +194,7 @@ def run_reference(args):
         l = wl.layers[li]
         src = x[0:1] if l.src < 0 else outs[l.src]
         inputs[li] = src["codes"] if isinstance(src, dict) else src
-        p = O.Params.from_synth(params[li])
+        p = O.Params.from_synth(params[li], wl.kbits)
         folded[li] = (p,) + O.fold(p, l.k * l.k * l.cin)
     # calibrate the oracle's rate (MAC/s per thread) on a few channels of the first layer
     l0 = wl.layers[convs[0]]
@@ -211,7 +213,7 @@ def run_reference(args):
 
         def one(ch):
             sub = O.Params(p.alpha[ch], p.gamma[ch], p.beta[ch], p.mean[ch], p.var[ch], None, p.delta_in,
-                           p.q_base, p.q_offset, p.eps)
+                           p.q_base, p.q_offset, p.eps, p.kbits)
             A = O.conv_acc(inputs[li], params[li].w[ch], l.stride, l.pad)
             O.check_chains(A, sub, T[ch], s[ch])
 
@@ -270,7 +272,7 @@ def run_ours(args):
     x, params = synth.draw_workload(wl)
     path = {"auto": ifq.IFQ_PATH_AUTO, "tc": ifq.IFQ_PATH_TC, "bitserial": ifq.IFQ_PATH_BITSERIAL}[args.path]
     st = DeviceStack(wl, params, device=str(dev), path=path)
-    x_host = torch.from_numpy(synth.pack_codes(x)).pin_memory()
+    x_host = torch.from_numpy(synth.pack_codes(x, wl.kbits)).pin_memory()
     xd = st.input_buffer()
     xd.copy_(x_host)
     stream = torch.cuda.Stream(device=dev)
@@ -346,7 +348,7 @@ def run_ours(args):
         conv_idx = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
         conv_ms = sum(per_layer_ms[i] for i in conv_idx)
         conv_ops_total = sum(conv_ops(wl.layers[i], B) for i in conv_idx)
-        conv_bytes_total = sum(alg_bytes(wl.layers[i], B) for i in conv_idx)
+        conv_bytes_total = sum(alg_bytes(wl.layers[i], B, wl.kbits) for i in conv_idx)
 
         # ---------------- end to end through the C ABI with host buffers
         leaves = st.leaf_layers()
@@ -384,7 +386,7 @@ def run_ours(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "e4m3xe4m3->f32 (exact integer: u2 codes x +-1 signs)", "data": "synthetic",
+        "dtype": f"e4m3xe4m3->f32 (exact integer: u{wl.kbits} codes x +-1 signs)", "data": "synthetic",
         "config": {"workload": wl.name, "batch_per_gpu": B, "layers": len(wl.layers),
                    "ops_per_step": ops, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "flushed between steps (256 MB write outside the step events)",

@@ -56,12 +56,12 @@ constexpr int kTmemA = 256;      // first tensor-memory column of the A stages
 constexpr int kAhead = 2;        // own K stages of packed codes a gather thread keeps in registers
 
 // SB: bits per stored code (2, or 4 for 3- and 4-bit codes).  Thresholds per column: a float4
-// (3 thresholds and the sign) for SB = 2, 16 floats (15 thresholds, padded with +inf, and the
-// sign) for SB = 4.
+// (3 thresholds and the sign) for SB = 2, five float4 (15 thresholds, padded with +inf, in the
+// order of the 4-ary search, and the sign) for SB = 4.
 template <int BN, int SB = 2>
 struct TcSmem {
   static constexpr int kB = BN * kBK;
-  static constexpr int kThrCol = SB == 2 ? 16 : 64;       // bytes of thresholds per column
+  static constexpr int kThrCol = SB == 2 ? 16 : 80;       // bytes of thresholds per column
   static constexpr int offB = 0;
   static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN columns
   static constexpr int offTab = offThr + 2 * BN * kThrCol; // kMaxTab x int2

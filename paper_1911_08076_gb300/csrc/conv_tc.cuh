@@ -63,15 +63,18 @@ __device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
       : "memory");
 }
 
-// The code of one accumulator against 15 ascending thresholds (t[0..14], +inf past 2^k - 1)
-// and the channel sign (t[15]): #{ i : sign*D > t[i] } by binary search.
-__device__ __forceinline__ uint32_t code15(float d, const float* t) {
-  const float sv = d * t[15];
-  int c = sv > t[7] ? 8 : 0;
-  c += sv > t[c + 3] ? 4 : 0;
-  c += sv > t[c + 1] ? 2 : 0;
-  c += sv > t[c] ? 1 : 0;
-  return (uint32_t)c;
+// The code of one accumulator against 15 ascending thresholds t[0..14] (+inf past 2^k - 1):
+// #{ i : sign*D > t[i] } as a 4-ary search over five float4 per column,
+//   t5[0] = {t3, t7, t11, sign},  t5[1+q] = {t(4q), t(4q+1), t(4q+2), -}  (q = 0..3):
+// q = #{ t3, t7, t11 below sign*D } picks the group of four codes, and the group's three
+// thresholds give the code 4q + #{ t(4q+j) below }.  Two dependent loads, the first one the same
+// for every row of the column.
+__device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
+  const float4 h = t5[0];
+  const float sv = d * h.w;
+  const uint32_t q = (uint32_t)(sv > h.x) + (uint32_t)(sv > h.y) + (uint32_t)(sv > h.z);
+  const float4 g = t5[1 + q];
+  return 4u * q + (uint32_t)(sv > g.x) + (uint32_t)(sv > g.y) + (uint32_t)(sv > g.z);
 }
 
 // GB: bytes per gathered granule: 16, 4 or 1 (the largest that divides the packed bytes of a
@@ -89,8 +92,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sB = sbase + L::offB;
-  float4* sThr = (float4*)(smem + L::offThr);      // SB = 2
-  float* sThr16 = (float*)(smem + L::offThr);       // SB = 4
+  float4* sThr = (float4*)(smem + L::offThr);      // SB = 2: one float4 per column, SB = 4: five
   int2* sTab = (int2*)(smem + L::offTab);
   const uint32_t barBase = sbase + L::offBar;
   // full[s]: the arrivals of the 4 warps of the gather group that owns stage s, plus
@@ -332,11 +334,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
                               (float)args.thr[3 * nn + 2] * (1.0f / 512.0f), (float)args.sign[nn]);
             sThr[tb * BN + c] = v;
           } else {
-            float* t16 = sThr16 + (size_t)(tb * BN + c) * 16;
+            float4* t5 = sThr + (size_t)(tb * BN + c) * 5;
+            auto T = [&](int i) {
+              return has && i < args.lvl ? (float)args.thr[(size_t)args.lvl * nn + i] * (1.0f / 512.0f) : INFINITY;
+            };
+            t5[0] = make_float4(T(3), T(7), T(11), has ? (float)args.sign[nn] : 1.0f);
 #pragma unroll
-            for (int i = 0; i < 15; ++i)
-              t16[i] = has && i < args.lvl ? (float)args.thr[(size_t)args.lvl * nn + i] * (1.0f / 512.0f) : INFINITY;
-            t16[15] = has ? (float)args.sign[nn] : 1.0f;
+            for (int q = 0; q < 4; ++q) t5[1 + q] = make_float4(T(4 * q), T(4 * q + 1), T(4 * q + 2), 0.0f);
           }
         }
         named_bar(1, kEpiWarps * 32);
@@ -346,8 +350,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       if (!ok) continue;
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
-      const float4* th = sThr + tb * BN + c_lo;
-      const float* th16 = sThr16 + (size_t)(tb * BN + c_lo) * 16;
+      const float4* th = sThr + (size_t)(tb * BN + c_lo) * (SB == 2 ? 1 : 5);
       constexpr int kPW = CW * SB / 32;          // 32-bit words of packed codes per thread
       uint32_t packed[kPW];
 #pragma unroll
@@ -385,7 +388,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
               const float sv = a4[j] * tq.w;
               bits |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
             } else {
-              bits |= code15(a4[j], th16 + (c0 + sub + j) * 16) << (4 * j);
+              bits |= code15(a4[j], th + (c0 + sub + j) * 5) << (4 * j);
             }
           }
           const int cabs = n0 + c_lo + c0 + sub;
@@ -420,7 +423,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           for (int h = 0; h < 2; ++h) {
             uint32_t wd = 0;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) wd |= code15(__uint_as_float(v[8 * h + j]), th16 + (c0 + 8 * h + j) * 16) << (4 * j);
+            for (int j = 0; j < 8; ++j) wd |= code15(__uint_as_float(v[8 * h + j]), th + (c0 + 8 * h + j) * 5) << (4 * j);
             packed[c0 / 8 + h] = wd;
           }
         }
