@@ -235,7 +235,8 @@ int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo);
  * composed conv/BN/quantizer map is monotone in the accumulator (increasing
  * for +1, decreasing for -1), this equals quantizing the max of Y^conv.  With
  * sign NULL it is the plain max of the codes (pooling after the quantizer).
- * x, y (device): packed codes of width d->kbits.
+ * x, y (device): packed codes of width d->kbits.  Limit: the output's packed
+ * bytes n*ho*wo*c*f/8 < 2^31 (IFQ_ERANGE).
  */
 int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, void* stream);
 

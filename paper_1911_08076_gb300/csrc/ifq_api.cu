@@ -381,7 +381,29 @@ int check_pool(const ifq_pool_desc* d, int* ho, int* wo, int* sb = nullptr) {
   if (sb) *sb = f;
   if (d->c % 4 != 0 || d->pad >= d->k) return IFQ_ESHAPE;
   if ((long long)d->n * d->h * d->w * d->c >= (1LL << 40)) return IFQ_ERANGE;
+  // the pool kernels index output bytes of codes with 32-bit integers
+  if ((long long)d->n * *ho * *wo * (d->c * f / 8) >= (1LL << 31)) return IFQ_ERANGE;
   return IFQ_OK;
+}
+
+// The word-vector pool kernel for U words per item, field width sb and window k (k = 2, 3 have
+// their own instances that load the whole window first).
+template <int U, int SB>
+cudaError_t launch_pool_u(int k, dim3 grid, const PoolArgs& a, cudaStream_t st) {
+  if (k == 2) return launch_k(maxpool_codes_kernel<U, SB, 2>, grid, dim3(256), 0, st, a);
+  if (k == 3) return launch_k(maxpool_codes_kernel<U, SB, 3>, grid, dim3(256), 0, st, a);
+  return launch_k(maxpool_codes_kernel<U, SB, 0>, grid, dim3(256), 0, st, a);
+}
+
+cudaError_t launch_pool_words(int U, int sb, int k, dim3 grid, const PoolArgs& a, cudaStream_t st) {
+  if (sb == 2) {
+    if (U == 4) return launch_pool_u<4, 2>(k, grid, a, st);
+    if (U == 2) return launch_pool_u<2, 2>(k, grid, a, st);
+    return launch_pool_u<1, 2>(k, grid, a, st);
+  }
+  if (U == 4) return launch_pool_u<4, 4>(k, grid, a, st);
+  if (U == 2) return launch_pool_u<2, 4>(k, grid, a, st);
+  return launch_pool_u<1, 4>(k, grid, a, st);
 }
 
 int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, cudaStream_t st) {
@@ -400,21 +422,20 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   a.ho = ho; a.wo = wo;
   const size_t pix = (size_t)d->n * ho * wo;
   const int pb = d->c * sb / 8;   // packed bytes per pixel
-  const dim3 b256(256);
+  // one vector of 16, 8 or 4 bytes (else one byte) of a pixel per item
+  const int vb = pb % 16 == 0 ? 16 : (pb % 8 == 0 ? 8 : (pb % 4 == 0 ? 4 : 1));
+  a.groups = pb / vb;
+  a.total = (int)(pix * a.groups);
+  a.div_groups = make_fastdiv((uint32_t)a.groups);
+  a.div_wo = make_fastdiv((uint32_t)wo);
+  a.div_ho = make_fastdiv((uint32_t)ho);
+  const dim3 b256(256), grid(launch_1d_blocks((size_t)a.total, 256, nsm));
   cudaError_t e;
-  if (pb % 16 == 0) {
-    const dim3 grid(launch_1d_blocks(pix * (pb / 16), 256, nsm));
-    e = sb == 2 ? launch_k(maxpool_codes_kernel<4, 2>, grid, b256, 0, st, a)
-                : launch_k(maxpool_codes_kernel<4, 4>, grid, b256, 0, st, a);
-  } else if (pb % 4 == 0) {
-    const dim3 grid(launch_1d_blocks(pix * (pb / 4), 256, nsm));
-    e = sb == 2 ? launch_k(maxpool_codes_kernel<1, 2>, grid, b256, 0, st, a)
-                : launch_k(maxpool_codes_kernel<1, 4>, grid, b256, 0, st, a);
-  } else {
-    const dim3 grid(launch_1d_blocks(pix * pb, 256, nsm));
+  if (vb >= 4)
+    e = launch_pool_words(vb / 4, sb, d->k, grid, a, st);
+  else
     e = sb == 2 ? launch_k(maxpool_codes_bytes_kernel<2>, grid, b256, 0, st, a)
                 : launch_k(maxpool_codes_bytes_kernel<4>, grid, b256, 0, st, a);
-  }
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 

@@ -3,7 +3,7 @@
 #pragma once
 #include <cstdint>
 
-#include "ptx.cuh"
+#include "conv_common.cuh"   // FastDiv
 
 namespace ifq {
 
@@ -16,29 +16,18 @@ namespace ifq {
 // per-channel mask), taking a plain field-wise max, and flipping back gives
 // both cases with one max.
 
-// field-wise max of the 32/SB fields of a word, kept as 8/SB groups of byte lanes
+// Field-wise max of two packed words.  2-bit fields (h1 h0): the larger high bit wins, and equal
+// high bits take the OR of the low bits; 4-bit fields: a byte-lane max on the low and on the high
+// nibbles (each masked in place, so no shifts).
 template <int SB>
-struct Lanes {
-  static constexpr int kG = 8 / SB;
-  static constexpr uint32_t kMask = SB == 2 ? 0x03030303u : 0x0F0F0F0Fu;
-  uint32_t g[kG];
-};
-template <int SB>
-__device__ __forceinline__ void lanes_split(uint32_t v, Lanes<SB>& L) {
-#pragma unroll
-  for (int s = 0; s < Lanes<SB>::kG; ++s) L.g[s] = (v >> (SB * s)) & Lanes<SB>::kMask;
-}
-template <int SB>
-__device__ __forceinline__ void lanes_max(Lanes<SB>& acc, uint32_t v) {
-#pragma unroll
-  for (int s = 0; s < Lanes<SB>::kG; ++s) acc.g[s] = __vmaxu4(acc.g[s], (v >> (SB * s)) & Lanes<SB>::kMask);
-}
-template <int SB>
-__device__ __forceinline__ uint32_t lanes_join(const Lanes<SB>& L) {
-  uint32_t v = 0;
-#pragma unroll
-  for (int s = 0; s < Lanes<SB>::kG; ++s) v |= L.g[s] << (SB * s);
-  return v;
+__device__ __forceinline__ uint32_t field_max(uint32_t a, uint32_t b) {
+  if constexpr (SB == 2) {
+    const uint32_t a1 = a & 0xAAAAAAAAu, b1 = b & 0xAAAAAAAAu;
+    const uint32_t ga = (a1 & ~b1) >> 1, gb = (b1 & ~a1) >> 1;   // where a (b) has the larger high bit
+    return a1 | b1 | (((a & ~gb) | (b & ~ga)) & 0x55555555u);
+  } else {
+    return __vmaxu4(a & 0x0F0F0F0Fu, b & 0x0F0F0F0Fu) | __vmaxu4(a & 0xF0F0F0F0u, b & 0xF0F0F0F0u);
+  }
 }
 
 // mask of the N fields of channels c0 .. c0+N-1: all ones in the fields of sign -1 channels
@@ -57,62 +46,107 @@ struct PoolArgs {
   const int8_t* sign;
   uint8_t* y;
   int n, h, w, c, k, stride, pad, ho, wo;
+  int groups;                          // vector groups (of U words or of single bytes) per pixel
+  int total;                           // n * ho * wo * groups (< 2^31)
+  FastDiv div_groups, div_wo, div_ho;
 };
 
-// U = 32-bit words handled per thread (4 or 1); needs the packed bytes of a pixel to be a
-// multiple of 4U.
-template <int U, int SB>
+template <int U>
+struct WordVec;
+template <>
+struct WordVec<1> {
+  static __device__ __forceinline__ void ld(const uint32_t* p, uint32_t* v) { v[0] = __ldg(p); }
+  static __device__ __forceinline__ void st(uint32_t* p, const uint32_t* v) { p[0] = v[0]; }
+};
+template <>
+struct WordVec<2> {
+  static __device__ __forceinline__ void ld(const uint32_t* p, uint32_t* v) {
+    const uint2 q = __ldg((const uint2*)p);
+    v[0] = q.x; v[1] = q.y;
+  }
+  static __device__ __forceinline__ void st(uint32_t* p, const uint32_t* v) { *(uint2*)p = make_uint2(v[0], v[1]); }
+};
+template <>
+struct WordVec<4> {
+  static __device__ __forceinline__ void ld(const uint32_t* p, uint32_t* v) {
+    const uint4 q = __ldg((const uint4*)p);
+    v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+  }
+  static __device__ __forceinline__ void st(uint32_t* p, const uint32_t* v) {
+    *(uint4*)p = make_uint4(v[0], v[1], v[2], v[3]);
+  }
+};
+
+// U = 32-bit words handled per thread (4, 2 or 1, one vector load per window cell); needs the
+// packed bytes of a pixel to be a multiple of 4U.  Item it = pixel * groups + group.  KW = 2 or 3:
+// the k x k window (k == KW) is loaded before it is reduced, so all its loads are in flight
+// together; the top-left cell (oy*stride, ox*stride) is always inside the image, and a cell past
+// the bottom or right edge takes its value (a no-op for the max).  KW = 0: any k, cell by cell.
+// When the grid stride is a multiple of the groups per pixel, a thread's group never changes and
+// its sign masks are built once.
+template <int U, int SB, int KW>
 __global__ void __launch_bounds__(256) maxpool_codes_kernel(const PoolArgs a) {
   grid_dep_launch();
   grid_dep_wait();
   constexpr int kCpw = 32 / SB;             // codes per word
   const int cw = a.c / kCpw;                // 32-bit words per pixel
-  const int groups = cw / U;
-  const long total = (long)a.n * a.ho * a.wo * groups;
-  for (long it = (long)blockIdx.x * blockDim.x + threadIdx.x; it < total; it += (long)gridDim.x * blockDim.x) {
-    const int gi = (int)(it % groups);
-    const long pix = it / groups;
-    const int ox = (int)(pix % a.wo);
-    const long t = pix / a.wo;
-    const int oy = (int)(t % a.ho);
-    const int b = (int)(t / a.ho);
-    uint32_t mask[U];
+  const size_t rowb = (size_t)a.w * (cw * 4);
+  const int stride = gridDim.x * blockDim.x;
+  const bool fixed_group = stride % a.groups == 0;
+  int mask_g = -1;
+  uint32_t mask[U];
+  for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < a.total; it += stride) {
+    const int pix = (int)fdiv((uint32_t)it, a.div_groups);
+    const int gi = it - pix * a.groups;
+    const int t = (int)fdiv((uint32_t)pix, a.div_wo);
+    const int ox = pix - t * a.wo;
+    const int b = (int)fdiv((uint32_t)t, a.div_ho);
+    const int oy = t - b * a.ho;
+    if (gi != mask_g) {
 #pragma unroll
-    for (int u = 0; u < U; ++u) mask[u] = flip_mask<SB, kCpw>(a.sign, (gi * U + u) * kCpw, a.c);
-    Lanes<SB> acc[U];
-    bool first = true;
-    for (int dy = 0; dy < a.k; ++dy) {
-      const int iy = oy * a.stride + dy;
-      if (iy >= a.h) continue;
-      for (int dx = 0; dx < a.k; ++dx) {
-        const int ix = ox * a.stride + dx;
-        if (ix >= a.w) continue;
-        const uint32_t* src = (const uint32_t*)(a.x + (((size_t)b * a.h + iy) * a.w + ix) * (size_t)(cw * 4)) + gi * U;
-        uint32_t v[U];
-        if constexpr (U == 4) {
-          const uint4 q = __ldg((const uint4*)src);
-          v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+      for (int u = 0; u < U; ++u) mask[u] = flip_mask<SB, kCpw>(a.sign, (gi * U + u) * kCpw, a.c);
+      mask_g = fixed_group ? gi : -1;
+    }
+    const int iy0 = oy * a.stride, ix0 = ox * a.stride;
+    const uint8_t* base = a.x + ((size_t)b * a.h + iy0) * rowb + (size_t)ix0 * (cw * 4) + (size_t)gi * (U * 4);
+    uint32_t m[U];                           // the window max of the flipped fields
+    if constexpr (KW > 0) {
+      uint32_t v[KW * KW][U];
+      WordVec<U>::ld((const uint32_t*)base, v[0]);
+#pragma unroll
+      for (int q = 1; q < KW * KW; ++q) {
+        const int dy = q / KW, dx = q % KW;
+        if (iy0 + dy < a.h && ix0 + dx < a.w) {
+          WordVec<U>::ld((const uint32_t*)(base + dy * rowb + (size_t)dx * (cw * 4)), v[q]);
         } else {
 #pragma unroll
-          for (int u = 0; u < U; ++u) v[u] = __ldg(src + u);
+          for (int u = 0; u < U; ++u) v[q][u] = v[0][u];
         }
+      }
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          if (first) lanes_split(v[u] ^ mask[u], acc[u]);
-          else lanes_max(acc[u], v[u] ^ mask[u]);
+      for (int u = 0; u < U; ++u) {
+        m[u] = v[0][u] ^ mask[u];
+#pragma unroll
+        for (int q = 1; q < KW * KW; ++q) m[u] = field_max<SB>(m[u], v[q][u] ^ mask[u]);
+      }
+    } else {
+      bool first = true;
+      for (int dy = 0; dy < a.k; ++dy) {
+        if (iy0 + dy >= a.h) continue;
+        for (int dx = 0; dx < a.k; ++dx) {
+          if (ix0 + dx >= a.w) continue;
+          uint32_t v[U];
+          WordVec<U>::ld((const uint32_t*)(base + dy * rowb + (size_t)dx * (cw * 4)), v);
+#pragma unroll
+          for (int u = 0; u < U; ++u) m[u] = first ? v[u] ^ mask[u] : field_max<SB>(m[u], v[u] ^ mask[u]);
+          first = false;
         }
-        first = false;
       }
     }
     uint32_t* dst = (uint32_t*)(a.y + (size_t)pix * (cw * 4)) + gi * U;
-    uint32_t o[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) o[u] = lanes_join(acc[u]) ^ mask[u];
-    if constexpr (U == 4) *(uint4*)dst = make_uint4(o[0], o[1], o[2], o[3]);
-    else {
-#pragma unroll
-      for (int u = 0; u < U; ++u) dst[u] = o[u];
-    }
+    for (int u = 0; u < U; ++u) m[u] ^= mask[u];
+    WordVec<U>::st(dst, m);
   }
 }
 
@@ -123,16 +157,15 @@ __global__ void __launch_bounds__(256) maxpool_codes_bytes_kernel(const PoolArgs
   grid_dep_wait();
   constexpr int kCpb = 8 / SB;
   const int cb = a.c / kCpb;
-  const long total = (long)a.n * a.ho * a.wo * cb;
-  for (long it = (long)blockIdx.x * blockDim.x + threadIdx.x; it < total; it += (long)gridDim.x * blockDim.x) {
-    const int bi = (int)(it % cb);
-    const long pix = it / cb;
-    const int ox = (int)(pix % a.wo);
-    const long t = pix / a.wo;
-    const int oy = (int)(t % a.ho);
-    const int b = (int)(t / a.ho);
+  for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < a.total; it += gridDim.x * blockDim.x) {
+    const int pix = (int)fdiv((uint32_t)it, a.div_groups);
+    const int bi = it - pix * cb;
+    const int t = (int)fdiv((uint32_t)pix, a.div_wo);
+    const int ox = pix - t * a.wo;
+    const int b = (int)fdiv((uint32_t)t, a.div_ho);
+    const int oy = t - b * a.ho;
     const uint32_t mask = flip_mask<SB, kCpb>(a.sign, bi * kCpb, a.c);
-    Lanes<SB> acc;
+    uint32_t m = 0;
     bool first = true;
     for (int dy = 0; dy < a.k; ++dy) {
       const int iy = oy * a.stride + dy;
@@ -141,12 +174,11 @@ __global__ void __launch_bounds__(256) maxpool_codes_bytes_kernel(const PoolArgs
         const int ix = ox * a.stride + dx;
         if (ix >= a.w) continue;
         const uint32_t v = a.x[(((size_t)b * a.h + iy) * a.w + ix) * cb + bi];
-        if (first) lanes_split(v ^ mask, acc);
-        else lanes_max(acc, v ^ mask);
+        m = first ? v ^ mask : field_max<SB>(m, v ^ mask);
         first = false;
       }
     }
-    a.y[(size_t)pix * cb + bi] = (uint8_t)((lanes_join(acc) ^ mask) & 0xFFu);
+    a.y[(size_t)pix * cb + bi] = (uint8_t)((m ^ mask) & 0xFFu);
   }
 }
 
