@@ -64,7 +64,7 @@ def alg_bytes(layer, batch, kbits=2):
     sign per channel, output codes at f bits (int32 for accumulators), after the fused pool when
     the launch has one."""
     cb = synth.field_bits(kbits) / 8
-    inp = batch * layer.h * layer.w * layer.cin * cb
+    inp = batch * layer.h * layer.w * layer.cin * (1 if getattr(layer, "in_bits", 0) == 8 else cb)
     wts = layer.cout * layer.k * layer.k * layer.cin / 8
     thr = (4 * ((1 << kbits) - 1) + 1) * layer.cout
     out = batch * layer.out_h * layer.out_w * layer.cout
@@ -195,7 +195,7 @@ def run_reference(args):
         src = x[0:1] if l.src < 0 else outs[l.src]
         inputs[li] = src["codes"] if isinstance(src, dict) else src
         p = O.Params.from_synth(params[li], wl.kbits)
-        folded[li] = (p,) + O.fold(p, l.k * l.k * l.cin)
+        folded[li] = (p,) + O.fold(p, O.fold_k(l) if wl.kbits == 2 else l.k * l.k * l.cin)
     # calibrate the oracle's rate (MAC/s per thread) on a few channels of the first layer
     l0 = wl.layers[convs[0]]
     t0 = time.perf_counter()
@@ -309,7 +309,7 @@ def run_ours(args):
     x, params = synth.draw_workload(wl)
     path = {"auto": ifq.IFQ_PATH_AUTO, "tc": ifq.IFQ_PATH_TC, "bitserial": ifq.IFQ_PATH_BITSERIAL}[args.path]
     st = DeviceStack(wl, params, device=str(dev), path=path)
-    x_host = torch.from_numpy(synth.pack_codes(x, wl.kbits)).pin_memory()
+    x_host = torch.from_numpy(synth.pack_codes(x, 8 if wl.in_bits == 8 else wl.kbits)).pin_memory()
     xd = st.input_buffer()
     xd.copy_(x_host)
     stream = torch.cuda.Stream(device=dev)

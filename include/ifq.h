@@ -73,7 +73,7 @@ enum { IFQ_OUT_CODES = 1, IFQ_OUT_ACC = 2, IFQ_OUT_BOTH = 3 };
 enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2 };
 
 /* Layer kinds of ifq_forward. */
-enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2 };
+enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2, IFQ_LAYER_FIXED = 3 };
 
 /* Text for a status code (static storage; never NULL). */
 const char* ifq_status_str(int status);
@@ -152,6 +152,13 @@ int ifq_codes_storage_bytes(int n, int h, int w, int c, int kbits, size_t* bytes
  * kbits: the code width k of the input codes and of the output codes (0
  * means 2; 2, 3 or 4, else IFQ_EUNSUPPORTED); the thresholds are then
  * [cout][2^k - 1] (Eq. (8)).
+ * in_bits: 0 (or kbits) for k-bit input codes; 8 for unsigned 8-bit input
+ * values, one byte each (a first layer on image pixels, whose substructure
+ * the integrated conversion covers as well: binary filters, integer inputs).
+ * An 8-bit input needs cin % 4 == 0 (pad RGB with a zero channel), the
+ * tensor-core path and 255*K <= 196608 (IFQ_EUNSUPPORTED otherwise); its
+ * layer can only read the stack input in ifq_forward, and its fold takes
+ * K_fold = ceil(255*K / (2^k - 1)) so that the clamp covers |A| <= 255*K.
  * pool: 0 or 1 for none; p = 2 or 4 max-pools the convolution output over
  * p x p windows with stride p before the thresholds (Sec. 2.1: the pool acts
  * on Y^conv, before BN and the quantizer), so that the codes are those of the
@@ -167,6 +174,7 @@ typedef struct {
   int path;
   int pool;
   int kbits;
+  int in_bits;
 } ifq_conv_desc;
 
 /* Output spatial size of a conv descriptor (host, pure). */
@@ -241,12 +249,45 @@ int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo);
 int ifq_maxpool2bit(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y, void* stream);
 
 /*
+ * ifq_fold_output_separated -- the separated fixed-point conversion (Sec. 2.2)
+ * of a NON-quantized substructure's output (the linear detection conv of a
+ * YOLO head; AlexNet's last substructure): with Q = 2^m,
+ *   mul[n] = floor(alpha[n]*Q) * floor(delta_in*Q),  add[n] = floor(bias[n]*Q^2)
+ * so that Y^conv = (mul*A + add) / Q^2 is Eq. (1) with every float floored at
+ * its own scale.  Host, pure.  alpha: [cout] > 0, finite; bias: [cout] or NULL;
+ * delta_in > 0; m in 1..24; mul_out, add_out: [cout] int64 (IFQ_EINVAL otherwise).
+ */
+int ifq_fold_output_separated(int cout, int m, const float* alpha, float delta_in, const float* bias,
+                              int64_t* mul_out, int64_t* add_out);
+
+/*
+ * ifq_fixed_output -- the fixed-point value of that output at scale Q = 2^m:
+ *   y[r][n] = floor((mul[n]*A[r][n] + add[n]) / 2^m)   (exact 64-bit integer
+ * arithmetic), saturated to the int32 range, i.e. y/Q is Y^conv with m
+ * fractional bits.  acc (device): int32 [rows][cout]; mul, add (device): int64
+ * [cout] from ifq_fold_output_separated; y (device): int32 [rows][cout];
+ * m in 1..24, rows >= 0, cout >= 1; pointers 8-byte aligned (mul, add) and
+ * 4-byte aligned (acc, y).
+ */
+int ifq_fixed_output(const int32_t* acc, int rows, int cout, const int64_t* mul, const int64_t* add, int m,
+                     int32_t* y, void* stream);
+
+/* Fixed-point output layer of ifq_forward (kind IFQ_LAYER_FIXED). */
+typedef struct {
+  int m;
+} ifq_fixed_desc;
+
+/*
  * One layer of a stack for ifq_forward.  src is the index of the layer whose
  * output codes are this layer's input (-1: the stack input x).  For a conv,
  * `conv`, w_prep, thr and sign describe it and y_codes / y_acc receive its
  * outputs per conv.out_mode; for a pool, `pool` describes it, sign is the
  * pooled layer's channel signs (or NULL for a plain max) and y_codes receives
- * the pooled codes.  All pointers are device pointers owned by the caller.
+ * the pooled codes.  For a fixed-point output (IFQ_LAYER_FIXED), src is a
+ * conv layer that writes int32 accumulators, `fixed`, fx_mul and fx_add
+ * describe the conversion (ifq_fixed_output) and y_acc receives the int32
+ * fixed-point values [rows][cout] of the source conv's shape.  All pointers
+ * are device pointers owned by the caller.
  */
 typedef struct {
   int kind;
@@ -258,6 +299,9 @@ typedef struct {
   const int8_t* sign;
   void* y_codes;
   int32_t* y_acc;
+  ifq_fixed_desc fixed;
+  const int64_t* fx_mul;
+  const int64_t* fx_add;
 } ifq_layer;
 
 /*

@@ -281,3 +281,37 @@ int ifqo_separated_chain(long M, int cout, const int32_t* A, int L, int m, const
   }
   return ORC_OK;
 }
+
+/*
+ * Separated fixed-point conversion of a NON-quantized substructure's output, Sec. 2.2
+ * (the linear detection conv of a YOLO head, AlexNet's substructure 7): with Q = 2^m,
+ *   a = floor(alpha*Q), d = floor(delta_in*Q), bq = floor(bias*Q^2)
+ *   Y^conv = (a*d*A + bq) / Q^2                                  (Eq. (1), each float floored)
+ * and the output kept at Q's scale, m fractional bits:
+ *   y = floor(Y^conv * Q) = floor((a*d*A + bq) / Q)
+ * evaluated exactly in 128-bit integers, then saturated to the int32 range.  m in 1..24.
+ */
+static int32_t sat32(__int128 v) {
+  if (v > (__int128)INT32_MAX) return INT32_MAX;
+  if (v < (__int128)INT32_MIN) return INT32_MIN;
+  return (int32_t)v;
+}
+
+int ifqo_fixed_output(long M, int cout, const int32_t* A, int m, const double* alpha, double delta_in,
+                      const double* bias, int32_t* out) {
+  if (M < 0 || cout <= 0 || m < 1 || m > 24) return ORC_EINVAL;
+  const double Q = ldexp(1.0, m);
+  const int64_t Qi = (int64_t)1 << m;
+  const int64_t d = floor_scaled(delta_in, Q);
+  for (int n = 0; n < cout; ++n) {
+    const int64_t a = floor_scaled(alpha[n], Q);
+    const int64_t bq = (int64_t)floor((bias ? bias[n] : 0.0) * Q * Q);
+    for (long r = 0; r < M; ++r) {
+      const __int128 N = (__int128)a * d * A[r * cout + n] + bq;
+      __int128 y = N / Qi;                              /* C division truncates toward zero */
+      if (N % Qi != 0 && N < 0) y -= 1;                 /* floor */
+      out[r * cout + n] = sat32(y);
+    }
+  }
+  return ORC_OK;
+}

@@ -58,6 +58,7 @@ def lib():
             L.ifqo_maxpool_acc.argtypes = [i, i, i, i, i, i, i, P, P]
             L.ifqo_maxpool_codes.argtypes = [i, i, i, i, i, i, i, P, P, P]
             L.ifqo_separated_chain.argtypes = [l, i, P, i, i, P, d, P, P, P, P, P, d, d, d, P]
+            L.ifqo_fixed_output.argtypes = [l, i, P, i, P, d, P, P]
             for f in ("ifqo_float_chain", "ifqo_fold", "ifqo_int_chain", "ifqo_conv_acc",
                       "ifqo_maxpool_acc", "ifqo_maxpool_codes", "ifqo_separated_chain"):
                 getattr(L, f).restype = ctypes.c_int
@@ -152,6 +153,24 @@ def separated_chain(A: np.ndarray, p: "Params", m: int) -> np.ndarray:
     return codes.reshape(A.shape)
 
 
+def fixed_output(A: np.ndarray, p: "Params", m: int) -> np.ndarray:
+    """Separated fixed-point output of a non-quantized substructure (Sec. 2.2) at Q_m = 2^m:
+    floor((floor(alpha Q) floor(delta Q) A + floor(b Q^2)) / Q), int32 of A's shape."""
+    cout = p.alpha.shape[0]
+    A2 = np.ascontiguousarray(A, dtype=np.int32).reshape(-1, cout)
+    out = np.empty(A2.shape, dtype=np.int32)
+    _check(lib().ifqo_fixed_output(A2.shape[0], cout, _p(A2), m, _p(p.alpha), p.delta_in,
+                                   _p(p.bias) if p.bias is not None else None, _p(out)), "fixed_output")
+    return out.reshape(A.shape)
+
+
+def fold_k(layer) -> int:
+    """K of a layer's fold: its kh*kw*cin, or for a layer on 8-bit input values the K whose
+    clamp range L*K covers every accumulator |A| <= 255*K (L = 3 for 2-bit output codes)."""
+    K = layer.k * layer.k * layer.cin
+    return -(-255 * K // 3) if getattr(layer, "in_bits", 0) == 8 else K
+
+
 def conv_acc(x: np.ndarray, w: np.ndarray, stride: int, pad: int) -> np.ndarray:
     """Integer core of Eq. (1): x uint8 codes [B][H][W][C], w int8 +-1 [cout][kh][kw][C] -> int32 NHWC."""
     x = np.ascontiguousarray(x, dtype=np.uint8)
@@ -226,7 +245,8 @@ def forward(workload, x: np.ndarray, params: Sequence, images: Optional[Sequence
     for li, layer in enumerate(workload.layers):
         if layer.kind == "conv":
             p = Params.from_synth(params[li], kbits)
-            folded[li] = (p, *fold(p, layer.k * layer.k * layer.cin))
+            kf = fold_k(layer) if kbits == 2 else layer.k * layer.k * layer.cin
+            folded[li] = (p, *fold(p, kf))
 
     def one(b):
         outs = {}
@@ -244,6 +264,9 @@ def forward(workload, x: np.ndarray, params: Sequence, images: Optional[Sequence
                 else:
                     codes = int_chain(A, T, s)
                 outs[li] = {"codes": codes, "acc": A} if layer.out == "both" else (A if layer.out == "acc" else codes)
+            elif layer.kind == "fixed":   # the separated fixed-point output of a conv's accumulators
+                acc = outs[layer.src]["acc"] if isinstance(outs[layer.src], dict) else outs[layer.src]
+                outs[li] = fixed_output(acc, folded[layer.src][0], layer.m)
             else:
                 sgn = folded[layer.src][2] if layer.signed else None
                 outs[li] = maxpool_codes(src, layer.k, layer.stride, layer.pad, sgn)

@@ -78,13 +78,14 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
 }
 
 // GB: bytes per gathered granule: 16, 4 or 1 (the largest that divides the packed bytes of a
-// pixel); SB: bits per stored code (2 for k = 2, 4 for k = 3 and 4).
-template <int BN, int GB, int SB>
+// pixel); SB: bits per stored input code (2 for k = 2, 4 for k = 3 and 4 and for the two nibbles of
+// an 8-bit input value); SBO: bits per stored output code (2 or 4).
+template <int BN, int GB, int SB, int SBO>
 __global__ void __launch_bounds__(kConvThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
   static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
-  static_assert(SB == 2 || SB == 4, "stored code width");
-  using L = TcSmem<BN, SB>;
+  static_assert((SB == 2 || SB == 4) && (SBO == 2 || SBO == 4), "stored code width");
+  using L = TcSmem<BN, SBO>;
   constexpr int kU = kBK * SB / 8 / 16;       // 16-byte units of packed codes per K stage
   constexpr int kCpb = 8 / SB;                // codes per byte
   constexpr int kS = kStages;
@@ -92,7 +93,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sB = sbase + L::offB;
-  float4* sThr = (float4*)(smem + L::offThr);      // SB = 2: one float4 per column, SB = 4: five
+  float4* sThr = (float4*)(smem + L::offThr);      // SBO = 2: one float4 per column, SBO = 4: five
   int2* sTab = (int2*)(smem + L::offTab);
   const uint32_t barBase = sbase + L::offBar;
   // full[s]: the arrivals of the 4 warps of the gather group that owns stage s, plus
@@ -327,7 +328,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           const int nn = n0 + c;
           const bool has = nn < args.cout && args.thr;
           // sign*A > T  <=>  sign*D > T/512 with D = A/512 (exact in fp32)
-          if constexpr (SB == 2) {
+          if constexpr (SBO == 2) {
             float4 v = make_float4(0.f, 0.f, 0.f, 1.f);
             if (has)
               v = make_float4((float)args.thr[3 * nn] * (1.0f / 512.0f), (float)args.thr[3 * nn + 1] * (1.0f / 512.0f),
@@ -350,8 +351,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       if (!ok) continue;
       tc_fence_after();
       const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
-      const float4* th = sThr + (size_t)(tb * BN + c_lo) * (SB == 2 ? 1 : 5);
-      constexpr int kPW = CW * SB / 32;          // 32-bit words of packed codes per thread
+      const float4* th = sThr + (size_t)(tb * BN + c_lo) * (SBO == 2 ? 1 : 5);
+      constexpr int kPW = CW * SBO / 32;          // 32-bit words of packed codes per thread
       uint32_t packed[kPW];
 #pragma unroll
       for (int c0 = 0; c0 < CW; c0 += 16) {
@@ -383,7 +384,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           uint32_t bits = 0;
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
-            if constexpr (SB == 2) {
+            if constexpr (SBO == 2) {
               const float4 tq = th[c0 + sub + j];
               const float sv = a4[j] * tq.w;
               bits |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
@@ -393,8 +394,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           }
           const int cabs = n0 + c_lo + c0 + sub;
           if (args.y_codes && m < args.M && cabs < args.cout) {
-            uint8_t* dst = args.y_codes + (size_t)(m >> 2) * ((args.cout * SB) >> 3) + ((cabs * SB) >> 3);
-            if constexpr (SB == 2) *dst = (uint8_t)bits;
+            uint8_t* dst = args.y_codes + (size_t)(m >> 2) * ((args.cout * SBO) >> 3) + ((cabs * SBO) >> 3);
+            if constexpr (SBO == 2) *dst = (uint8_t)bits;
             else *(uint16_t*)dst = (uint16_t)bits;   // cabs % 4 == 0: an even byte offset
           }
           continue;
@@ -408,7 +409,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
             v[j] = __float_as_uint(x);
           }
         }
-        if constexpr (SB == 2) {
+        if constexpr (SBO == 2) {
           uint32_t wd = 0;
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -455,9 +456,9 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       // the pooled pixel m >> 4)
       const bool store = args.y_codes && m < args.M && args.lpool != 1 && (m & ((1 << (2 * args.lpool)) - 1)) == 0;
       if (store) {
-        const int rowb = (args.cout * SB) >> 3;   // bytes per output pixel
+        const int rowb = (args.cout * SBO) >> 3;   // bytes per output pixel
         const int cb = n0 + c_lo;                 // first channel of this thread
-        const int cbb = (cb * SB) >> 3;           // its byte within the pixel
+        const int cbb = (cb * SBO) >> 3;           // its byte within the pixel
         uint8_t* dst = args.y_codes + (size_t)(m >> (2 * args.lpool)) * rowb + cbb;
         if (cb + CW <= args.cout && kPW >= 4 && (rowb & 15) == 0 && (cbb & 15) == 0) {
 #pragma unroll
@@ -468,7 +469,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 #pragma unroll
           for (int q = 0; q < kPW; ++q) *(uint32_t*)(dst + 4 * q) = packed[q];
         } else {
-          const int nbytes = (max(0, min(CW, args.cout - cb)) * SB) >> 3;
+          const int nbytes = (max(0, min(CW, args.cout - cb)) * SBO) >> 3;
 #pragma unroll
           for (int q = 0; q < 4 * kPW; ++q)   // unrolled: packed[] stays in registers
             if (q < nbytes) dst[q] = (uint8_t)(packed[q >> 2] >> (8 * (q & 3)));

@@ -82,28 +82,29 @@ cudaError_t launch_k(void (*kern)(Exp...), dim3 grid, dim3 block, size_t smem, c
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
 }
 
-template <int BN, int GB, int SB>
+template <int BN, int GB, int SB, int SBO>
 struct TcInst {
-  using L = TcSmem<BN, SB>;
+  using L = TcSmem<BN, SBO>;
   static_assert(L::bytes <= 232448, "shared memory budget");
   static cudaError_t set_attr() {
-    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB, SB>, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
+    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB, SB, SBO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                L::bytes);
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
     const int grid = a.ntiles < nsm ? a.ntiles : nsm;
-    return launch_k(conv_tc_kernel<BN, GB, SB>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
+    return launch_k(conv_tc_kernel<BN, GB, SB, SBO>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
   }
 };
 
 // The output-channel tile widths of the tensor-core kernel.
-#define IFQ_TC_VARIANTS(X, GB, SB) X(128, GB, SB) X(64, GB, SB) X(32, GB, SB)
+#define IFQ_TC_VARIANTS(X, GB, SB, SBO) X(128, GB, SB, SBO) X(64, GB, SB, SBO) X(32, GB, SB, SBO)
 
-template <int GB, int SB>
+template <int GB, int SB, int SBO>
 cudaError_t set_attrs_gb() {
   cudaError_t e = cudaSuccess;
-#define IFQ_SET(BN, G, S) \
-  if (e == cudaSuccess) e = TcInst<BN, G, S>::set_attr();
-  IFQ_TC_VARIANTS(IFQ_SET, GB, SB)
+#define IFQ_SET(BN, G, S, SO) \
+  if (e == cudaSuccess) e = TcInst<BN, G, S, SO>::set_attr();
+  IFQ_TC_VARIANTS(IFQ_SET, GB, SB, SBO)
 #undef IFQ_SET
   return e;
 }
@@ -123,9 +124,10 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   std::lock_guard<std::mutex> lk(g_dev_mu);
   DevState& d = g_dev[dev];
   if (!d.init) {
-    if (set_attrs_gb<16, 2>() != cudaSuccess || set_attrs_gb<4, 2>() != cudaSuccess ||
-        set_attrs_gb<1, 2>() != cudaSuccess || set_attrs_gb<16, 4>() != cudaSuccess ||
-        set_attrs_gb<4, 4>() != cudaSuccess)
+    if (set_attrs_gb<16, 2, 2>() != cudaSuccess || set_attrs_gb<4, 2, 2>() != cudaSuccess ||
+        set_attrs_gb<1, 2, 2>() != cudaSuccess || set_attrs_gb<16, 4, 4>() != cudaSuccess ||
+        set_attrs_gb<4, 4, 4>() != cudaSuccess || set_attrs_gb<16, 4, 2>() != cudaSuccess ||
+        set_attrs_gb<4, 4, 2>() != cudaSuccess)
       return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
     if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
@@ -176,9 +178,11 @@ int code_width(int kbits, int* k, int* sb, int* lvl) {
 }
 
 struct ConvGeom {
-  int ho, wo, M, K, Kpad, kwords;
+  int ho, wo, M, K, Kpad, kwords;   // K: kh*kw*cin of the filters; Kpad: the kernel's K rounded up to 128
   int pool, pho, pwo;   // fused pool window (1: none) and the output shape after it
-  int kb, sb, lvl;      // code width k, stored field bits, thresholds per channel
+  int kb, sb, lvl;      // output code width k, its stored field bits, thresholds per channel
+  bool in8;             // 8-bit input values (one byte each, read as two 4-bit fields)
+  int sbi, cink, Kk;    // input field bits, the kernel's input channels (fields) and its K
 };
 
 int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
@@ -186,6 +190,9 @@ int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   int rc = ifq_conv_out_shape(d, &g->pho, &g->pwo);   // output shape, after the fused pool if any
   if (rc) return rc;
   if ((rc = code_width(d->kbits, &g->kb, &g->sb, &g->lvl))) return rc;
+  if (d->in_bits < 0) return IFQ_EINVAL;
+  if (d->in_bits != 0 && d->in_bits != 8 && d->in_bits != g->kb) return IFQ_EUNSUPPORTED;
+  g->in8 = d->in_bits == 8;
   g->pool = d->pool > 1 ? d->pool : 1;
   g->ho = g->pho * g->pool;                            // the convolution's own output
   g->wo = g->pwo * g->pool;
@@ -200,7 +207,11 @@ int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if ((long long)d->n * d->h * d->w * d->cin >= (1LL << 40)) return IFQ_ERANGE;
   g->M = (int)M;
   g->K = (int)K;
-  g->Kpad = (int)round_up((size_t)K, kBK);
+  // an 8-bit value is two 4-bit fields (low nibble first): the kernel sees 2*cin fields of 4 bits
+  g->sbi = g->in8 ? 4 : g->sb;
+  g->cink = g->in8 ? 2 * d->cin : d->cin;
+  g->Kk = g->in8 ? 2 * (int)K : (int)K;
+  g->Kpad = (int)round_up((size_t)g->Kk, kBK);
   g->kwords = ceil_div((int)K, 32);
   return IFQ_OK;
 }
@@ -218,8 +229,8 @@ int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
     path = forced ? forced : IFQ_PATH_TC;
   }
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
-  // the fused pool exists on the tensor-core path only
-  if (g.pool > 1 && path != IFQ_PATH_TC) return -1;
+  // the fused pool and 8-bit inputs exist on the tensor-core path only
+  if ((g.pool > 1 || g.in8) && path != IFQ_PATH_TC) return -1;
   return path;
 }
 
@@ -246,17 +257,17 @@ int choose_bn(const ConvGeom& g, int cout, int nsm) {
   return best;
 }
 
-template <int GB, int SB>
+template <int GB, int SB, int SBO>
 cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
-#define IFQ_LAUNCH(BN, G, S) \
-  if (bn == BN) return TcInst<BN, G, S>::launch(tm, a, nsm, st);
-  IFQ_TC_VARIANTS(IFQ_LAUNCH, GB, SB)
+#define IFQ_LAUNCH(BN, G, S, SO) \
+  if (bn == BN) return TcInst<BN, G, S, SO>::launch(tm, a, nsm, st);
+  IFQ_TC_VARIANTS(IFQ_LAUNCH, GB, SB, SBO)
 #undef IFQ_LAUNCH
   return cudaErrorInvalidValue;
 }
 
 // Bytes of packed codes per input pixel.
-int pixel_bytes(const ifq_conv_desc* d, const ConvGeom& g) { return d->cin * g.sb / 8; }
+int pixel_bytes(const ifq_conv_desc* d, const ConvGeom& g) { return g.cink * g.sbi / 8; }
 
 // Bytes of packed codes per gathered granule: the largest of 16, 4, 1 that divides a pixel's bytes.
 int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
@@ -268,10 +279,11 @@ int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
 // checked exact range, taps addressable by 32-bit masks, a K-granule table that fits, and an
 // instantiated granule (4-bit fields need 4-byte granules, cin % 8 == 0).
 bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
-  if ((long long)g.lvl * g.K > kTcMaxAcc || d->kh > 32 || d->kw > 32) return false;
+  const long long amax = (long long)(g.in8 ? 255 : g.lvl) * g.K;   // largest |A|
+  if (amax > kTcMaxAcc || d->kh > 32 || d->kw > 32) return false;
   const int gb = granule_bytes(d, g);
-  if (g.sb == 4 && gb == 1) return false;
-  if ((long long)g.Kpad * g.sb / 8 / gb > kMaxTab) return false;
+  if (g.sbi == 4 && gb == 1) return false;
+  if ((long long)g.Kpad * g.sbi / 8 / gb > kMaxTab) return false;
   const long long pb = pixel_bytes(d, g);
   const long long span = ((long long)(d->kh - 1) * d->w + d->kw) * pb + pb;
   return span < (1LL << 31);
@@ -296,16 +308,16 @@ void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const voi
   a->sign = sign;
   a->y_codes = yc;
   a->y_acc = ya;
-  a->n = d->n; a->h = d->h; a->w = d->w; a->cin = d->cin; a->cout = d->cout;
+  a->n = d->n; a->h = d->h; a->w = d->w; a->cin = g.cink; a->cout = d->cout;
   a->kh = d->kh; a->kw = d->kw; a->stride = d->stride; a->pad = d->pad; a->ho = g.ho; a->wo = g.wo;
   a->cinb = pixel_bytes(d, g);
   a->lvl = g.lvl;
   a->M = g.M;
-  a->K = g.K;
+  a->K = g.Kk;
   a->nk = g.Kpad / kBK;
   a->nt = ceil_div(d->cout, bn);
   a->ntiles = ceil_div(g.M, kBM) * a->nt;
-  a->ntab = g.Kpad * g.sb / 8 / granule_bytes(d, g);
+  a->ntab = g.Kpad * g.sbi / 8 / granule_bytes(d, g);
   a->div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
   a->div_wo = make_fastdiv((uint32_t)g.wo);
   a->div_nt = make_fastdiv((uint32_t)a->nt);
@@ -338,13 +350,16 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
     const int gb = granule_bytes(d, g);
-    if (g.sb == 2) {
-      if (gb == 16) e = launch_tc_gb<16, 2>(bn, tm, a, nsm, st);
-      else if (gb == 4) e = launch_tc_gb<4, 2>(bn, tm, a, nsm, st);
-      else e = launch_tc_gb<1, 2>(bn, tm, a, nsm, st);
-    } else {
-      if (gb == 16) e = launch_tc_gb<16, 4>(bn, tm, a, nsm, st);
-      else e = launch_tc_gb<4, 4>(bn, tm, a, nsm, st);
+    if (g.sbi == 2) {
+      if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, tm, a, nsm, st);
+      else if (gb == 4) e = launch_tc_gb<4, 2, 2>(bn, tm, a, nsm, st);
+      else e = launch_tc_gb<1, 2, 2>(bn, tm, a, nsm, st);
+    } else if (g.sb == 4) {
+      if (gb == 16) e = launch_tc_gb<16, 4, 4>(bn, tm, a, nsm, st);
+      else e = launch_tc_gb<4, 4, 4>(bn, tm, a, nsm, st);
+    } else {   // 8-bit input values, 2-bit output codes
+      if (gb == 16) e = launch_tc_gb<16, 4, 2>(bn, tm, a, nsm, st);
+      else e = launch_tc_gb<4, 4, 2>(bn, tm, a, nsm, st);
     }
   } else {
     BsArgs a;
@@ -439,9 +454,41 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
+int check_fixed(int rows, int cout, int m) {
+  if (rows < 0 || cout < 1 || m < 1 || m > 24) return IFQ_EINVAL;
+  if ((long long)rows * cout >= (1LL << 31)) return IFQ_ERANGE;
+  return IFQ_OK;
+}
+
+int run_fixed(const int32_t* acc, int rows, int cout, const int64_t* mul, const int64_t* add, int m, int32_t* y,
+              cudaStream_t st) {
+  int rc = check_fixed(rows, cout, m);
+  if (rc) return rc;
+  if (!acc || !mul || !add || !y) return IFQ_EINVAL;
+  if (((uintptr_t)acc & 3u) || ((uintptr_t)y & 3u) || ((uintptr_t)mul & 7u) || ((uintptr_t)add & 7u)) return IFQ_EALIGN;
+  if (rows == 0) return IFQ_OK;
+  int nsm = 0;
+  if ((rc = ensure_init(&nsm))) return rc;
+  const int total = rows * cout;
+  const cudaError_t e = launch_k(fixed_output_kernel, dim3(launch_1d_blocks((size_t)total, 256, nsm)), dim3(256), 0,
+                                 st, acc, total, make_fastdiv((uint32_t)cout), mul, add, m, y);
+  return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
 // Output shape (n, h, w, c) of a layer, whether it produces codes, and their width k (a layer's
-// input codes and its output codes have the same width).
-int layer_out(const ifq_layer& l, int* n, int* h, int* w, int* c, bool* codes, int* kb) {
+// input codes and its output codes have the same width).  A fixed-point output layer has its
+// source conv's shape and no codes.
+int layer_out(const ifq_layer* layers, int i, int* n, int* h, int* w, int* c, bool* codes, int* kb) {
+  const ifq_layer& l = layers[i];
+  if (l.kind == IFQ_LAYER_FIXED) {
+    if (l.src < 0 || l.src >= i || layers[l.src].kind != IFQ_LAYER_CONV) return IFQ_EINVAL;
+    int rc = layer_out(layers, l.src, n, h, w, c, codes, kb);
+    if (rc) return rc;
+    if (!(layers[l.src].conv.out_mode & IFQ_OUT_ACC)) return IFQ_ESHAPE;
+    if ((rc = check_fixed(*n * *h * *w, *c, l.fixed.m))) return rc;
+    *codes = false;
+    return IFQ_OK;
+  }
   if (l.kind == IFQ_LAYER_CONV) {
     ConvGeom g;
     int rc = check_conv(&l.conv, &g);
@@ -469,14 +516,17 @@ int check_stack(const ifq_layer* layers, int nlayers, const void* x) {
     const ifq_layer& l = layers[i];
     int n, h, w, c, kb;
     bool codes;
-    int rc = layer_out(l, &n, &h, &w, &c, &codes, &kb);
-    if (rc) return rc;
     if (l.src < -1 || l.src >= i) return IFQ_EINVAL;
+    int rc = layer_out(layers, i, &n, &h, &w, &c, &codes, &kb);
+    if (rc) return rc;
+    if (l.kind == IFQ_LAYER_FIXED) continue;   // reads its source conv's accumulators (checked above)
     if (l.src >= 0) {
       int sn, sh, sw, sc, skb;
       bool sc_codes;
-      layer_out(layers[l.src], &sn, &sh, &sw, &sc, &sc_codes, &skb);
-      if (!sc_codes || skb != kb) return IFQ_ESHAPE;
+      layer_out(layers, l.src, &sn, &sh, &sw, &sc, &sc_codes, &skb);
+      // the width a layer reads: its code width, or 8 for a layer on 8-bit input values
+      const int in_kb = l.kind == IFQ_LAYER_CONV && l.conv.in_bits == 8 ? 8 : kb;
+      if (!sc_codes || skb != in_kb) return IFQ_ESHAPE;
       const int in_n = l.kind == IFQ_LAYER_CONV ? l.conv.n : l.pool.n;
       const int in_h = l.kind == IFQ_LAYER_CONV ? l.conv.h : l.pool.h;
       const int in_w = l.kind == IFQ_LAYER_CONV ? l.conv.w : l.pool.w;
@@ -508,7 +558,7 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     if (layers[i].kind != IFQ_LAYER_CONV) return false;
     ConvGeom g;
     if (check_conv(&layers[i].conv, &g)) return false;
-    if (g.pool > 1 || g.kb != 2) return false;   // the persistent kernel: 2-bit codes, no fused pool
+    if (g.pool > 1 || g.kb != 2 || g.in8) return false;   // the persistent kernel: 2-bit codes, no fused pool
     if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
     tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g));
   }
@@ -655,10 +705,16 @@ int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t 
     const ifq_layer& l = layers[i];
     const void* in = l.src < 0 ? x : layers[l.src].y_codes;
     int rc;
-    if (l.kind == IFQ_LAYER_CONV)
+    if (l.kind == IFQ_LAYER_CONV) {
       rc = run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st);
-    else
+    } else if (l.kind == IFQ_LAYER_POOL) {
       rc = run_pool(&l.pool, in, l.sign, l.y_codes, st);
+    } else {
+      const ifq_layer& sl = layers[l.src];
+      ConvGeom g;
+      if ((rc = check_conv(&sl.conv, &g))) return rc;
+      rc = run_fixed(sl.y_acc, sl.conv.n * g.pho * g.pwo, sl.conv.cout, l.fx_mul, l.fx_add, l.fixed.m, l.y_acc, st);
+    }
     if (rc) return rc;
   }
   return IFQ_OK;
@@ -693,7 +749,7 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
   uint8_t* base = (uint8_t*)w_prep;
   const int blocks = launch_1d_blocks((size_t)d->cout * (g.Kpad / 4), 256, nsm);
   prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
-                                                     d->cout, g.K, g.Kpad, g.kwords, 32 / g.sb);
+                                                     d->cout, g.Kk, g.Kpad, g.kwords, 32 / g.sbi, g.in8 ? 1 : 0);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
@@ -846,6 +902,11 @@ int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* strea
   pack_signs_kernel<<<launch_1d_blocks((size_t)rows * kwords, 256, nsm), 256, 0, S(stream)>>>(w, bits, rows, K,
                                                                                                kwords);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_fixed_output(const int32_t* acc, int rows, int cout, const int64_t* mul, const int64_t* add, int m,
+                     int32_t* y, void* stream) {
+  return run_fixed(acc, rows, cout, mul, add, m, y, S(stream));
 }
 
 int ifq_device_status(void* stream, int* status) {

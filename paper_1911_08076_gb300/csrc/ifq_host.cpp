@@ -23,7 +23,7 @@ extern "C" const char* ifq_status_str(int s) {
   }
 }
 
-extern "C" int ifq_version(void) { return 200; }   // 2.0: k-bit descriptors (kbits fields)
+extern "C" int ifq_version(void) { return 300; }   // 3.0: in_bits, fixed-point output layers
 
 // Eq. (3)'s uniform level i (1-based) in the compact form of Sec. 3.2.
 static inline double level(int i, double q_base, double q_offset) { return (double)i * q_base + q_offset; }
@@ -130,6 +130,25 @@ extern "C" int ifq_fold_layer_separated(int cout, int K, int kbits, int m, const
       }
       thr_out[(size_t)n * L + (i - 1)] = (int32_t)T;
     }
+  }
+  return IFQ_OK;
+}
+
+extern "C" int ifq_fold_output_separated(int cout, int m, const float* alpha, float delta_in, const float* bias,
+                                         int64_t* mul_out, int64_t* add_out) {
+  if (cout < 1 || m < 1 || m > 24 || !alpha || !mul_out || !add_out) return IFQ_EINVAL;
+  const double din = delta_in;
+  if (!(din > 0.0) || !std::isfinite(din)) return IFQ_EINVAL;
+  for (int n = 0; n < cout; ++n) {
+    const double a = alpha[n], b = bias ? (double)bias[n] : 0.0;
+    if (!(a > 0.0) || !std::isfinite(a) || !std::isfinite(b)) return IFQ_EINVAL;
+    if (std::fabs(a) * std::ldexp(1.0, m) > 9.0e15 || std::fabs(b) * std::ldexp(1.0, 2 * m) > 9.0e15) return IFQ_EINVAL;
+  }
+  const double Q = std::ldexp(1.0, m);
+  const int64_t d = (int64_t)std::floor(din * Q);
+  for (int n = 0; n < cout; ++n) {
+    mul_out[n] = (int64_t)std::floor((double)alpha[n] * Q) * d;
+    add_out[n] = (int64_t)std::floor((bias ? (double)bias[n] : 0.0) * Q * Q);
   }
   return IFQ_OK;
 }

@@ -182,6 +182,23 @@ __global__ void __launch_bounds__(256) maxpool_codes_bytes_kernel(const PoolArgs
   }
 }
 
+// ---------------------------------------------------------------- fixed-point output
+
+// y = floor((mul[n] * A + add[n]) / 2^m) for item i = r * cout + n (the separated conversion of a
+// non-quantized substructure's output, Sec. 2.2), in 128-bit integers, saturated to int32.
+__global__ void fixed_output_kernel(const int32_t* acc, int total, FastDiv div_cout, const int64_t* mul,
+                                    const int64_t* add, int m, int32_t* y) {
+  grid_dep_launch();
+  grid_dep_wait();
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+    const int r = (int)fdiv((uint32_t)i, div_cout);
+    const int n = i - r * (int)div_cout.d;
+    const __int128 v = (__int128)mul[n] * acc[i] + add[n];
+    const __int128 q = v >> m;   // arithmetic shift: the floor of v / 2^m
+    y[i] = q > (__int128)INT32_MAX ? INT32_MAX : (q < (__int128)INT32_MIN ? INT32_MIN : (int32_t)q);
+  }
+}
+
 // ---------------------------------------------------------------- packing
 
 // one code per byte <-> SB-bit fields, 8/SB codes per packed byte (codes keep their low SB bits)
@@ -223,8 +240,11 @@ __global__ void pack_signs_kernel(const int8_t* w, uint32_t* bits, int rows, int
 // tensor-core A expansion: with cpw codes per packed word (16 for 2-bit, 8 for
 // 4-bit fields), byte p of chunk j holds k = cpw*j + (cpw/4)*(p%4) + p/4;
 // +1 -> 0x38, -1 -> 0xB8, k >= K -> 0; followed by a copy of the sign words.
+// in8: the input is 8-bit values read as two 4-bit fields, so kernel position k
+// is filter position k/2 times 1 (low nibble, k even) or 16 (high nibble):
+// +-16 are the e4m3 bytes 0x58 / 0xD8.  K is the kernel's K (twice the filter's).
 __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_t* bits_copy, int cout, int K,
-                                    int Kpad, int kwords, int cpw) {
+                                    int Kpad, int kwords, int cpw, int in8) {
   const long total = (long)cout * (Kpad / 4);
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
     const int n = (int)(i / (Kpad / 4));
@@ -236,7 +256,12 @@ __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_
       const int j = pos / cpw, p = pos - j * cpw;
       const int k = cpw * j + (cpw >> 2) * (p & 3) + (p >> 2);
       uint32_t byte = 0;
-      if (k < K) byte = ((bits[(size_t)n * kwords + (k >> 5)] >> (k & 31)) & 1u) ? 0x38u : 0xB8u;
+      if (k < K) {
+        const int kf = in8 ? (k >> 1) : k;                       // filter position
+        const bool hi = in8 && (k & 1);
+        const bool pos = (bits[(size_t)n * kwords + (kf >> 5)] >> (kf & 31)) & 1u;
+        byte = pos ? (hi ? 0x58u : 0x38u) : (hi ? 0xD8u : 0xB8u);
+      }
       out |= byte << (8 * t);
     }
     *(uint32_t*)(e4m3 + (size_t)n * Kpad + p4) = out;

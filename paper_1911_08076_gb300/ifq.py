@@ -22,7 +22,7 @@ _lib = None
 IFQ_OK, IFQ_EINVAL, IFQ_ESHAPE, IFQ_EALIGN, IFQ_ERANGE, IFQ_ECUDA, IFQ_ETIMEOUT, IFQ_EUNSUPPORTED, IFQ_EWORKSPACE = range(9)
 IFQ_OUT_CODES, IFQ_OUT_ACC, IFQ_OUT_BOTH = 1, 2, 3
 IFQ_PATH_AUTO, IFQ_PATH_TC, IFQ_PATH_BITSERIAL = 0, 1, 2
-IFQ_LAYER_CONV, IFQ_LAYER_POOL = 1, 2
+IFQ_LAYER_CONV, IFQ_LAYER_POOL, IFQ_LAYER_FIXED = 1, 2, 3
 
 
 class IfqError(RuntimeError):
@@ -33,17 +33,23 @@ class IfqError(RuntimeError):
 
 class ConvDesc(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int) for f in
-                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path", "pool", "kbits")]
+                ("n", "h", "w", "cin", "cout", "kh", "kw", "stride", "pad", "out_mode", "path", "pool", "kbits",
+                 "in_bits")]
 
 
 class PoolDesc(ctypes.Structure):
     _fields_ = [(f, ctypes.c_int) for f in ("n", "h", "w", "c", "k", "stride", "pad", "kbits")]
 
 
+class FixedDesc(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int)]
+
+
 class Layer(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("src", ctypes.c_int), ("conv", ConvDesc), ("pool", PoolDesc),
                 ("w_prep", ctypes.c_void_p), ("thr", ctypes.c_void_p), ("sign", ctypes.c_void_p),
-                ("y_codes", ctypes.c_void_p), ("y_acc", ctypes.c_void_p)]
+                ("y_codes", ctypes.c_void_p), ("y_acc", ctypes.c_void_p), ("fixed", FixedDesc),
+                ("fx_mul", ctypes.c_void_p), ("fx_add", ctypes.c_void_p)]
 
 
 _P = ctypes.c_void_p
@@ -56,6 +62,8 @@ _SIGS = {
     "ifq_version": ([], _I),
     "ifq_fold_layer": ([_I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
     "ifq_fold_layer_separated": ([_I, _I, _I, _I, _P, _F, _P, _P, _P, _P, _P, _F, _F, _F, _P, _P], _I),
+    "ifq_fold_output_separated": ([_I, _I, _P, _F, _P, _P, _P], _I),
+    "ifq_fixed_output": ([_P, _I, _I, _P, _P, _I, _P, _P], _I),
     "ifq_codes_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
     "ifq_codes_storage_bytes": ([_I, _I, _I, _I, _I, ctypes.POINTER(_SZ)], _I),
     "ifq_conv_out_shape": ([ctypes.POINTER(ConvDesc), ctypes.POINTER(_I), ctypes.POINTER(_I)], _I),
@@ -170,6 +178,22 @@ def ifq_fold_layer_separated(K: int, m: int, alpha, gamma, beta, mean, var, delt
     return T, s
 
 
+def ifq_fold_output_separated(m: int, alpha, delta_in: float = 0.5, bias=None):
+    """Separated fixed-point conversion of a non-quantized conv output (host): (mul, add) int64 [cout]."""
+    al = np.ascontiguousarray(alpha, dtype=np.float32)
+    bi = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    mul = np.empty(al.shape[0], np.int64)
+    add = np.empty(al.shape[0], np.int64)
+    _ok(lib().ifq_fold_output_separated(al.shape[0], int(m), _ptr(al), delta_in, _ptr(bi), _ptr(mul), _ptr(add)),
+        "ifq_fold_output_separated")
+    return mul, add
+
+
+def ifq_fixed_output(acc, rows: int, cout: int, mul, add, m: int, y, stream=None):
+    _ok(lib().ifq_fixed_output(_ptr(acc), rows, cout, _ptr(mul), _ptr(add), m, _ptr(y), _stream(stream)),
+        "ifq_fixed_output")
+
+
 def ifq_codes_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> int:
     out = _SZ()
     _ok(lib().ifq_codes_bytes(n, h, w, c, kbits, ctypes.byref(out)), "ifq_codes_bytes")
@@ -183,8 +207,9 @@ def ifq_codes_storage_bytes(n: int, h: int, w: int, c: int, kbits: int = 2) -> i
 
 
 def conv_desc(n, h, w, cin, cout, k, stride=1, pad=0, out_mode=IFQ_OUT_CODES, path=IFQ_PATH_AUTO, kw=None, pool=0,
-              kbits=2):
-    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path, pool, kbits)
+              kbits=2, in_bits=0):
+    return ConvDesc(n, h, w, cin, cout, k, k if kw is None else kw, stride, pad, out_mode, path, pool, kbits,
+                    in_bits)
 
 
 def pool_desc(n, h, w, c, k, stride, pad=0, kbits=2):

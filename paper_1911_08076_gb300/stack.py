@@ -33,19 +33,23 @@ class DeviceStack:
         self.layers: List[ifq.Layer] = []
         self.host_thr: Dict[int, np.ndarray] = {}
         self.host_sign: Dict[int, np.ndarray] = {}
+        self.fx: Dict[int, tuple] = {}
         B = self.batch
+        kinds = {"conv": ifq.IFQ_LAYER_CONV, "pool": ifq.IFQ_LAYER_POOL, "fixed": ifq.IFQ_LAYER_FIXED}
         for li, l in enumerate(workload.layers):
             rec = ifq.Layer()
-            rec.kind = ifq.IFQ_LAYER_CONV if l.kind == "conv" else ifq.IFQ_LAYER_POOL
+            rec.kind = kinds[l.kind]
             rec.src = l.src
             if l.kind == "conv":
                 p = params[li]
                 mode = {"codes": ifq.IFQ_OUT_CODES, "acc": ifq.IFQ_OUT_ACC, "both": ifq.IFQ_OUT_BOTH}[l.out]
                 d = ifq.conv_desc(B, l.h, l.w, l.cin, l.cout, l.k, l.stride, l.pad, mode, path, pool=l.pool,
-                                  kbits=kbits)
+                                  kbits=kbits, in_bits=l.in_bits)
                 K = l.k * l.k * l.cin
-                T, s = ifq.ifq_fold_layer(K, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias, p.eps,
-                                          p.q_base, p.q_offset, kbits)
+                # a layer on 8-bit input values has |A| <= 255 K: its fold clamps at L K_fold >= 255 K
+                K_fold = -(-255 * K // ((1 << kbits) - 1)) if l.in_bits == 8 else K
+                T, s = ifq.ifq_fold_layer(K_fold, p.alpha, p.gamma, p.beta, p.mean, p.var, p.delta_in, p.bias,
+                                          p.eps, p.q_base, p.q_offset, kbits)
                 self.host_thr[li], self.host_sign[li] = T, s
                 self.thr[li] = torch.from_numpy(T).to(self.device)
                 self.sign[li] = torch.from_numpy(s).to(self.device)
@@ -69,6 +73,15 @@ class DeviceStack:
                 rec.sign = self.sign[li].data_ptr()
                 rec.y_codes = self.y_codes[li].data_ptr() if li in self.y_codes else None
                 rec.y_acc = self.y_acc[li].data_ptr() if li in self.y_acc else None
+            elif l.kind == "fixed":
+                sl, sp = workload.layers[l.src], params[l.src]
+                mul, add = ifq.ifq_fold_output_separated(l.m, sp.alpha, sp.delta_in, sp.bias)
+                self.fx[li] = (torch.from_numpy(mul).to(self.device), torch.from_numpy(add).to(self.device))
+                self.y_acc[li] = torch.empty((B, sl.out_h, sl.out_w, sl.cout), dtype=torch.int32, device=self.device)
+                rec.fixed = ifq.FixedDesc(l.m)
+                rec.fx_mul = self.fx[li][0].data_ptr()
+                rec.fx_add = self.fx[li][1].data_ptr()
+                rec.y_acc = self.y_acc[li].data_ptr()
             else:
                 d = ifq.pool_desc(B, l.h, l.w, l.c, l.k, l.stride, l.pad, kbits)
                 ho, wo = ifq.ifq_pool_out_shape(d)
@@ -84,7 +97,7 @@ class DeviceStack:
 
     def input_buffer(self) -> torch.Tensor:
         wl = self.wl
-        fb = 2 if self.kbits == 2 else 4
+        fb = 8 if getattr(wl, "in_bits", 0) == 8 else (2 if self.kbits == 2 else 4)
         return torch.empty((self.batch, wl.h, wl.w, wl.c * fb // 8), dtype=torch.uint8, device=self.device)
 
     def forward(self, x: torch.Tensor, stream=None):
@@ -94,12 +107,16 @@ class DeviceStack:
         """ifq_forward's launches issued one ifq_conv2bit / ifq_maxpool2bit call at a time, with
         optional callbacks before and after each layer (for per-launch CUDA events)."""
         for li, rec in enumerate(self.layers):
-            src = x if rec.src < 0 else self.y_codes[rec.src]
+            src = x if rec.src < 0 else self.y_codes.get(rec.src)
             if before:
                 before(li)
             if rec.kind == ifq.IFQ_LAYER_CONV:
                 ifq.ifq_conv2bit(rec.conv, src, rec.w_prep, rec.thr, rec.sign, rec.y_codes, rec.y_acc, self.ws,
                                  self.ws_bytes, stream)
+            elif rec.kind == ifq.IFQ_LAYER_FIXED:
+                sl = self.wl.layers[rec.src]
+                ifq.ifq_fixed_output(self.y_acc[rec.src], self.batch * sl.out_h * sl.out_w, sl.cout,
+                                     self.fx[li][0], self.fx[li][1], rec.fixed.m, self.y_acc[li], stream)
             else:
                 ifq.ifq_maxpool2bit(rec.pool, src, rec.sign, rec.y_codes, stream)
             if after:

@@ -58,6 +58,7 @@ class Conv:
     src: int
     out: str = "codes"
     pool: int = 0
+    in_bits: int = 0    # 8: the layer reads 8-bit input values (image pixels), not codes
     kind: str = field(default="conv", init=False)
 
     @property
@@ -88,6 +89,16 @@ class Pool:
 
 
 @dataclass
+class Fixed:
+    """Separated fixed-point output (Sec. 2.2, Q_m = 2^m) of the int32 accumulators of conv
+    layer `src`: the non-quantized last substructure of a network (a YOLO detection conv)."""
+    name: str
+    src: int
+    m: int
+    kind: str = field(default="fixed", init=False)
+
+
+@dataclass
 class Workload:
     name: str
     index: int
@@ -97,6 +108,7 @@ class Workload:
     c: int
     layers: list
     kbits: int = 2      # code width k of every quantized layer's input and output codes
+    in_bits: int = 0    # 8: the stack input is 8-bit values (an image), read by the first conv
 
     @property
     def seed(self) -> int:
@@ -169,6 +181,24 @@ def tiny_yolo(batch: int = 64, tinier: bool = False) -> Workload:
     return Workload(name, 3, batch, 208, 208, ch[0], L)
 
 
+def tinier_yolo_full(batch: int = 64) -> Workload:
+    """IFQ-Tinier-YOLO end to end at 416 (Sec. 4.2): every conv binarized, the first one on the
+    8-bit RGB image (padded to 4 channels, pixel step 1/255, the integrated conversion to 2-bit
+    codes), the Tinier backbone, and the 1x1 detection conv (a non-quantized substructure) as
+    int32 accumulators converted to fixed point by the separated method at m = 14."""
+    body = tiny_yolo(batch, True)
+    L = [Conv("conv1", 4, 8, 3, 1, 1, 416, 416, 416, 416, -1, in_bits=8),
+         Pool("pool1", 8, 2, 2, 0, 416, 416, 208, 208, 0)]
+    for l in body.layers:
+        src = l.src + 2 if l.src >= 0 else 1
+        if l.kind == "conv":
+            L.append(Conv(l.name, l.cin, l.cout, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.out, l.pool))
+        else:
+            L.append(Pool(l.name, l.c, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.signed))
+    L.append(Fixed("det_fixed", len(L) - 1, 14))
+    return Workload(f"tinier_yolo_full416_b{batch}", 5, batch, 416, 416, 4, L, 2, 8)
+
+
 def roofline(batch: int = 256, which: str = "3x3") -> Workload:
     """Large single layers: 3x3 256->256 at 56x56, or 1x1 512->512 at 28x28."""
     if which == "3x3":
@@ -209,16 +239,19 @@ def fuse_pools(wl: Workload) -> Workload:
         if l.kind == "conv":
             old = [j for j, m in enumerate(wl.layers) if m is l][0]
             p = wl.layers[fused_into[old]].k if old in fused_into else l.pool
-            out.append(Conv(l.name, l.cin, l.cout, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.out, p))
+            out.append(Conv(l.name, l.cin, l.cout, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.out, p,
+                            l.in_bits))
+        elif l.kind == "fixed":
+            out.append(Fixed(l.name, src, l.m))
         else:
             out.append(Pool(l.name, l.c, l.k, l.stride, l.pad, l.h, l.w, l.ho, l.wo, src, l.signed))
-    return Workload(wl.name + "_fused", wl.index, wl.batch, wl.h, wl.w, wl.c, out, wl.kbits)
+    return Workload(wl.name + "_fused", wl.index, wl.batch, wl.h, wl.w, wl.c, out, wl.kbits, wl.in_bits)
 
 
 def with_kbits(wl: Workload, kbits: int) -> Workload:
     """The same stack with k-bit codes between layers (Table 2's k = 3, 4 columns; Eq. (8)).
     Same index, so the same filter and parameter draws."""
-    return Workload(f"{wl.name}_k{kbits}", wl.index, wl.batch, wl.h, wl.w, wl.c, wl.layers, kbits)
+    return Workload(f"{wl.name}_k{kbits}", wl.index, wl.batch, wl.h, wl.w, wl.c, wl.layers, kbits, wl.in_bits)
 
 
 WORKLOADS = {
@@ -235,6 +268,8 @@ WORKLOADS = {
     "alexnet_k4": lambda batch=128: with_kbits(alexnet(batch), 4),
     "resnet18_k4": lambda batch=32: with_kbits(resnet18(batch), 4),
     "tinyyolo_fused_k4": lambda batch=64: with_kbits(fuse_pools(tiny_yolo(batch, False)), 4),
+    "tinieryolo_full": tinier_yolo_full,
+    "tinieryolo_full_fused": lambda batch=64: fuse_pools(tinier_yolo_full(batch)),
 }
 
 
@@ -293,21 +328,33 @@ def draw_codes(rng: np.random.Generator, shape, kbits: int = 2) -> np.ndarray:
     return rng.integers(0, 1 << kbits, size=shape, dtype=np.uint8)
 
 
+PIXEL_STEP = 1.0 / 255.0   # input step of a layer on 8-bit image values (pixels scaled to [0, 1])
+
+
 def draw_workload(wl: Workload, batch: Optional[int] = None):
-    """Input codes [B][H][W][C] (uint8) and per-layer ConvParams (None for pools)."""
+    """Input [B][H][W][C] (uint8: k-bit codes, or 8-bit pixels with a zero 4th channel for an image
+    input) and per-layer ConvParams (None for pools and fixed-point outputs)."""
     rng = np.random.default_rng(wl.seed)
     params = [draw_conv_params(rng, l) if l.kind == "conv" else None for l in wl.layers]
+    for l, p in zip(wl.layers, params):
+        if l.kind == "conv" and l.in_bits == 8:
+            p.delta_in = PIXEL_STEP
     b = wl.batch if batch is None else batch
-    x = draw_codes(rng, (b, wl.h, wl.w, wl.c), wl.kbits)
+    if wl.in_bits == 8:
+        x = rng.integers(0, 256, size=(b, wl.h, wl.w, wl.c), dtype=np.uint8)
+        x[..., 3:] = 0
+    else:
+        x = draw_codes(rng, (b, wl.h, wl.w, wl.c), wl.kbits)
     return x, params
 
 
 # ----------------------------------------------------------------------------- formats
 
 def field_bits(kbits: int) -> int:
-    """Bits of the storage field of a k-bit code: 2 for k = 2, 4 for k = 3 and 4."""
-    assert kbits in (2, 3, 4), kbits
-    return 2 if kbits == 2 else 4
+    """Bits of the storage field of a k-bit code: 2 for k = 2, 4 for k = 3 and 4, 8 for 8-bit
+    input values."""
+    assert kbits in (2, 3, 4, 8), kbits
+    return {2: 2, 3: 4, 4: 4, 8: 8}[kbits]
 
 
 def pack_codes(codes: np.ndarray, kbits: int = 2) -> np.ndarray:
@@ -315,6 +362,8 @@ def pack_codes(codes: np.ndarray, kbits: int = 2) -> np.ndarray:
     f = field_bits(kbits)
     c = np.ascontiguousarray(codes, dtype=np.uint8)
     assert c.shape[-1] % 4 == 0
+    if f == 8:
+        return c.copy()
     assert c.size == 0 or int(c.max()) < (1 << kbits)
     per = 8 // f
     q = c.reshape(c.shape[:-1] + (c.shape[-1] // per, per))
@@ -329,6 +378,8 @@ def unpack_codes(packed: np.ndarray, c: Optional[int] = None, kbits: int = 2) ->
     f = field_bits(kbits)
     per = 8 // f
     p = np.ascontiguousarray(packed, dtype=np.uint8)
+    if f == 8:
+        return p.copy() if c is None else p[..., :c].copy()
     out = np.stack([(p >> (f * l)) & ((1 << f) - 1) for l in range(per)], axis=-1)
     out = out.reshape(p.shape[:-1] + (p.shape[-1] * per,))
     return out if c is None else out[..., :c]

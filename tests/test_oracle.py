@@ -393,3 +393,64 @@ def test_separated_converges_and_is_monotone():
         d = np.diff(sc, axis=0)
         up = p.gamma > 0
         assert (d[:, up] >= 0).all() and (d[:, ~up] <= 0).all()
+
+
+# ----------------------------------------------------------------------------- non-quantized ends
+
+def test_fixed_output_hand_case():
+    """Separated fixed-point output (Sec. 2.2) by hand: alpha = 0.3, delta = 0.5, b = 0.1 at m = 4
+    (Q = 16): a = floor(4.8) = 4, d = floor(8) = 8, bq = floor(25.6) = 25, y = floor((32 A + 25)/16):
+    A = 10 -> floor(345/16) = 21; A = -3 -> floor(-71/16) = -5; A = 0 -> floor(25/16) = 1."""
+    p = O.Params([0.3], [1.0], [0.0], [0.0], [1.0], [0.1], 0.5, 0.5, -0.25, 0.0)
+    A = np.array([[10], [-3], [0]], np.int32)
+    assert O.fixed_output(A, p, 4).ravel().tolist() == [21, -5, 1]
+
+
+@pytest.mark.parametrize("m", [8, 14, 20])
+def test_fixed_output_within_the_floor_error_of_the_float_value(m):
+    """|y/Q - (alpha delta A + b)| is bounded by the three floors and the final one:
+    (|A| (alpha + delta) Q + |A| + 1) / Q^2 + 1/Q, and the bound shrinks as 2^-m."""
+    rng = np.random.default_rng(m)
+    cout, Q = 30, 2.0 ** m
+    p = O.Params(rng.uniform(0.01, 1.5, cout), np.ones(cout), np.zeros(cout), np.zeros(cout), np.ones(cout),
+                 rng.normal(0, 1, cout), 0.5, 0.5, -0.25, 0.0)
+    amax = min(3000, int(0.5 * 2.0 ** 31 / Q / 0.8))    # |alpha delta A + b| stays inside int32 / Q
+    A = rng.integers(-amax, amax, (500, cout)).astype(np.int32)
+    y = O.fixed_output(A, p, m).astype(np.float64) / Q
+    ref = p.alpha * p.delta_in * A + p.bias
+    bound = (np.abs(A) * (p.alpha + p.delta_in) * Q + np.abs(A) + 1) / Q ** 2 + 1 / Q
+    assert (np.abs(y - ref) <= bound + 1e-12).all()
+    assert np.abs(y - ref).max() < 4000 * 2.0 ** -m * 2
+    # beyond the int32 range the output saturates
+    big = np.full((1, cout), 2 ** 30, np.int32)
+    assert (O.fixed_output(big, p, 24) == np.iinfo(np.int32).max).all()
+    assert (O.fixed_output(-big, p, 24) == np.iinfo(np.int32).min).all()
+
+
+def test_conv_on_8bit_values_matches_torch():
+    """The integer core of the first (image) layer: 8-bit input values, +-1 filters."""
+    rng = np.random.default_rng(8)
+    x = rng.integers(0, 256, (2, 11, 9, 4), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (8, 3, 3, 4)) == 1, 1, -1).astype(np.int8)
+    A = O.conv_acc(x, w, 1, 1)
+    ref = F.conv2d(torch.from_numpy(x.astype(np.float64)).permute(0, 3, 1, 2),
+                   torch.from_numpy(w.astype(np.float64)).permute(0, 3, 1, 2), padding=1).permute(0, 2, 3, 1)
+    assert (A == ref.numpy().astype(np.int64)).all()
+    assert np.abs(A).max() > 3 * 36          # beyond any 2-bit input's range
+
+
+def test_fold_for_8bit_input_covers_the_whole_range():
+    """A first layer on pixels (step 1/255): with K_fold = ceil(255 K / 3) the fold's clamp covers
+    every |A| <= 255 K, and the integer chain equals the float chain on all of them."""
+    rng = np.random.default_rng(255)
+    layer = synth.Conv("c1", 4, 8, 3, 1, 1, 8, 8, 8, 8, -1, in_bits=8)
+    K = 36
+    assert O.fold_k(layer) == -(-255 * K // 3)
+    p = _random_params(rng, 24)
+    p.delta_in = 1.0 / 255.0
+    p.alpha = p.alpha * (4.0 / np.sqrt(K)) * 20.0
+    amax = 255 * K
+    A = np.repeat(np.arange(-amax, amax + 1, dtype=np.int32)[:, None], p.cout, axis=1)
+    T, s = O.fold(p, O.fold_k(layer))
+    codes, ties = O.check_chains(A, p, T, s)
+    assert ties == 0 and codes.min() == 0 and codes.max() == 3
