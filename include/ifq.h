@@ -70,7 +70,7 @@ typedef enum {
 enum { IFQ_OUT_CODES = 1, IFQ_OUT_ACC = 2, IFQ_OUT_BOTH = 3 };
 
 /* Kernel path of a convolution (ifq_conv_desc.path). */
-enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2 };
+enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2, IFQ_PATH_DIRECT = 3 };
 
 /* Layer kinds of ifq_forward. */
 enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2, IFQ_LAYER_FIXED = 3 };
@@ -197,11 +197,14 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
 
 /*
  * The kernel path ifq_conv2bit takes for `d` (host; reads IFQ_FORCE_PATH as
- * ifq_conv2bit does): IFQ_PATH_TC or IFQ_PATH_BITSERIAL.  The tensor-core path
- * needs (2^k - 1)*K <= 196608 (the accumulator range checked exact on the fp8
- * tensor cores), kh, kw <= 32, and for k = 3, 4 cin % 8 == 0; a request for it
- * outside that range takes the bit-serial path.  IFQ_EUNSUPPORTED for a fused
- * pool off the tensor-core path.
+ * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL or IFQ_PATH_DIRECT.  The
+ * tensor-core path needs (2^k - 1)*K <= 196608 (the accumulator range checked
+ * exact on the fp8 tensor cores; 255*K for 8-bit inputs), kh, kw <= 32, and
+ * for k = 3, 4 cin % 8 == 0; a request for it outside that range takes the
+ * bit-serial path.  The direct CUDA-core path serves layers on 8-bit inputs
+ * with cout <= 32 and K <= 257 (the default for them); a request for it
+ * elsewhere takes the tensor-core path.  IFQ_EUNSUPPORTED for a fused pool
+ * or an 8-bit input that would land on the bit-serial path.
  */
 int ifq_conv_plan(const ifq_conv_desc* d, int* path);
 

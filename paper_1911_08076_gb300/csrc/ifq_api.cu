@@ -15,6 +15,7 @@
 #include <vector>
 
 #include "conv_bitserial.cuh"
+#include "conv_direct.cuh"
 #include "conv_tc.cuh"
 #include "ifq.h"
 #include "pool_pack.cuh"
@@ -146,6 +147,12 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   return IFQ_OK;
 }
 
+int launch_1d_blocks(size_t items, int threads, int nsm) {
+  size_t b = (items + threads - 1) / threads;
+  if (b > (size_t)nsm * 32) b = (size_t)nsm * 32;
+  return b < 1 ? 1 : (int)b;
+}
+
 // Multiply-high divisor for n / d with 0 <= n < 2^31 (d >= 1): shift = ceil(log2 d),
 // mul = floor(2^32 * (2^shift - d) / d) + 1, n / d = (umulhi(n, mul) + n) >> shift.
 FastDiv make_fastdiv(uint32_t d) {
@@ -200,7 +207,7 @@ int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if (d->cin % 4 != 0) return IFQ_ESHAPE;
   if (d->out_mode < IFQ_OUT_CODES || d->out_mode > IFQ_OUT_BOTH) return IFQ_EINVAL;
   if ((d->out_mode & IFQ_OUT_CODES) && d->cout % 4 != 0) return IFQ_ESHAPE;
-  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_BITSERIAL) return IFQ_EINVAL;
+  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_DIRECT) return IFQ_EINVAL;
   const long long K = (long long)d->kh * d->kw * d->cin;
   const long long M = (long long)d->n * g->ho * g->wo;
   if (K > kMaxK || d->cout > 65536 || M >= (1LL << 31)) return IFQ_ERANGE;
@@ -220,17 +227,34 @@ size_t prep_bits_offset(const ifq_conv_desc* d, const ConvGeom& g) {
   return round_up((size_t)d->cout * g.Kpad, 256);
 }
 
+// Prepared filters: e4m3 rows, then the sign words, then (layers on 8-bit inputs) the per-tap
+// masks of the direct path.
+size_t prep_masks_offset(const ifq_conv_desc* d, const ConvGeom& g) {
+  return prep_bits_offset(d, g) + round_up((size_t)d->cout * g.kwords * 4, 256);
+}
+
+size_t prep_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
+  return g.in8 ? prep_masks_offset(d, g) + (size_t)g.K * 4 : prep_bits_offset(d, g) + (size_t)d->cout * g.kwords * 4;
+}
+
 bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g);
+
+// The direct CUDA-core path: layers on 8-bit input values with at most 32 output channels and
+// K <= 257 (the two 16-bit channel sums of a register stay apart).
+bool direct_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  return g.in8 && d->cout <= kDirectMaxCout && g.K <= kDirectMaxK;
+}
 
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
-    path = forced ? forced : IFQ_PATH_TC;
+    path = forced ? forced : (direct_supported(d, g) ? IFQ_PATH_DIRECT : IFQ_PATH_TC);
   }
+  if (path == IFQ_PATH_DIRECT && !direct_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
-  // the fused pool and 8-bit inputs exist on the tensor-core path only
-  if ((g.pool > 1 || g.in8) && path != IFQ_PATH_TC) return -1;
+  // the fused pool and 8-bit inputs have no bit-serial form
+  if ((g.pool > 1 || g.in8) && path == IFQ_PATH_BITSERIAL) return -1;
   return path;
 }
 
@@ -343,7 +367,38 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   const int path = choose_path(d, g);
   if (path < 0) return IFQ_EUNSUPPORTED;
   cudaError_t e;
-  if (path == IFQ_PATH_TC) {
+  if (path == IFQ_PATH_DIRECT) {
+    DirectArgs a;
+    a.x = (const uint8_t*)x;
+    a.wmask = (const uint32_t*)((const uint8_t*)w_prep + prep_masks_offset(d, g));
+    a.thr = thr;
+    a.sign = sign;
+    a.y_codes = yc;
+    a.y_acc = ya;
+    a.n = d->n; a.h = d->h; a.w = d->w; a.cin = d->cin; a.cout = d->cout;
+    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad; a.ho = g.ho; a.wo = g.wo;
+    a.K = g.K;
+    a.lvl = g.lvl;
+    a.sbo = g.sb;
+    a.pool = g.pool;
+    a.pho = g.pho;
+    a.pwo = g.pwo;
+    a.total = d->n * g.pho * g.pwo;
+    a.div_pwo = make_fastdiv((uint32_t)g.pwo);
+    a.div_pho = make_fastdiv((uint32_t)g.pho);
+    const dim3 grid(launch_1d_blocks((size_t)a.total, kDirectThreads, nsm)), block(kDirectThreads);
+    // the RGB first layer (cin 4, 3x3, stride 1, pool 1 or 2) has its own instances
+    const bool rgb3 = d->cin == 4 && d->kh == 3 && d->kw == 3 && d->stride == 1 && (g.pool == 1 || g.pool == 2);
+    if (rgb3 && d->cout <= 8)
+      e = g.pool == 2 ? launch_k(conv_direct_rgb3_kernel<4, 2>, grid, block, 0, st, a)
+                      : launch_k(conv_direct_rgb3_kernel<4, 1>, grid, block, 0, st, a);
+    else if (rgb3 && d->cout <= 16)
+      e = g.pool == 2 ? launch_k(conv_direct_rgb3_kernel<8, 2>, grid, block, 0, st, a)
+                      : launch_k(conv_direct_rgb3_kernel<8, 1>, grid, block, 0, st, a);
+    else if (d->cout <= 8) e = launch_k(conv_direct_kernel<4>, grid, block, 0, st, a);
+    else if (d->cout <= 16) e = launch_k(conv_direct_kernel<8>, grid, block, 0, st, a);
+    else e = launch_k(conv_direct_kernel<16>, grid, block, 0, st, a);
+  } else if (path == IFQ_PATH_TC) {
     const int bn = choose_bn(g, d->cout, nsm);
     CUtensorMap tm;
     if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
@@ -380,12 +435,6 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     else e = launch_k(conv_bitserial_kernel<4>, grid, dim3(kBsThreads), 0, st, a);
   }
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
-}
-
-int launch_1d_blocks(size_t items, int threads, int nsm) {
-  size_t b = (items + threads - 1) / threads;
-  if (b > (size_t)nsm * 32) b = (size_t)nsm * 32;
-  return b < 1 ? 1 : (int)b;
 }
 
 int check_pool(const ifq_pool_desc* d, int* ho, int* wo, int* sb = nullptr) {
@@ -734,7 +783,7 @@ int ifq_weights_prep_bytes(const ifq_conv_desc* d, size_t* bytes) {
   if (!bytes) return IFQ_EINVAL;
   int rc = check_conv(d, &g);
   if (rc) return rc;
-  *bytes = prep_bits_offset(d, g) + (size_t)d->cout * g.kwords * 4;
+  *bytes = prep_bytes(d, g);
   return IFQ_OK;
 }
 
@@ -750,6 +799,10 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
   const int blocks = launch_1d_blocks((size_t)d->cout * (g.Kpad / 4), 256, nsm);
   prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
                                                      d->cout, g.Kk, g.Kpad, g.kwords, 32 / g.sbi, g.in8 ? 1 : 0);
+  if (g.in8)
+    prep_direct_masks_kernel<<<launch_1d_blocks((size_t)g.K, 256, nsm), 256, 0, S(stream)>>>(
+        (const uint32_t*)(base + prep_bits_offset(d, g)), (uint32_t*)(base + prep_masks_offset(d, g)), d->cout, g.K,
+        g.kwords);
   return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 

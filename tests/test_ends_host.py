@@ -7,7 +7,7 @@ from oracle import oracle as O
 from paper_1911_08076_gb300 import ifq, synth
 
 FAKE = 1 << 20
-TC, BS = ifq.IFQ_PATH_TC, ifq.IFQ_PATH_BITSERIAL
+TC, BS, DI = ifq.IFQ_PATH_TC, ifq.IFQ_PATH_BITSERIAL, ifq.IFQ_PATH_DIRECT
 
 
 def _status(fn, *a, **kw):
@@ -18,13 +18,18 @@ def _status(fn, *a, **kw):
 
 def test_8bit_input_plan_and_refusals():
     d = ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, ifq.IFQ_OUT_BOTH, in_bits=8)
+    assert ifq.ifq_conv_plan(d) == DI                          # few channels: the direct path
+    d.path = TC
     assert ifq.ifq_conv_plan(d) == TC
-    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, pool=2, in_bits=8)) == TC
+    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, pool=2, in_bits=8)) == DI
+    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 64, 3, 1, 1, in_bits=8)) == TC      # cout > 32
+    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 32, 8, 3, 1, 1, in_bits=8)) == TC      # K = 288 > 257
+    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 64, 64, 3, 1, 1, path=DI)) == TC      # 2-bit codes
     assert _status(ifq.ifq_conv_plan, ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, path=BS, in_bits=8)) == \
         ifq.IFQ_EUNSUPPORTED                                   # no bit-serial path for 8-bit values
     assert _status(ifq.ifq_conv_plan, ifq.conv_desc(1, 9, 9, 88, 8, 3, 1, 1, in_bits=8)) == \
         ifq.IFQ_EUNSUPPORTED                                   # 255 * 792 > 196608
-    assert ifq.ifq_conv_plan(ifq.conv_desc(1, 9, 9, 84, 8, 3, 1, 1, in_bits=8)) == TC   # 255 * 756
+    assert ifq.ifq_conv_plan(ifq.conv_desc(1, 9, 9, 84, 8, 3, 1, 1, in_bits=8)) == TC   # 255 * 756, K > 257
     assert _status(ifq.ifq_weights_prep_bytes, ifq.conv_desc(1, 9, 9, 4, 8, 3, in_bits=5)) == ifq.IFQ_EUNSUPPORTED
     assert _status(ifq.ifq_weights_prep_bytes, ifq.conv_desc(1, 9, 9, 4, 8, 3, in_bits=-1)) == ifq.IFQ_EINVAL
     assert ifq.ifq_weights_prep_bytes(ifq.conv_desc(1, 9, 9, 4, 8, 3, in_bits=2)) > 0   # = kbits: plain codes

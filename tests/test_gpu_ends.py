@@ -21,11 +21,15 @@ IN8_CASES = [
     (1, 13, 11, 16, 32, 3, 2, 1, 0),      # 16-byte pixels, stride 2, ragged M
     (3, 9, 9, 20, 64, 3, 1, 1, 0),        # 20-byte pixels
     (2, 12, 12, 8, 16, 5, 1, 2, 0),       # 5x5 window
+    (2, 17, 19, 4, 16, 3, 1, 1, 0),       # RGB first layer, 16 channels, odd sizes
+    (2, 18, 18, 4, 12, 3, 1, 1, 2),       # 12 channels, fused pool
+    (1, 10, 10, 4, 8, 3, 1, 0, 2),        # no padding, fused pool
 ]
 
 
+@pytest.mark.parametrize("path", [ifq.IFQ_PATH_TC, ifq.IFQ_PATH_DIRECT], ids=["tc", "direct"])
 @pytest.mark.parametrize("case", IN8_CASES, ids=[str(c) for c in IN8_CASES])
-def test_conv_on_8bit_values_matches_oracle(case):
+def test_conv_on_8bit_values_matches_oracle(case, path):
     B, H, W, C, cout, k, s, p, pool = case
     rng = np.random.default_rng(abs(hash(case)) % (2 ** 32))
     x = rng.integers(0, 256, (B, H, W, C), dtype=np.uint8)
@@ -37,8 +41,9 @@ def test_conv_on_8bit_values_matches_oracle(case):
                    rng.normal(0, 0.5, cout), rng.normal(0, 1.0, cout), rng.uniform(0.5, 2.0, cout), None,
                    synth.PIXEL_STEP, 0.5, -0.25, synth.EPS)
     mode = ifq.IFQ_OUT_CODES if pool else ifq.IFQ_OUT_BOTH
-    d = ifq.conv_desc(B, H, W, C, cout, k, s, p, mode, ifq.IFQ_PATH_AUTO, pool=pool, in_bits=8)
-    assert ifq.ifq_conv_plan(d) == ifq.IFQ_PATH_TC
+    d = ifq.conv_desc(B, H, W, C, cout, k, s, p, mode, path, pool=pool, in_bits=8)
+    direct_ok = cout <= 32 and K <= 257
+    assert ifq.ifq_conv_plan(d) == (path if (path == ifq.IFQ_PATH_TC or direct_ok) else ifq.IFQ_PATH_TC)
     T, sg = ifq.ifq_fold_layer(K_fold, prm.alpha, prm.gamma, prm.beta, prm.mean, prm.var, prm.delta_in, None,
                                prm.eps, prm.q_base, prm.q_offset)
     bits = torch.from_numpy(synth.pack_signs(w).view(np.int32)).to(DEV)
