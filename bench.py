@@ -165,13 +165,16 @@ def cpu_baseline(wl, x, params):
     O.build()
     threads = len(os.sched_getaffinity(0))
     n = wl.batch
-    t0 = time.perf_counter()
-    O.forward(wl, x[:n], params, images=list(range(n)), threads=threads)
-    dt = time.perf_counter() - t0
-    ops = sum(conv_ops(l, n) for l in wl.layers if l.kind == "conv")
+    passes, dt = 0, 0.0
+    while passes == 0 or (dt < 10.0 and passes < 50):   # about 10 s of host work, at most 50 passes
+        t0 = time.perf_counter()
+        O.forward(wl, x[:n], params, images=list(range(n)), threads=threads)
+        dt += time.perf_counter() - t0
+        passes += 1
+    ops = passes * sum(conv_ops(l, n) for l in wl.layers if l.kind == "conv")
     return {"value": ops / dt / 1e12, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"all {n} images of the batch through all {len(wl.layers)} layers, float and integer "
-                      f"chains, {dt:.2f} s wall", "images_per_s": n / dt}
+            "sample": f"{passes} passes of all {n} images of the batch through all {len(wl.layers)} layers, "
+                      f"float and integer chains, {dt:.2f} s wall", "images_per_s": passes * n / dt}
 
 
 def run_reference(args):
