@@ -23,6 +23,8 @@
  *   - Device-side failures (a bounded wait that ran out, a failed bounds
  *     check) never trap: they set a device status word that
  *     ifq_device_status reads.
+ *   - A batch of n = 0 images is valid everywhere: arguments are checked as
+ *     usual and nothing is launched.
  *
  * Data formats:
  *   - Codes: NHWC, packed along C in fields of f bits: f = 2 for k = 2 (four
@@ -147,7 +149,7 @@ int ifq_codes_storage_bytes(int n, int h, int w, int c, int kbits, size_t* bytes
  * Convolution descriptor.  Input codes NHWC [n][h][w][cin] (cin % 4 == 0),
  * filters [cout][kh][kw][cin], output [n][ho][wo][cout].  out_mode is one of
  * IFQ_OUT_*; codes output needs cout % 4 == 0.  path selects a kernel path
- * (IFQ_PATH_AUTO lets the library choose).  Limits: all sizes >= 1,
+ * (IFQ_PATH_AUTO lets the library choose).  Limits: n >= 0, all other sizes >= 1,
  * K = kh*kw*cin <= 65536, cout <= 65536, n*ho*wo < 2^31.
  * kbits: the code width k of the input codes and of the output codes (0
  * means 2; 2, 3 or 4, else IFQ_EUNSUPPORTED); the thresholds are then

@@ -360,6 +360,7 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
   if ((d->out_mode & IFQ_OUT_ACC) && !y_acc) return IFQ_EINVAL;
   if (!aligned16(x) || !aligned16(w_prep) || (y_codes && !aligned16(y_codes)) || (y_acc && !aligned16(y_acc)))
     return IFQ_EALIGN;
+  if (g.M == 0) return IFQ_OK;   // an empty batch: nothing to compute
   int nsm = 0;
   if ((rc = ensure_init(&nsm))) return rc;
   uint8_t* yc = (d->out_mode & IFQ_OUT_CODES) ? (uint8_t*)y_codes : nullptr;
@@ -476,6 +477,7 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   if (rc) return rc;
   if (!x || !y) return IFQ_EINVAL;
   if (!aligned16(x) || !aligned16(y)) return IFQ_EALIGN;
+  if (d->n == 0) return IFQ_OK;   // an empty batch
   int nsm = 0;
   if ((rc = ensure_init(&nsm))) return rc;
   PoolArgs a;
@@ -608,6 +610,7 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     ConvGeom g;
     if (check_conv(&layers[i].conv, &g)) return false;
     if (g.pool > 1 || g.kb != 2 || g.in8) return false;   // the persistent kernel: 2-bit codes, no fused pool
+    if (g.M == 0) return false;                           // an empty batch runs (as nothing) layer by layer
     if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
     tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g));
   }

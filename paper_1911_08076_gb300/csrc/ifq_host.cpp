@@ -172,7 +172,7 @@ extern "C" int ifq_codes_storage_bytes(int n, int h, int w, int c, int kbits, si
 
 extern "C" int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo) {
   if (!d || !ho || !wo) return IFQ_EINVAL;
-  if (d->n < 1 || d->h < 1 || d->w < 1 || d->cin < 1 || d->cout < 1 || d->kh < 1 || d->kw < 1 || d->stride < 1 ||
+  if (d->n < 0 || d->h < 1 || d->w < 1 || d->cin < 1 || d->cout < 1 || d->kh < 1 || d->kw < 1 || d->stride < 1 ||
       d->pad < 0)
     return IFQ_ESHAPE;
   const int a = d->h + 2 * d->pad - d->kh, b = d->w + 2 * d->pad - d->kw;
@@ -193,7 +193,7 @@ extern "C" int ifq_conv_out_shape(const ifq_conv_desc* d, int* ho, int* wo) {
 
 extern "C" int ifq_pool_out_shape(const ifq_pool_desc* d, int* ho, int* wo) {
   if (!d || !ho || !wo) return IFQ_EINVAL;
-  if (d->n < 1 || d->h < 1 || d->w < 1 || d->c < 1 || d->k < 1 || d->stride < 1 || d->pad < 0) return IFQ_ESHAPE;
+  if (d->n < 0 || d->h < 1 || d->w < 1 || d->c < 1 || d->k < 1 || d->stride < 1 || d->pad < 0) return IFQ_ESHAPE;
   const int a = d->h + d->pad - d->k, b = d->w + d->pad - d->k;
   if (a < 0 || b < 0) return IFQ_ESHAPE;
   *ho = a / d->stride + 1;

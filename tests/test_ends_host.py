@@ -95,3 +95,22 @@ def test_tinier_yolo_full_layer_table():
     x, params = synth.draw_workload(wl, batch=2)
     assert x.shape == (2, 416, 416, 4) and x[..., 3].max() == 0 and x[..., :3].max() > 200
     assert params[0].delta_in == synth.PIXEL_STEP
+
+
+def test_empty_batch_is_a_validated_no_op():
+    """n = 0: shapes as usual, arguments still checked, nothing launched (so this runs without a GPU)."""
+    d = ifq.conv_desc(0, 14, 14, 64, 64, 3, 1, 1, ifq.IFQ_OUT_BOTH)
+    assert ifq.ifq_conv_out_shape(d) == (14, 14)
+    ifq.ifq_conv2bit(d, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, stream=0)
+    assert _status(ifq.ifq_conv2bit, d, None, FAKE, FAKE, FAKE, FAKE, FAKE, stream=0) == ifq.IFQ_EINVAL
+    assert _status(ifq.ifq_conv2bit, d, FAKE + 4, FAKE, FAKE, FAKE, FAKE, FAKE, stream=0) == ifq.IFQ_EALIGN
+    ifq.ifq_conv2bit(ifq.conv_desc(0, 16, 16, 64, 64, 3, 1, 1, pool=2), FAKE, FAKE, FAKE, FAKE, FAKE, stream=0)
+    ifq.ifq_conv2bit(ifq.conv_desc(0, 16, 16, 4, 8, 3, 1, 1, in_bits=8), FAKE, FAKE, FAKE, FAKE, FAKE, stream=0)
+    p = ifq.pool_desc(0, 8, 8, 64, 2, 2)
+    assert ifq.ifq_pool_out_shape(p) == (4, 4)
+    ifq.ifq_maxpool2bit(p, FAKE, None, FAKE, stream=0)
+    layers = [ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=i - 1, conv=ifq.conv_desc(0, 8, 8, 64, 64, 3, 1, 1),
+                        w_prep=FAKE, thr=FAKE, sign=FAKE, y_codes=FAKE) for i in range(3)]
+    ifq.ifq_forward(layers, FAKE, stream=0)
+    ifq.ifq_forward_noalloc(layers, FAKE, stream=0)
+    assert _status(ifq.ifq_conv_out_shape, ifq.conv_desc(-1, 8, 8, 64, 64, 3)) == ifq.IFQ_ESHAPE

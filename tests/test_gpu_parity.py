@@ -422,3 +422,50 @@ def test_separated_conversion_on_the_kernel(m):
     integ, _ = O.check_chains(A, p, *O.fold(p, K))
     if m <= 8:
         assert (sep != integ).any()
+
+
+# ----------------------------------------------------------------------------- edge cases
+
+@pytest.mark.parametrize("path", [ifq.IFQ_PATH_TC, ifq.IFQ_PATH_BITSERIAL], ids=["tc", "bitserial"])
+def test_maximum_output_channels(path):
+    """cout = 65536, the largest the library accepts: 512 channel tiles of 128 on the tensor cores,
+    1024 blocks of 64 channels on the bit-serial path."""
+    rng = np.random.default_rng(65536)
+    B, H, W, C, cout = 2, 8, 8, 64, 65536
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, 1, 1, C)) == 1, 1, -1).astype(np.int8)
+    prm = _params(rng, cout, C)
+    T, sg = _fold_gpu(prm, C)
+    codes, acc = _run_conv(x, w, T, sg, 1, 0, ifq.IFQ_OUT_BOTH, path)
+    A = O.conv_acc(x, w, 1, 0)
+    assert (acc == A).all()
+    assert (codes == O.int_chain(A, *O.fold(prm, C))).all()
+
+
+@pytest.mark.parametrize("path", [ifq.IFQ_PATH_TC, ifq.IFQ_PATH_BITSERIAL], ids=["tc", "bitserial"])
+def test_all_zero_input(path):
+    """Codes all 0: every accumulator is 0 and every code is #{ i : 0 > T_i } of its channel."""
+    rng = np.random.default_rng(0)
+    B, H, W, C, cout = 2, 9, 9, 64, 96
+    x = np.zeros((B, H, W, C), np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, 3, 3, C)) == 1, 1, -1).astype(np.int8)
+    prm = _params(rng, cout, 9 * C)
+    T, sg = _fold_gpu(prm, 9 * C)
+    codes, acc = _run_conv(x, w, T, sg, 1, 1, ifq.IFQ_OUT_BOTH, path)
+    assert (acc == 0).all()
+    expect = (0 > T.astype(np.int64)).sum(axis=1)
+    assert (codes == expect[None, None, None, :]).all()
+
+
+def test_empty_batch_leaves_outputs_untouched():
+    d = ifq.conv_desc(0, 14, 14, 64, 64, 3, 1, 1, ifq.IFQ_OUT_BOTH)
+    buf = torch.full((4096,), 0x5A, dtype=torch.uint8, device=DEV)
+    acc = torch.full((1024,), 7, dtype=torch.int32, device=DEV)
+    prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=DEV)
+    thr = torch.zeros((64, 3), dtype=torch.int32, device=DEV)
+    sg = torch.ones(64, dtype=torch.int8, device=DEV)
+    ifq.ifq_conv2bit(d, buf, prep, thr, sg, buf, acc)
+    ifq.ifq_maxpool2bit(ifq.pool_desc(0, 8, 8, 64, 2, 2), buf, sg, buf)
+    torch.cuda.synchronize()
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    assert (buf == 0x5A).all() and (acc == 7).all()
