@@ -361,7 +361,10 @@ int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, voi
  * CUDA-graph form of ifq_forward: ifq_graph_create captures the launches of
  * ifq_forward(layers, nlayers, x, ws, ws_bytes) on `stream` into a graph that
  * ifq_graph_launch replays on any stream with the same buffers.  The graph is
- * owned by the returned handle; ifq_graph_destroy frees it.
+ * owned by the returned handle; ifq_graph_destroy frees it.  In the graph a
+ * layer whose output no later layer reads (other than the last layer) hangs
+ * off its source layer as a side branch joined at the end, so it overlaps the
+ * layers after it (IFQ_GRAPH_BRANCH=0 keeps one chain); results are identical.
  */
 typedef struct ifq_graph ifq_graph;
 int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream,

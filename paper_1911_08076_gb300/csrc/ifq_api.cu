@@ -752,25 +752,78 @@ int noalloc_counters(void** out) {
   return IFQ_OK;
 }
 
+int run_layer(const ifq_layer* layers, int i, const void* x, cudaStream_t st) {
+  const ifq_layer& l = layers[i];
+  const void* in = l.src < 0 ? x : layers[l.src].y_codes;
+  if (l.kind == IFQ_LAYER_CONV) return run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st);
+  if (l.kind == IFQ_LAYER_POOL) return run_pool(&l.pool, in, l.sign, l.y_codes, st);
+  const ifq_layer& sl = layers[l.src];
+  ConvGeom g;
+  int rc = check_conv(&sl.conv, &g);
+  if (rc) return rc;
+  return run_fixed(sl.y_acc, sl.conv.n * g.pho * g.pwo, sl.conv.cout, l.fx_mul, l.fx_add, l.fixed.m, l.y_acc, st);
+}
+
 int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t st) {
   for (int i = 0; i < nlayers; ++i) {
-    const ifq_layer& l = layers[i];
-    const void* in = l.src < 0 ? x : layers[l.src].y_codes;
-    int rc;
-    if (l.kind == IFQ_LAYER_CONV) {
-      rc = run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st);
-    } else if (l.kind == IFQ_LAYER_POOL) {
-      rc = run_pool(&l.pool, in, l.sign, l.y_codes, st);
-    } else {
-      const ifq_layer& sl = layers[l.src];
-      ConvGeom g;
-      if ((rc = check_conv(&sl.conv, &g))) return rc;
-      rc = run_fixed(sl.y_acc, sl.conv.n * g.pho * g.pwo, sl.conv.cout, l.fx_mul, l.fx_add, l.fixed.m, l.y_acc, st);
-    }
+    const int rc = run_layer(layers, i, x, st);
     if (rc) return rc;
   }
   return IFQ_OK;
 }
+
+// Stream capture of a stack with its side branches: a layer whose output no later layer reads (a
+// ResNet shortcut conv), other than the last, does not hold up the layers after it, so it runs on a
+// second stream that forks from the main stream when its source layer has run and joins it at the
+// end.  The graph then lets it overlap the main chain, on SMs that under-filled layers leave idle.
+// Outputs are the same; only the graph's edges differ.  The streams and events live until the
+// capture has ended (release()).
+struct BranchedCapture {
+  cudaStream_t side = nullptr;
+  std::vector<cudaEvent_t> events;
+
+  int run(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t main) {
+    std::vector<char> read(nlayers, 0);
+    for (int i = 0; i < nlayers; ++i)
+      if (layers[i].src >= 0) read[layers[i].src] = 1;
+    std::vector<char> is_side(nlayers, 0);
+    int nside = 0;
+    for (int i = 0; i + 1 < nlayers; ++i)
+      if (!read[i]) is_side[i] = 1, ++nside;
+    const char* v = getenv("IFQ_GRAPH_BRANCH");
+    if (nside == 0 || (v && v[0] == '0')) return run_stack(layers, nlayers, x, main);
+    if (cudaStreamCreateWithFlags(&side, cudaStreamNonBlocking) != cudaSuccess) return IFQ_ECUDA;
+    auto fork = [&](int s) -> int {   // side layer s after everything issued so far on main
+      cudaEvent_t e;
+      if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return IFQ_ECUDA;
+      events.push_back(e);
+      if (cudaEventRecord(e, main) != cudaSuccess || cudaStreamWaitEvent(side, e, 0) != cudaSuccess) return IFQ_ECUDA;
+      return run_layer(layers, s, x, side);
+    };
+    int rc;
+    for (int s = 0; s < nlayers; ++s)   // side layers on the stack input fork before anything runs
+      if (is_side[s] && layers[s].src < 0 && (rc = fork(s))) return rc;
+    for (int i = 0; i < nlayers; ++i) {
+      if (is_side[i]) continue;
+      if ((rc = run_layer(layers, i, x, main))) return rc;
+      for (int s = i + 1; s < nlayers; ++s)
+        if (is_side[s] && layers[s].src == i && (rc = fork(s))) return rc;
+    }
+    cudaEvent_t join;
+    if (cudaEventCreateWithFlags(&join, cudaEventDisableTiming) != cudaSuccess) return IFQ_ECUDA;
+    events.push_back(join);
+    if (cudaEventRecord(join, side) != cudaSuccess || cudaStreamWaitEvent(main, join, 0) != cudaSuccess)
+      return IFQ_ECUDA;
+    return IFQ_OK;
+  }
+
+  void release() {
+    for (cudaEvent_t e : events) cudaEventDestroy(e);
+    events.clear();
+    if (side) cudaStreamDestroy(side);
+    side = nullptr;
+  }
+};
 
 }  // namespace
 
@@ -886,8 +939,11 @@ int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* 
   rc = IFQ_OK;
   if (cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) rc = IFQ_ECUDA;
   if (!rc) {
-    const int frc = ifq_forward(layers, nlayers, x, ws, ws_bytes, cap);
+    BranchedCapture bc;
+    int frc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, cap);
+    if (frc == IFQ_EUNSUPPORTED) frc = bc.run(layers, nlayers, x, cap);
     const cudaError_t e = cudaStreamEndCapture(cap, &g->graph);
+    bc.release();
     if (frc) rc = frc;
     else if (e != cudaSuccess) rc = IFQ_ECUDA;
   }
