@@ -245,16 +245,44 @@ bool direct_supported(const ifq_conv_desc* d, const ConvGeom& g) {
   return g.in8 && d->cout <= kDirectMaxCout && g.K <= kDirectMaxK;
 }
 
+// The narrow bit-serial kernel: 2-bit codes, cin 4, 8 or 16, 3x3, stride 1, cout <= 32 (and a
+// multiple of 4), pool 1 or 2.
+bool narrow_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  return g.kb == 2 && !g.in8 && (d->cin == 4 || d->cin == 8 || d->cin == 16) && d->kh == 3 && d->kw == 3 &&
+         d->stride == 1 && d->cout <= 32 && d->cout % 4 == 0 && (g.pool == 1 || g.pool == 2);
+}
+
+// Where the narrow kernel beats the tensor cores (measured on GB300): the narrowest layers, whose
+// 128-pixel tiles of one K stage each are per-tile-overhead bound on the tensor cores.
+bool narrow_wins(const ifq_conv_desc* d, const ConvGeom& g) {
+  return narrow_supported(d, g) && d->cin * d->cout <= 128;
+}
+
+// The narrow bit-serial kernel instance for cin, pool and the channel bound.
+template <int CIN, int P>
+cudaError_t launch_narrow_cp(int cout, dim3 grid, dim3 block, const NarrowArgs& a, cudaStream_t st) {
+  if (cout <= 8) return launch_k(conv_bitserial_narrow_kernel<CIN, P, 8>, grid, block, 0, st, a);
+  if (cout <= 16) return launch_k(conv_bitserial_narrow_kernel<CIN, P, 16>, grid, block, 0, st, a);
+  return launch_k(conv_bitserial_narrow_kernel<CIN, P, 32>, grid, block, 0, st, a);
+}
+
+cudaError_t launch_narrow(int cin, int pool, int cout, dim3 grid, dim3 block, const NarrowArgs& a, cudaStream_t st) {
+  if (cin == 4) return pool == 2 ? launch_narrow_cp<4, 2>(cout, grid, block, a, st) : launch_narrow_cp<4, 1>(cout, grid, block, a, st);
+  if (cin == 8) return pool == 2 ? launch_narrow_cp<8, 2>(cout, grid, block, a, st) : launch_narrow_cp<8, 1>(cout, grid, block, a, st);
+  return pool == 2 ? launch_narrow_cp<16, 2>(cout, grid, block, a, st) : launch_narrow_cp<16, 1>(cout, grid, block, a, st);
+}
+
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
-    path = forced ? forced : (direct_supported(d, g) ? IFQ_PATH_DIRECT : IFQ_PATH_TC);
+    path = forced ? forced
+                  : (direct_supported(d, g) ? IFQ_PATH_DIRECT : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL : IFQ_PATH_TC));
   }
   if (path == IFQ_PATH_DIRECT && !direct_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
-  // the fused pool and 8-bit inputs have no bit-serial form
-  if ((g.pool > 1 || g.in8) && path == IFQ_PATH_BITSERIAL) return -1;
+  // the fused pool has a bit-serial form only in the narrow kernel; 8-bit inputs have none
+  if (path == IFQ_PATH_BITSERIAL && (g.in8 || (g.pool > 1 && !narrow_supported(d, g)))) return -1;
   return path;
 }
 
@@ -417,6 +445,21 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
       if (gb == 16) e = launch_tc_gb<16, 4, 2>(bn, tm, a, nsm, st);
       else e = launch_tc_gb<4, 4, 2>(bn, tm, a, nsm, st);
     }
+  } else if (narrow_supported(d, g)) {
+    NarrowArgs a;
+    a.x = (const uint8_t*)x;
+    a.wbits = (const uint32_t*)((const uint8_t*)w_prep + prep_bits_offset(d, g));
+    a.thr = thr;
+    a.sign = sign;
+    a.y_codes = yc;
+    a.y_acc = ya;
+    a.n = d->n; a.h = d->h; a.w = d->w; a.cout = d->cout; a.pad = d->pad;
+    a.ho = g.ho; a.wo = g.wo; a.pho = g.pho; a.pwo = g.pwo; a.kwords = g.kwords;
+    a.total = d->n * g.pho * g.pwo;
+    a.div_pwo = make_fastdiv((uint32_t)g.pwo);
+    a.div_pho = make_fastdiv((uint32_t)g.pho);
+    const dim3 grid(launch_1d_blocks((size_t)a.total, kNarrowThreads, nsm)), block(kNarrowThreads);
+    e = launch_narrow(d->cin, g.pool, d->cout, grid, block, a, st);
   } else {
     BsArgs a;
     a.x = (const uint8_t*)x;

@@ -469,3 +469,40 @@ def test_empty_batch_leaves_outputs_untouched():
     torch.cuda.synchronize()
     assert ifq.ifq_device_status() == ifq.IFQ_OK
     assert (buf == 0x5A).all() and (acc == 7).all()
+
+
+NARROW_CASES = [
+    # B, H, W, C, cout, pool: the narrow bit-serial kernel (3x3, stride 1, pad 1)
+    (2, 20, 20, 8, 16, 0),
+    (2, 20, 20, 8, 16, 2),
+    (3, 13, 11, 4, 8, 0),
+    (2, 18, 14, 4, 12, 2),
+    (2, 11, 9, 16, 32, 0),
+    (2, 16, 16, 16, 32, 2),
+    (1, 7, 9, 16, 4, 0),
+]
+
+
+@pytest.mark.parametrize("case", NARROW_CASES, ids=[str(c) for c in NARROW_CASES])
+def test_narrow_bitserial_matches_oracle(case):
+    """The narrow bit-serial kernel (interleaved-code popcounts, one thread per output or pooled
+    pixel), bit-exact, with negative BN scales, alone and with the fused pool."""
+    B, H, W, C, cout, pool = case
+    rng = np.random.default_rng(abs(hash(case)) % (2 ** 32))
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, 3, 3, C)) == 1, 1, -1).astype(np.int8)
+    K = 9 * C
+    prm = _params(rng, cout, K)
+    prm.gamma[1::3] = -np.abs(prm.gamma[1::3])
+    T, sg = _fold_gpu(prm, K)
+    mode = ifq.IFQ_OUT_CODES if pool else ifq.IFQ_OUT_BOTH
+    assert ifq.ifq_conv_plan(ifq.conv_desc(B, H, W, C, cout, 3, 1, 1, mode, ifq.IFQ_PATH_BITSERIAL, pool=pool)) == \
+        ifq.IFQ_PATH_BITSERIAL
+    codes, acc = _run_conv(x, w, T, sg, 1, 1, mode, ifq.IFQ_PATH_BITSERIAL, pool=pool)
+    A = O.conv_acc(x, w, 1, 1)
+    if pool:
+        ref = O.int_chain(O.maxpool_acc(A, pool, pool, 0), *O.fold(prm, K))
+    else:
+        assert (acc == A).all()
+        ref = O.int_chain(A, *O.fold(prm, K))
+    assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
