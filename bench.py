@@ -391,27 +391,33 @@ def run_ours(args):
         conv_bytes_total = sum(alg_bytes(wl.layers[i], B, wl.kbits) for i in conv_idx)
 
         # ---------------- end to end through the C ABI with host buffers
-        leaves = st.leaf_layers()
-        outs_dev = [st.y_codes[li] if li in st.y_codes else st.y_acc[li] for li in leaves]
-        outs_host = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outs_dev]
+        # every result (the leaf layers' outputs) sits in one contiguous device block: one copy back
+        outs_dev = [st.leaf_block]
+        outs_host = [torch.empty(st.leaf_block.shape, dtype=torch.uint8).pin_memory()]
         h2d = x_host.numel() * x_host.element_size()
         d2h = sum(t.numel() * t.element_size() for t in outs_dev)
         KE = min(K, 1000)
         es = [torch.cuda.Event(enable_timing=True) for _ in range(KE)]
         ee = [torch.cuda.Event(enable_timing=True) for _ in range(KE)]
-        for i in range(min(W, 20)):
-            xd.copy_(x_host, non_blocking=True)
-            st.replay(stream)
+        # input in and results out through the library's copy (on the SMs, over the CPU-GPU link)
+        def copy_in():
+            ifq.ifq_copy_bytes(xd, x_host, x_host.numel() * x_host.element_size(), stream)
+
+        def copy_out():
             for h, d in zip(outs_host, outs_dev):
-                h.copy_(d, non_blocking=True)
+                ifq.ifq_copy_bytes(h, d, d.numel() * d.element_size(), stream)
+
+        for i in range(min(W, 20)):
+            copy_in()
+            st.replay(stream)
+            copy_out()
         torch.cuda.synchronize()
         barrier()
         for i in range(KE):
             es[i].record(stream)
-            xd.copy_(x_host, non_blocking=True)
+            copy_in()
             st.replay(stream)
-            for h, d in zip(outs_host, outs_dev):
-                h.copy_(d, non_blocking=True)
+            copy_out()
             ee[i].record(stream)
             flush.fill_(i & 0xFF)
         torch.cuda.synchronize()

@@ -385,6 +385,17 @@ int ifq_unpack_codes_kbits(const void* packed, uint8_t* codes, size_t n, int kbi
 int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* stream);
 
 /*
+ * ifq_copy_bytes -- copy n bytes on `stream` (either side may be device memory
+ * or pinned host memory that the device addresses directly under unified
+ * addressing).  With both pointers 16-byte aligned, n % 16 == 0 and both
+ * addressable by the device at the same address (device memory, or host memory
+ * from cudaHostAlloc / cudaHostRegister), the SMs do the copy with 16-byte loads
+ * and stores (on a GB300 over NVLink-C2C for host memory); otherwise it is
+ * cudaMemcpyAsync.  For staging a stack's inputs and results.
+ */
+int ifq_copy_bytes(void* dst, const void* src, size_t n, void* stream);
+
+/*
  * ifq_device_status -- synchronize `stream`, then read and clear the device
  * status word of the current device: IFQ_OK, or the first device-side error
  * recorded (IFQ_ETIMEOUT, IFQ_ERANGE) since the last read.

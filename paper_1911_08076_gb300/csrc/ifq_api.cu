@@ -1064,6 +1064,33 @@ int ifq_fixed_output(const int32_t* acc, int rows, int cout, const int64_t* mul,
   return run_fixed(acc, rows, cout, mul, add, m, y, S(stream));
 }
 
+// Whether the device can dereference p as is: device or managed memory, or host memory that
+// cudaHostAlloc / cudaHostRegister mapped at the same address (unified addressing).
+bool device_addressable(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();   // an unregistered pointer is not an error to keep
+    return false;
+  }
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) return true;
+  return at.type == cudaMemoryTypeHost && at.devicePointer == p;
+}
+
+int ifq_copy_bytes(void* dst, const void* src, size_t n, void* stream) {
+  if ((!dst || !src) && n) return IFQ_EINVAL;
+  if (n == 0) return IFQ_OK;
+  if (!aligned16(dst) || !aligned16(src) || n % 16 != 0 || !device_addressable(dst) || !device_addressable(src))
+    return cudaMemcpyAsync(dst, src, n, cudaMemcpyDefault, S(stream)) == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+  int nsm = 0, rc;
+  if ((rc = ensure_init(&nsm))) return rc;
+  const size_t n16 = n / 16;
+  size_t blocks = (n16 + 255) / 256;
+  if (blocks > (size_t)nsm * 8) blocks = (size_t)nsm * 8;
+  const cudaError_t e = launch_k(copy16_kernel, dim3((unsigned)blocks), dim3(256), 0, S(stream), (const uint4*)src,
+                                 (uint4*)dst, n16);
+  return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
 int ifq_device_status(void* stream, int* status) {
   if (!status) return IFQ_EINVAL;
   if (cudaStreamSynchronize(S(stream)) != cudaSuccess) return IFQ_ECUDA;

@@ -201,6 +201,16 @@ __global__ void fixed_output_kernel(const int32_t* acc, int total, FastDiv div_c
 
 // ---------------------------------------------------------------- packing
 
+// 16-byte vector copy on the SMs (either side may be host memory the device addresses directly:
+// pinned host memory under unified addressing, read or written over the CPU-GPU link).
+__global__ void copy16_kernel(const uint4* src, uint4* dst, size_t n16) {
+  grid_dep_launch();
+  grid_dep_wait();
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (size_t)gridDim.x * blockDim.x)
+    dst[i] = src[i];
+}
+
+
 // one code per byte <-> SB-bit fields, 8/SB codes per packed byte (codes keep their low SB bits)
 template <int SB>
 __global__ void pack_codes_kernel(const uint8_t* codes, uint8_t* packed, size_t nbytes) {

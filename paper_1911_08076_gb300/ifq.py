@@ -85,6 +85,7 @@ _SIGS = {
     "ifq_pack_codes_kbits": ([_P, _P, _SZ, _I, _P], _I),
     "ifq_unpack_codes_kbits": ([_P, _P, _SZ, _I, _P], _I),
     "ifq_pack_signs": ([_P, _P, _I, _I, _P], _I),
+    "ifq_copy_bytes": ([_P, _P, _SZ, _P], _I),
     "ifq_device_status": ([_P, ctypes.POINTER(_I)], _I),
 }
 
@@ -316,6 +317,10 @@ def ifq_unpack_codes_kbits(packed, codes, n: int, kbits: int, stream=None):
 
 def ifq_pack_signs(w, bits, rows: int, K: int, stream=None):
     _ok(lib().ifq_pack_signs(_ptr(w), _ptr(bits), rows, K, _stream(stream)), "ifq_pack_signs")
+
+
+def ifq_copy_bytes(dst, src, n: int, stream=None):
+    _ok(lib().ifq_copy_bytes(_ptr(dst), _ptr(src), n, _stream(stream)), "ifq_copy_bytes")
 
 
 def ifq_device_status(stream=None) -> int:

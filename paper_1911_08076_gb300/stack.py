@@ -36,6 +36,31 @@ class DeviceStack:
         self.fx: Dict[int, tuple] = {}
         B = self.batch
         kinds = {"conv": ifq.IFQ_LAYER_CONV, "pool": ifq.IFQ_LAYER_POOL, "fixed": ifq.IFQ_LAYER_FIXED}
+        # The outputs of the leaf layers (the stack's results) share one contiguous block, so that a
+        # caller reads every result back with one copy.
+        leaves = set(self.leaf_layers())
+        specs = []
+        for li in sorted(leaves):
+            for shape, dtype in self._out_specs(li, B, fb):
+                specs.append((li, shape, dtype))
+        offs, total = [], 0
+        for _, shape, dtype in specs:
+            offs.append(total)
+            nbytes = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+            total += (nbytes + 255) // 256 * 256
+        self.leaf_block = torch.empty(max(total, 1), dtype=torch.uint8, device=self.device)
+        self._leaf_out = {}
+        for (li, shape, dtype), off in zip(specs, offs):
+            nbytes = int(np.prod(shape)) * torch.empty((), dtype=dtype).element_size()
+            self._leaf_out.setdefault(li, []).append(self.leaf_block[off:off + nbytes].view(dtype).view(shape))
+
+        def out(li, shape, dtype):
+            if li in self._leaf_out:
+                t = self._leaf_out[li].pop(0)
+                assert tuple(t.shape) == tuple(shape) and t.dtype == dtype, (li, t.shape, shape)
+                return t
+            return torch.empty(shape, dtype=dtype, device=self.device)
+
         for li, l in enumerate(workload.layers):
             rec = ifq.Layer()
             rec.kind = kinds[l.kind]
@@ -63,10 +88,9 @@ class DeviceStack:
                 ho, wo = ifq.ifq_conv_out_shape(d)   # after the fused pool, if any
                 assert (ho, wo) == (l.out_h, l.out_w), (l.name, ho, wo)
                 if mode & ifq.IFQ_OUT_CODES:
-                    self.y_codes[li] = torch.empty((B, ho, wo, l.cout * fb // 8), dtype=torch.uint8,
-                                                   device=self.device)
+                    self.y_codes[li] = out(li, (B, ho, wo, l.cout * fb // 8), torch.uint8)
                 if mode & ifq.IFQ_OUT_ACC:
-                    self.y_acc[li] = torch.empty((B, ho, wo, l.cout), dtype=torch.int32, device=self.device)
+                    self.y_acc[li] = out(li, (B, ho, wo, l.cout), torch.int32)
                 rec.conv = d
                 rec.w_prep = prep.data_ptr()
                 rec.thr = self.thr[li].data_ptr()
@@ -77,7 +101,7 @@ class DeviceStack:
                 sl, sp = workload.layers[l.src], params[l.src]
                 mul, add = ifq.ifq_fold_output_separated(l.m, sp.alpha, sp.delta_in, sp.bias)
                 self.fx[li] = (torch.from_numpy(mul).to(self.device), torch.from_numpy(add).to(self.device))
-                self.y_acc[li] = torch.empty((B, sl.out_h, sl.out_w, sl.cout), dtype=torch.int32, device=self.device)
+                self.y_acc[li] = out(li, (B, sl.out_h, sl.out_w, sl.cout), torch.int32)
                 rec.fixed = ifq.FixedDesc(l.m)
                 rec.fx_mul = self.fx[li][0].data_ptr()
                 rec.fx_add = self.fx[li][1].data_ptr()
@@ -86,7 +110,7 @@ class DeviceStack:
                 d = ifq.pool_desc(B, l.h, l.w, l.c, l.k, l.stride, l.pad, kbits)
                 ho, wo = ifq.ifq_pool_out_shape(d)
                 assert (ho, wo) == (l.ho, l.wo), (l.name, ho, wo)
-                self.y_codes[li] = torch.empty((B, ho, wo, l.c * fb // 8), dtype=torch.uint8, device=self.device)
+                self.y_codes[li] = out(li, (B, ho, wo, l.c * fb // 8), torch.uint8)
                 rec.pool = d
                 rec.sign = self.sign[l.src].data_ptr() if l.signed else None
                 rec.y_codes = self.y_codes[li].data_ptr()
@@ -94,6 +118,21 @@ class DeviceStack:
         self.ws_bytes = ifq.ifq_forward_workspace_bytes(self.layers)
         self.ws = torch.empty(max(self.ws_bytes, 1), dtype=torch.uint8, device=self.device)
         self._graph = None
+
+    def _out_specs(self, li: int, B: int, fb: int):
+        """(shape, dtype) of each output buffer of layer li, in the order the constructor makes them."""
+        l = self.wl.layers[li]
+        if l.kind == "conv":
+            specs = []
+            if l.out in ("codes", "both"):
+                specs.append(((B, l.out_h, l.out_w, l.cout * fb // 8), torch.uint8))
+            if l.out in ("acc", "both"):
+                specs.append(((B, l.out_h, l.out_w, l.cout), torch.int32))
+            return specs
+        if l.kind == "fixed":
+            sl = self.wl.layers[l.src]
+            return [((B, sl.out_h, sl.out_w, sl.cout), torch.int32)]
+        return [((B, l.ho, l.wo, l.c * fb // 8), torch.uint8)]
 
     def input_buffer(self) -> torch.Tensor:
         wl = self.wl

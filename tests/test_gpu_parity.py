@@ -506,3 +506,23 @@ def test_narrow_bitserial_matches_oracle(case):
         assert (acc == A).all()
         ref = O.int_chain(A, *O.fold(prm, K))
     assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
+
+
+def test_copy_bytes_between_device_and_host():
+    """ifq_copy_bytes: the SM copy between device memory and pinned host memory, and the
+    cudaMemcpyAsync fallback for unaligned sizes and for pageable host memory."""
+    rng = np.random.default_rng(16)
+    src = torch.from_numpy(rng.integers(0, 256, 1 << 20, dtype=np.uint8)).pin_memory()
+    dev = torch.empty(1 << 20, dtype=torch.uint8, device=DEV)
+    ifq.ifq_copy_bytes(dev, src, 1 << 20)                          # pinned host -> device (SMs)
+    back = torch.zeros(1 << 20, dtype=torch.uint8).pin_memory()
+    ifq.ifq_copy_bytes(back, dev, 1 << 20)                         # device -> pinned host (SMs)
+    torch.cuda.synchronize()
+    assert torch.equal(back, src)
+    odd = torch.zeros(1 << 20, dtype=torch.uint8).pin_memory()
+    ifq.ifq_copy_bytes(odd, dev, 1000003)                          # size not a multiple of 16
+    pageable = torch.zeros(1 << 20, dtype=torch.uint8)
+    ifq.ifq_copy_bytes(pageable, dev, 1 << 20)                     # pageable host: cudaMemcpyAsync
+    torch.cuda.synchronize()
+    assert torch.equal(odd[:1000003], src[:1000003]) and (odd[1000003:] == 0).all()
+    assert torch.equal(pageable, src)
