@@ -283,6 +283,22 @@ def measure_pool_hbm(ifq, torch, dev, stream, flush, reps=20):
             "l2": "not flushed: input (177 MB) larger than L2 (129 MB)"}
 
 
+def reduce_max(v: float, world: int, device) -> float:
+    """The maximum of v over all ranks (the slowest replica sets the job's step time)."""
+    if world == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ops_per_rank_step: float, world: int, step_ms_max: float) -> float:
+    """Whole-job TOPS of `world` replicas, each doing ops_per_rank_step per step, at the max step time."""
+    return world * ops_per_rank_step / (step_ms_max * 1e-3) / 1e12
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -301,11 +317,7 @@ def run_ours(args):
             dist.barrier()
 
     def max_over_ranks(v):
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(v, world, dev)
 
     wl = synth.get(args.workload, args.batch)
     B = wl.batch
@@ -424,7 +436,7 @@ def run_ours(args):
         e2e_ms = max_over_ranks(sum(s.elapsed_time(e) for s, e in zip(es, ee)) / KE)
 
     pool_hbm = measure_pool_hbm(ifq, torch, dev, stream, flush)
-    value = world * ops / (step_ms * 1e-3) / 1e12
+    value = job_throughput(ops, world, step_ms)
     imgs = world * B / (step_ms * 1e-3)
     bf16, bf16_sus, hbm, src = read_peaks()
     peak = bf16 * FP8_PER_BF16

@@ -1,0 +1,66 @@
+"""The N > 1 paths on the CPU (gloo, world size 2): the replicas-only aggregation of bench.py (no
+data-path collective: each rank runs its own replica; the job's step time is the slowest rank's,
+and the job's throughput counts every rank's work) and the reference arm launched the way the
+driver launches a multi-GPU bench (rank 0 alone runs and prints; the other ranks exit 0)."""
+import json
+import os
+import socket
+import subprocess
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(HERE)
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _replica(rank, world, port, out):
+    import torch
+    import torch.distributed as dist
+    sys.path.insert(0, ROOT)
+    import bench
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world)
+    step_ms = 1.0 + rank                           # rank 1 is the slower replica
+    slowest = bench.reduce_max(step_ms, world, "cpu")
+    value = bench.job_throughput(1e12, world, slowest)
+    dist.barrier()
+    out.put((rank, slowest, value))
+    dist.destroy_process_group()
+
+
+def test_replica_aggregation_on_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_replica, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(out.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    # both ranks see the slowest step (2 ms); the job does 2 x 1e12 ops per 2 ms = 1000 TOPS
+    assert [r[1] for r in res] == [2.0, 2.0]
+    assert all(abs(r[2] - 1000.0) < 1e-9 for r in res)
+
+
+def test_reference_arm_under_torchrun_two_ranks():
+    port = _free_port()
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--impl", "reference",
+           "--gpus", "2", "--steps", "2", "--warmup", "3"]
+    r = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600,
+                       env=dict(os.environ, OMP_NUM_THREADS="1"))
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
