@@ -396,6 +396,15 @@ int ifq_pack_signs(const int8_t* w, uint32_t* bits, int rows, int K, void* strea
 int ifq_copy_bytes(void* dst, const void* src, size_t n, void* stream);
 
 /*
+ * ifq_wait_selftest -- exercise the failure path of the bounded device waits:
+ * one warp waits on an mbarrier phase that nothing completes for limit_us
+ * microseconds (1..1000000), then records IFQ_ETIMEOUT in the device status
+ * word and returns normally, as every kernel's waits do after 2 s.  Read it
+ * with ifq_device_status; the context stays usable.
+ */
+int ifq_wait_selftest(int limit_us, void* stream);
+
+/*
  * ifq_device_status -- synchronize `stream`, then read and clear the device
  * status word of the current device: IFQ_OK, or the first device-side error
  * recorded (IFQ_ETIMEOUT, IFQ_ERANGE) since the last read.

@@ -19,6 +19,7 @@
 #include "conv_tc.cuh"
 #include "ifq.h"
 #include "pool_pack.cuh"
+#include "selftest.cuh"
 #include "stack_tc.cuh"
 
 namespace {
@@ -1089,6 +1090,14 @@ int ifq_copy_bytes(void* dst, const void* src, size_t n, void* stream) {
   const cudaError_t e = launch_k(copy16_kernel, dim3((unsigned)blocks), dim3(256), 0, S(stream), (const uint4*)src,
                                  (uint4*)dst, n16);
   return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+}
+
+int ifq_wait_selftest(int limit_us, void* stream) {
+  if (limit_us < 1 || limit_us > 1000000) return IFQ_EINVAL;
+  int rc;
+  if ((rc = ensure_init(nullptr))) return rc;
+  wait_selftest_kernel<<<1, 32, 0, S(stream)>>>((unsigned long long)limit_us * 1000ull);
+  return cudaGetLastError() == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
 }
 
 int ifq_device_status(void* stream, int* status) {

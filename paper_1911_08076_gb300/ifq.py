@@ -86,6 +86,7 @@ _SIGS = {
     "ifq_unpack_codes_kbits": ([_P, _P, _SZ, _I, _P], _I),
     "ifq_pack_signs": ([_P, _P, _I, _I, _P], _I),
     "ifq_copy_bytes": ([_P, _P, _SZ, _P], _I),
+    "ifq_wait_selftest": ([_I, _P], _I),
     "ifq_device_status": ([_P, ctypes.POINTER(_I)], _I),
 }
 
@@ -321,6 +322,10 @@ def ifq_pack_signs(w, bits, rows: int, K: int, stream=None):
 
 def ifq_copy_bytes(dst, src, n: int, stream=None):
     _ok(lib().ifq_copy_bytes(_ptr(dst), _ptr(src), n, _stream(stream)), "ifq_copy_bytes")
+
+
+def ifq_wait_selftest(limit_us: int, stream=None):
+    _ok(lib().ifq_wait_selftest(int(limit_us), _stream(stream)), "ifq_wait_selftest")
 
 
 def ifq_device_status(stream=None) -> int:

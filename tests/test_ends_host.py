@@ -114,3 +114,8 @@ def test_empty_batch_is_a_validated_no_op():
     ifq.ifq_forward(layers, FAKE, stream=0)
     ifq.ifq_forward_noalloc(layers, FAKE, stream=0)
     assert _status(ifq.ifq_conv_out_shape, ifq.conv_desc(-1, 8, 8, 64, 64, 3)) == ifq.IFQ_ESHAPE
+
+
+def test_wait_selftest_refuses_bad_limits():
+    assert _status(ifq.ifq_wait_selftest, 0, stream=0) == ifq.IFQ_EINVAL
+    assert _status(ifq.ifq_wait_selftest, 2000000, stream=0) == ifq.IFQ_EINVAL

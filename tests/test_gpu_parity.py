@@ -526,3 +526,21 @@ def test_copy_bytes_between_device_and_host():
     torch.cuda.synchronize()
     assert torch.equal(odd[:1000003], src[:1000003]) and (odd[1000003:] == 0).all()
     assert torch.equal(pageable, src)
+
+
+def test_bounded_wait_reports_timeout_and_the_context_survives():
+    """A wait that nothing completes runs out after its limit, sets IFQ_ETIMEOUT in the device status
+    word (read and cleared by ifq_device_status) and returns; kernels run normally afterwards."""
+    assert ifq.ifq_device_status() == ifq.IFQ_OK
+    t0 = __import__("time").perf_counter()
+    ifq.ifq_wait_selftest(20000)                      # 20 ms
+    assert ifq.ifq_device_status() == ifq.IFQ_ETIMEOUT
+    assert __import__("time").perf_counter() - t0 >= 0.019
+    assert ifq.ifq_device_status() == ifq.IFQ_OK      # cleared by the read
+    rng = np.random.default_rng(5)
+    x = rng.integers(0, 4, (1, 8, 8, 64), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (64, 3, 3, 64)) == 1, 1, -1).astype(np.int8)
+    prm = _params(rng, 64, 576)
+    T, sg = _fold_gpu(prm, 576)
+    codes, acc = _run_conv(x, w, T, sg, 1, 1, ifq.IFQ_OUT_BOTH, ifq.IFQ_PATH_TC)
+    assert (acc == O.conv_acc(x, w, 1, 1)).all()
