@@ -126,22 +126,32 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_kernel(const Direc
   }
 }
 
+// a . b + c over four byte lanes, a unsigned (pixel values), b signed (+-1 weights).
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
+  int d;
+  asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
 // The common first layer: cin = 4 (RGB and a zero channel: one 32-bit word per pixel), 3x3,
-// stride 1, pool P = 1 or 2.  The (P + 2)^2 input words of a thread's window are loaded first (all
-// in flight together, each reused by up to P^2 conv pixels), and the loop runs over the 36 taps
-// outermost, so each tap's pair masks are loaded once for the P^2 conv pixels.
-template <int NP, int P>
+// stride 1, pool P = 1 or 2.  A tap is one word of four 8-bit values, so A[n] is nine dp4a of the
+// pixel words with filter n's +-1 byte words (0x01 / 0xFF).  The (P + 2)^2 input words of a
+// thread's window are loaded first, and the loop runs over the 9 taps outermost, so each tap's
+// weight words are read once for the P^2 conv pixels.
+template <int NC, int P>
 __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const DirectArgs a) {
-  constexpr int KS = 3, WIN = P + KS - 1, K = KS * KS * 4;
-  __shared__ __align__(16) uint32_t sM[K * NP];
-  __shared__ int32_t sT[2 * NP * 15];
-  __shared__ int32_t sS[2 * NP];
+  constexpr int KS = 3, WIN = P + KS - 1, TAPS = KS * KS;
+  __shared__ __align__(16) uint32_t sW[TAPS * NC];   // [tap][n] +-1 byte words
+  __shared__ int32_t sT[NC * 15];
+  __shared__ int32_t sS[NC];
   grid_dep_launch();
   grid_dep_wait();
-  for (int i = threadIdx.x; i < K * NP; i += blockDim.x) {
-    const int k = i / NP, j = i - k * NP;
-    const uint32_t mk = a.wmask[k];
-    sM[i] = ((mk >> (2 * j)) & 1u) | (((mk >> (2 * j + 1)) & 1u) << 16);
+  for (int i = threadIdx.x; i < TAPS * NC; i += blockDim.x) {
+    const int t = i / NC, n = i - t * NC;
+    uint32_t wv = 0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) wv |= (((a.wmask[4 * t + c] >> n) & 1u) ? 0x01u : 0xFFu) << (8 * c);
+    sW[i] = wv;
   }
   if (a.thr)
     for (int i = threadIdx.x; i < a.cout * a.lvl; i += blockDim.x) sT[i] = a.thr[i];
@@ -164,48 +174,35 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
         const bool in = (unsigned)iy < (unsigned)a.h && (unsigned)ix < (unsigned)a.w;   // else zero padding
         win[wy * WIN + wx] = in ? __ldg(x32 + ((size_t)b * a.h + iy) * a.w + ix) : 0u;
       }
-    uint32_t Pp[P * P][NP];
-    int S[P * P];
+    int acc[P * P][NC];
 #pragma unroll
-    for (int q = 0; q < P * P; ++q) {
-      S[q] = 0;
+    for (int q = 0; q < P * P; ++q)
 #pragma unroll
-      for (int j = 0; j < NP; ++j) Pp[q][j] = 0;
-    }
+      for (int n = 0; n < NC; ++n) acc[q][n] = 0;
 #pragma unroll
     for (int dy = 0; dy < KS; ++dy)
 #pragma unroll
-      for (int dx = 0; dx < KS; ++dx)
+      for (int dx = 0; dx < KS; ++dx) {
+        const uint32_t* wt = sW + (dy * KS + dx) * NC;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const uint32_t* m = sM + ((dy * KS + dx) * 4 + c) * NP;
-          uint32_t mv[NP];
+        for (int n = 0; n < NC; ++n) {
+          const uint32_t wv = wt[n];
 #pragma unroll
-          for (int j = 0; j < NP; ++j) mv[j] = m[j];
-#pragma unroll
-          for (int q = 0; q < P * P; ++q) {
-            const uint32_t xv = (win[(q / P + dy) * WIN + (q % P + dx)] >> (8 * c)) & 0xFFu;
-            S[q] += (int)xv;
-#pragma unroll
-            for (int j = 0; j < NP; ++j) Pp[q][j] += xv * mv[j];
-          }
+          for (int q = 0; q < P * P; ++q) acc[q][n] = dp4a_us(win[(q / P + dy) * WIN + (q % P + dx)], wv, acc[q][n]);
         }
-    int amax[2 * NP];
-#pragma unroll
-    for (int j = 0; j < NP; ++j) {
-      int a0 = INT32_MIN, a1 = INT32_MIN;
-#pragma unroll
-      for (int q = 0; q < P * P; ++q) {
-        a0 = max(a0, 2 * (int)(Pp[q][j] & 0xFFFFu) - S[q]);
-        a1 = max(a1, 2 * (int)(Pp[q][j] >> 16) - S[q]);
       }
-      amax[2 * j] = a0;
-      amax[2 * j + 1] = a1;
+    int amax[NC];
+#pragma unroll
+    for (int n = 0; n < NC; ++n) {
+      int m = acc[0][n];
+#pragma unroll
+      for (int q = 1; q < P * P; ++q) m = max(m, acc[q][n]);
+      amax[n] = m;
     }
     if (P == 1 && a.y_acc) {
       int32_t* dst = a.y_acc + (size_t)it * a.cout;
 #pragma unroll
-      for (int n = 0; n < 2 * NP; ++n)
+      for (int n = 0; n < NC; ++n)
         if (n < a.cout) dst[n] = amax[n];
     }
     if (a.y_codes) {
@@ -213,7 +210,7 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
       uint32_t byte = 0;
       int nbits = 0, bi = 0;
 #pragma unroll
-      for (int n = 0; n < 2 * NP; ++n) {
+      for (int n = 0; n < NC; ++n) {
         if (n < a.cout) {
           const int sv = sS[n] * amax[n];
           uint32_t code = 0;

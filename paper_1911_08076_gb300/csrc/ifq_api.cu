@@ -420,11 +420,11 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     // the RGB first layer (cin 4, 3x3, stride 1, pool 1 or 2) has its own instances
     const bool rgb3 = d->cin == 4 && d->kh == 3 && d->kw == 3 && d->stride == 1 && (g.pool == 1 || g.pool == 2);
     if (rgb3 && d->cout <= 8)
-      e = g.pool == 2 ? launch_k(conv_direct_rgb3_kernel<4, 2>, grid, block, 0, st, a)
-                      : launch_k(conv_direct_rgb3_kernel<4, 1>, grid, block, 0, st, a);
-    else if (rgb3 && d->cout <= 16)
       e = g.pool == 2 ? launch_k(conv_direct_rgb3_kernel<8, 2>, grid, block, 0, st, a)
                       : launch_k(conv_direct_rgb3_kernel<8, 1>, grid, block, 0, st, a);
+    else if (rgb3 && d->cout <= 16)
+      e = g.pool == 2 ? launch_k(conv_direct_rgb3_kernel<16, 2>, grid, block, 0, st, a)
+                      : launch_k(conv_direct_rgb3_kernel<16, 1>, grid, block, 0, st, a);
     else if (d->cout <= 8) e = launch_k(conv_direct_kernel<4>, grid, block, 0, st, a);
     else if (d->cout <= 16) e = launch_k(conv_direct_kernel<8>, grid, block, 0, st, a);
     else e = launch_k(conv_direct_kernel<16>, grid, block, 0, st, a);
