@@ -473,7 +473,8 @@ def run_ours(args):
                                     "avg_launch_us": 1e3 * conv_ms / len(conv_idx),
                                     "timing": f"each launch alone between CUDA events ({timing_mode})"}},
         "e2e": {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+                "sequence": "per step: L2 flush (untimed), input copy, step, result copy, one stream"},
         "pool_hbm": pool_hbm,
         "gpu_launches": K * n_kernels,
         "clocks": clocks,
