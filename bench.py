@@ -41,7 +41,7 @@ UNIT = "TOPS"
 INT8_PEAK_TOPS = 151.4
 FP8_PER_BF16 = 2.0          # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK_BF16_TFLOPS = 1900.0
-PROFILE = os.path.join(ROOT, "profiles", "conv_tc_resnet18_b32.md")
+PROFILES = os.path.join(ROOT, "profiles")
 KERNEL_SRC = [os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", f) for f in ("conv_tc.cuh", "conv_common.cuh", "ptx.cuh")]
 
 
@@ -92,17 +92,21 @@ def kernel_sha():
     return h.hexdigest()[:16]
 
 
-def profiled_traffic():
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on this kernel source."""
-    try:
-        txt = open(PROFILE).read()
-    except OSError:
-        return None
-    sha = re.search(r"kernel_sha:\s*([0-9a-f]+)", txt)
-    tb = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt)
-    if not sha or not tb or sha.group(1) != kernel_sha():
-        return None
-    return float(tb.group(1))
+def profiled_traffic(workload: str):
+    """DRAM bytes per conv launch from the committed ncu summary of this workload, if it was taken
+    on this kernel source (a summary names its `workload:` and `kernel_sha:`)."""
+    import glob
+    for path in sorted(glob.glob(os.path.join(PROFILES, "conv_tc_*.md"))):
+        try:
+            txt = open(path).read()
+        except OSError:
+            continue
+        wl = re.search(r"^workload:\s*(\S+)", txt, re.M)
+        sha = re.search(r"^kernel_sha:\s*([0-9a-f]+)", txt, re.M)
+        tb = re.search(r"^traffic_bytes_per_launch:\s*([0-9.eE+]+)", txt, re.M)
+        if wl and sha and tb and wl.group(1) == workload and sha.group(1) == kernel_sha():
+            return float(tb.group(1))
+    return None
 
 
 class ClockSampler:
@@ -277,7 +281,7 @@ def measure_pool_hbm(ifq, torch, dev, stream, flush, reps=20):
     _, _, hbm, src = read_peaks()
     gbs = bytes_moved / (us * 1e-6) / 1e9
     del x, y
-    return {"kernel": "maxpool_codes_kernel", "shape": f"2x2/2 pool, {n}x{h}x{w}x{c} 2-bit codes",
+    return {"kernel": "maxpool2x2_rowpair_kernel", "shape": f"2x2/2 pool, {n}x{h}x{w}x{c} 2-bit codes",
             "algorithmic_bytes": bytes_moved, "us": us, "achieved_gbs": gbs, "peak_gbs": hbm,
             "frac": gbs / hbm, "peak_source": f"{src} STREAM copy",
             "l2": "not flushed: input (177 MB) larger than L2 (129 MB)"}
@@ -449,7 +453,7 @@ def run_ours(args):
     conv_in_step_ms = step_ms * conv_share
     achieved = conv_ops_total / (conv_in_step_ms * 1e-3) / 1e12
     achieved_serial = conv_ops_total / (conv_ms * 1e-3) / 1e12
-    traffic = profiled_traffic()
+    traffic = profiled_traffic(wl.name)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
         "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,

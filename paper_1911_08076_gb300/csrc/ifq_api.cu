@@ -539,6 +539,21 @@ int run_pool(const ifq_pool_desc* d, const void* x, const int8_t* sign, void* y,
   a.div_groups = make_fastdiv((uint32_t)a.groups);
   a.div_wo = make_fastdiv((uint32_t)wo);
   a.div_ho = make_fastdiv((uint32_t)ho);
+  // 2x2 / stride 2 without padding on 4- or 8-byte pixels: whole 16-byte row segments per item
+  const int kp = pb == 4 ? 2 : 1;
+  if (d->k == 2 && d->stride == 2 && d->pad == 0 && (pb == 4 || pb == 8) && ((size_t)d->w * pb) % 16 == 0 &&
+      wo % kp == 0) {
+    a.wq = wo / kp;
+    a.div_wq = make_fastdiv((uint32_t)a.wq);
+    a.total = (int)((size_t)d->n * ho * a.wq);
+    const dim3 grid(launch_1d_blocks((size_t)a.total, 256, nsm));
+    cudaError_t e;
+    if (sb == 2) e = pb == 4 ? launch_k(maxpool2x2_rowpair_kernel<2, 4>, grid, dim3(256), 0, st, a)
+                             : launch_k(maxpool2x2_rowpair_kernel<2, 8>, grid, dim3(256), 0, st, a);
+    else e = pb == 4 ? launch_k(maxpool2x2_rowpair_kernel<4, 4>, grid, dim3(256), 0, st, a)
+                     : launch_k(maxpool2x2_rowpair_kernel<4, 8>, grid, dim3(256), 0, st, a);
+    return e == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+  }
   const dim3 b256(256), grid(launch_1d_blocks((size_t)a.total, 256, nsm));
   cudaError_t e;
   if (vb >= 4)

@@ -49,6 +49,8 @@ struct PoolArgs {
   int groups;                          // vector groups (of U words or of single bytes) per pixel
   int total;                           // n * ho * wo * groups (< 2^31)
   FastDiv div_groups, div_wo, div_ho;
+  int wq;                              // 2x2 row-pair kernel: items per output row
+  FastDiv div_wq;
 };
 
 template <int U>
@@ -147,6 +149,64 @@ __global__ void __launch_bounds__(256) maxpool_codes_kernel(const PoolArgs a) {
 #pragma unroll
     for (int u = 0; u < U; ++u) m[u] ^= mask[u];
     WordVec<U>::st(dst, m);
+  }
+}
+
+// 2x2 / stride 2 pool without padding on narrow pixels of PB = 4 or 8 packed bytes.  An item is
+// the 16 contiguous bytes of input row 2*oy under P = 16 / (2 PB) adjacent output pixels (2 P input
+// pixels) and the same 16 bytes of row 2*oy + 1: two 128-bit loads and one 64-bit store, where the
+// general kernel issues a 4- or 8-byte load per window cell.  Each thread takes two items per
+// round (four loads in flight); the loads are streaming (evict-first: each input byte is read once).
+// Needs w * PB % 16 == 0 and wo % P == 0 (checked by the host); every cell is inside the image
+// because ho = h / 2 and wo = w / 2 (floor).
+template <int SB, int PB>
+__global__ void __launch_bounds__(256) maxpool2x2_rowpair_kernel(const PoolArgs a) {
+  grid_dep_launch();
+  grid_dep_wait();
+  constexpr int kCpw = 32 / SB;             // codes per word
+  constexpr int kP = 16 / (2 * PB);         // output pixels per item
+  static_assert(PB == 4 || PB == 8, "pixel bytes");
+  // flip masks of the pixel's words (one word for PB = 4, two for PB = 8)
+  const uint32_t m0 = flip_mask<SB, kCpw>(a.sign, 0, a.c);
+  const uint32_t m1 = PB == 8 ? flip_mask<SB, kCpw>(a.sign, kCpw, a.c) : m0;
+  const size_t rowb = (size_t)a.w * PB;
+  // item it: output row t = (b, oy), segment q; returns the first input byte of the segment
+  auto src = [&](int it, int& t, int& q) {
+    t = (int)fdiv((uint32_t)it, a.div_wq);
+    q = it - t * a.wq;
+    const int b = (int)fdiv((uint32_t)t, a.div_ho);
+    const int oy = t - b * a.ho;
+    return a.x + ((size_t)b * a.h + 2 * oy) * rowb + (size_t)q * 16;
+  };
+  auto max4 = [](uint32_t p, uint32_t q, uint32_t r, uint32_t u, uint32_t m) {
+    return field_max<SB>(field_max<SB>(p ^ m, q ^ m), field_max<SB>(r ^ m, u ^ m)) ^ m;
+  };
+  auto reduce_store = [&](const uint4& r0, const uint4& r1, int t, int q) {
+    uint2 o;
+    if constexpr (PB == 8) {   // input pixels (x, y) and (z, w) -> one output pixel of two words
+      o.x = max4(r0.x, r0.z, r1.x, r1.z, m0);
+      o.y = max4(r0.y, r0.w, r1.y, r1.w, m1);
+    } else {                   // input pixels x, y -> output pixel 2q; z, w -> 2q + 1
+      o.x = max4(r0.x, r0.y, r1.x, r1.y, m0);
+      o.y = max4(r0.z, r0.w, r1.z, r1.w, m0);
+    }
+    *(uint2*)(a.y + ((size_t)t * a.wo + (size_t)q * kP) * PB) = o;
+  };
+  const int gs = gridDim.x * blockDim.x;
+  int it = blockIdx.x * blockDim.x + threadIdx.x;
+  for (; it + gs < a.total; it += 2 * gs) {   // items it and it + gs
+    int t0, q0, t1, q1;
+    const uint8_t* p0 = src(it, t0, q0);
+    const uint8_t* p1 = src(it + gs, t1, q1);
+    const uint4 a0 = __ldcs((const uint4*)p0), b0 = __ldcs((const uint4*)(p0 + rowb));
+    const uint4 a1 = __ldcs((const uint4*)p1), b1 = __ldcs((const uint4*)(p1 + rowb));
+    reduce_store(a0, b0, t0, q0);
+    reduce_store(a1, b1, t1, q1);
+  }
+  if (it < a.total) {
+    int t, q;
+    const uint8_t* p = src(it, t, q);
+    reduce_store(__ldcs((const uint4*)p), __ldcs((const uint4*)(p + rowb)), t, q);
   }
 }
 

@@ -146,6 +146,9 @@ KPOOL_CASES = [
     (1, 13, 13, 512, 2, 1, 1, True),
     (2, 9, 9, 16, 2, 2, 0, False),
     (1, 7, 5, 12, 3, 2, 1, True),          # 6-byte pixels: bytes
+    (2, 8, 12, 8, 2, 2, 0, True),          # 4-byte pixels, 2x2 / 2: the row-pair kernel
+    (1, 10, 14, 16, 2, 2, 0, True),        # 8-byte pixels, 2x2 / 2: the row-pair kernel
+    (1, 9, 14, 8, 2, 2, 0, True),          # 4-byte pixels, rows of 56 bytes: the general kernel
 ]
 
 

@@ -204,6 +204,14 @@ POOL_CASES = [
     (1, 7, 7, 8, 2, 2, 0, True),
     (1, 7, 5, 4, 3, 2, 1, True),
     (3, 208, 208, 32, 2, 2, 0, True),
+    # 2x2 / stride 2 on 4- and 8-byte pixels: the row-pair kernel (16-byte row segments) ...
+    (2, 16, 16, 16, 2, 2, 0, True),
+    (1, 12, 20, 16, 2, 2, 0, True),
+    (2, 11, 14, 32, 2, 2, 0, True),             # odd height: the last input row is unused
+    (1, 9, 6, 32, 2, 2, 0, False),
+    # ... and the general kernel where a row is not a whole number of 16-byte segments
+    (2, 6, 10, 16, 2, 2, 0, True),
+    (1, 8, 7, 32, 2, 2, 0, True),
 ]
 
 

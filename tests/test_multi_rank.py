@@ -64,3 +64,18 @@ def test_reference_arm_under_torchrun_two_ranks():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_profiled_traffic_is_keyed_by_workload_and_kernel_source(tmp_path, monkeypatch):
+    """bench.py reports an ncu DRAM-traffic figure only from a summary taken on the same workload
+    and on the kernel source as it stands (a stale or foreign figure is null)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    sha = bench.kernel_sha()
+    (tmp_path / "conv_tc_a.md").write_text(f"# a\n\nworkload: wl_a\nkernel_sha: {sha}\ntraffic_bytes_per_launch: 123\n")
+    (tmp_path / "conv_tc_b.md").write_text("# b\n\nworkload: wl_b\nkernel_sha: 0000000000000000\n"
+                                           "traffic_bytes_per_launch: 456\n")
+    monkeypatch.setattr(bench, "PROFILES", str(tmp_path))
+    assert bench.profiled_traffic("wl_a") == 123.0
+    assert bench.profiled_traffic("wl_b") is None        # taken on another kernel source
+    assert bench.profiled_traffic("wl_c") is None        # no summary for this workload
