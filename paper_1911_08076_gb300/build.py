@@ -8,6 +8,7 @@ paper_1911_08076_gb300/_build/libifq.so.
 from __future__ import annotations
 
 import os
+import re
 import shutil
 import subprocess
 import sys
@@ -41,6 +42,25 @@ def _stale() -> bool:
     return any(os.path.getmtime(s) > t for s in _sources())
 
 
+# The warp-specialised tensor-core kernels run at the 72-register cap of 864 threads per CTA; every
+# instance must fit it without spilling to local memory (a build with spills is refused).
+_GUARDED = ("conv_tc_kernel", "conv_stack_kernel")
+
+
+def spilling_kernels(ptxas_log: str):
+    """Entry points of the guarded kernels whose ptxas report shows spill stores or loads."""
+    bad, cur = [], None
+    for line in ptxas_log.splitlines():
+        m = re.search(r"Compiling entry function '([^']+)'", line)
+        if m:
+            cur = m.group(1)
+            continue
+        m = re.search(r"(\d+) bytes spill stores, (\d+) bytes spill loads", line)
+        if m and cur and any(g in cur for g in _GUARDED) and (int(m.group(1)) or int(m.group(2))):
+            bad.append(cur)
+    return bad
+
+
 def build(force: bool = False, verbose: bool = False) -> str:
     if not force and not _stale():
         return LIB
@@ -51,7 +71,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     o_cpp = os.path.join(OUT, f"ifq_host.{tag}.o")
     cmds = [
         [nvcc, *ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
-         "-Xptxas", "-v" if verbose else "-O3", "-c", os.path.join(CSRC, "ifq_api.cu"), "-o", o_cu],
+         "-Xptxas", "-v", "-c", os.path.join(CSRC, "ifq_api.cu"), "-o", o_cu],
         ["g++", "-O2", "-std=c++17", "-fPIC", "-ffp-contract=off", "-fno-fast-math", "-I", INCLUDE, "-c",
          os.path.join(CSRC, "ifq_host.cpp"), "-o", o_cpp],
     ]
@@ -64,6 +84,9 @@ def build(force: bool = False, verbose: bool = False) -> str:
 
     with ThreadPoolExecutor(2) as ex:
         logs = list(ex.map(run, cmds))
+    spilled = spilling_kernels(logs[0])
+    if spilled:
+        raise RuntimeError("tensor-core kernels spill registers to local memory: " + ", ".join(spilled))
     tmp = LIB + f".{tag}.tmp"
     cudalib = os.path.join(os.path.dirname(os.path.dirname(nvcc)), "lib64")
     run([nvcc, *ARCH, "-shared", "-cudart", "shared", o_cu, o_cpp, "-Xlinker", f"-rpath={cudalib}", "-o", tmp])

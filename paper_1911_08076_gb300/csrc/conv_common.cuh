@@ -58,15 +58,21 @@ constexpr int kAhead = 2;        // own K stages of packed codes a gather thread
 // SB: bits per stored code (2, or 4 for 3- and 4-bit codes).  Thresholds per column: a float4
 // (3 thresholds and the sign) for SB = 2, five float4 (15 thresholds, padded with +inf, in the
 // order of the 4-ary search, and the sign) for SB = 4.
-template <int BN, int SB = 2>
+// KS > 1 (split K over a cluster of KS CTAs): KS - 1 receive slots of fp32 partial sums, one per
+// partner, each 128 rows x BN / KS columns (rows padded by 16 bytes), and two more barriers.
+template <int BN, int SB = 2, int KS = 1>
 struct TcSmem {
   static constexpr int kB = BN * kBK;
   static constexpr int kThrCol = SB == 2 ? 16 : 80;       // bytes of thresholds per column
+  static constexpr int kRecvRow = BN / KS + 4;             // floats per row of a receive slot
+  static constexpr int kRecvSlot = kBM * kRecvRow * 4;     // bytes of a receive slot
   static constexpr int offB = 0;
   static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN columns
   static constexpr int offTab = offThr + 2 * BN * kThrCol; // kMaxTab x int2
-  static constexpr int offBar = offTab + kMaxTab * 8;
-  static constexpr int nBar = 2 * kStages + 5;             // full, empty, acc_full[2], acc_empty[2], done
+  static constexpr int offRecv = offTab + kMaxTab * 8;
+  static constexpr int offBar = offRecv + (KS - 1) * kRecvSlot;
+  // full, empty, acc_full[2], acc_empty[2], done (+ recv_full, send_ok)
+  static constexpr int nBar = 2 * kStages + 5 + (KS > 1 ? 2 : 0);
   static constexpr int offTmem = offBar + nBar * 8;
   static constexpr int bytes = offTmem + 16 + 1024;        // + alignment slack
 };
@@ -173,41 +179,61 @@ __device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, in
   return v;
 }
 
-// 64 packed codes -> 16 tensor-memory columns of e4m3 bytes (column 4j+q holds
-// byte t = code 4t + q of the 16 codes in word j).
-__device__ __forceinline__ void expand_tmem_store(uint32_t taddr, uint4 v) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  uint32_t o[16];
-#pragma unroll
-  for (int j = 0; j < 4; ++j)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+// 16 columns of zeros into tensor memory (this warp's 32 lanes), with the wait for the store.
+__device__ __forceinline__ void tmem_zero16_sync(uint32_t taddr) {
   asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+      "r"(0u)
+      : "memory");
+}
+
+// 32 lanes x 16 consecutive columns of 32-bit tensor memory -> 16 registers per thread.  The load
+// writes its destination registers asynchronously; the wait is in the same asm statement, so the
+// compiler never sees the registers before they hold the data.
+__device__ __forceinline__ void tmem_ld16_sync(uint32_t taddr, uint32_t (&v)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+      : "r"(taddr)
+      : "memory");
+}
+
+// 16 registers -> 16 consecutive tensor-memory columns of this warp's 32 lanes, and the wait for
+// the store in the same asm statement, so the compiler cannot reuse the source registers while the
+// asynchronous store may still read them.
+__device__ __forceinline__ void tmem_st16_sync(uint32_t taddr, const uint32_t* o) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
       "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
       "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
       : "memory");
 }
 
-// 64 four-bit codes (two 16-byte units, 8 words) -> 16 tensor-memory columns of e4m3 bytes:
-// word j of the 8 contributes column 2j (its codes 0, 2, 4, 6 as bytes 0..3) and column
-// 2j+1 (codes 1, 3, 5, 7).  A code c in 0..15 is the e4m3 byte c, the value c * 2^-9 (0..7
-// subnormal, 8..15 with exponent field 1).
-__device__ __forceinline__ void expand4_tmem_store(uint32_t taddr, uint4 a, uint4 b) {
+// 64 packed two-bit codes -> 16 registers of e4m3 bytes (register 4j+q holds byte t = code 4t + q
+// of the 16 codes in word j).
+__device__ __forceinline__ void expand2(uint4 v, uint32_t* o) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+}
+
+// 64 four-bit codes (two 16-byte units, 8 words) -> 16 registers of e4m3 bytes: word j of the 8
+// gives register 2j (its codes 0, 2, 4, 6 as bytes 0..3) and register 2j+1 (codes 1, 3, 5, 7).
+// A code c in 0..15 is the e4m3 byte c, the value c * 2^-9 (0..7 subnormal, 8..15 with exponent
+// field 1).
+__device__ __forceinline__ void expand4(uint4 a, uint4 b, uint32_t* o) {
   const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-  uint32_t o[16];
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     o[2 * j] = w[j] & 0x0F0F0F0Fu;
     o[2 * j + 1] = (w[j] >> 4) & 0x0F0F0F0Fu;
   }
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
-      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7]), "r"(o[8]), "r"(o[9]),
-      "r"(o[10]), "r"(o[11]), "r"(o[12]), "r"(o[13]), "r"(o[14]), "r"(o[15])
-      : "memory");
 }
 
 }  // namespace ifq

@@ -54,15 +54,6 @@ namespace ifq {
 constexpr int kWarpMma2 = kWarpEpi0 + kEpiWarps;
 constexpr int kConvThreads = kTcThreads + 32;
 
-// 16 columns of zeros into tensor memory (this warp's 32 lanes).
-__device__ __forceinline__ void tmem_zero16(uint32_t taddr) {
-  const uint32_t z = 0u;
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1,%1};" ::"r"(taddr),
-      "r"(z)
-      : "memory");
-}
-
 // The code of one accumulator against 15 ascending thresholds t[0..14] (+inf past 2^k - 1):
 // #{ i : sign*D > t[i] } as a 4-ary search over five float4 per column,
 //   t5[0] = {t3, t7, t11, sign},  t5[1+q] = {t(4q), t(4q+1), t(4q+2), -}  (q = 0..3):
@@ -80,12 +71,24 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
 // GB: bytes per gathered granule: 16, 4 or 1 (the largest that divides the packed bytes of a
 // pixel); SB: bits per stored input code (2 for k = 2, 4 for k = 3 and 4 and for the two nibbles of
 // an 8-bit input value); SBO: bits per stored output code (2 or 4).
-template <int BN, int GB, int SB, int SBO>
+//
+// KS > 1: split K.  The grid is made of clusters of KS CTAs; cluster c takes tiles c, c + C, ...
+// (C clusters) and CTA r of it the K stages [r nk / KS, (r+1) nk / KS) of each, into its own
+// accumulator.  Column block r of the tile (BN / KS columns) belongs to CTA r: in the epilogue every
+// CTA sends the other blocks of its partial sum to their owners' receive slots (distributed shared
+// memory), waits for the partners' partials of its own block, adds them and thresholds that block.
+// The partial sums are exact integers (multiples of 2^-9 far inside the fp32 significand), so their
+// order does not matter.  A receive slot is reused for the next tile once its owner has read it
+// (send_ok); clusters synchronise once after setup and once before exit, so no CTA's shared memory
+// goes away while a partner may still write it.
+template <int BN, int GB, int SB, int SBO, int KS = 1>
 __global__ void __launch_bounds__(kConvThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
   static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
   static_assert((SB == 2 || SB == 4) && (SBO == 2 || SBO == 4), "stored code width");
-  using L = TcSmem<BN, SBO>;
+  static_assert(KS == 1 || KS == 2 || KS == 4, "K split");
+  static_assert(BN / KS / 2 >= 16, "an epilogue thread takes at least 16 columns of a block");
+  using L = TcSmem<BN, SBO, KS>;
   constexpr int kU = kBK * SB / 8 / 16;       // 16-byte units of packed codes per K stage
   constexpr int kCpb = 8 / SB;                // codes per byte
   constexpr int kS = kStages;
@@ -103,13 +106,22 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   auto acc_full = [&](int b) { return barBase + 8u * (2 * kS + b); };
   auto acc_empty = [&](int b) { return barBase + 8u * (2 * kS + 2 + b); };
   const uint32_t done_bar = barBase + 8u * (2 * kS + 4);
+  // KS > 1: recv_full completes when every partner has stored its partial of this CTA's column
+  // block; send_ok when every partner has read the partial this CTA stored in its slot
+  const uint32_t recv_full = barBase + 8u * (2 * kS + 5);
+  const uint32_t send_ok = barBase + 8u * (2 * kS + 6);
   uint32_t* tmem_slot = (uint32_t*)(smem + L::offTmem);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   constexpr uint32_t kCols = 512;
-  const int G = gridDim.x;
-  const int n_local = (args.ntiles - (int)blockIdx.x + G - 1) / G;
-  const int nk = args.nk;
+  // tile schedule: cluster cid of G takes tiles cid, cid + G, ... (a cluster is one CTA for KS = 1)
+  const uint32_t crank = KS > 1 ? cluster_ctarank() : 0u;
+  const int cid = KS > 1 ? (int)cluster_id_x() : (int)blockIdx.x;
+  const int G = KS > 1 ? (int)nclusters_x() : (int)gridDim.x;
+  const int n_local = (args.ntiles - cid + G - 1) / G;
+  // this CTA's K stages of every tile: [kb, kb + nk)
+  const int kb = (int)((crank * (uint32_t)args.nk) / KS);
+  const int nk = (int)(((crank + 1u) * (uint32_t)args.nk) / KS) - kb;
 
   // ---- setup (reads no global memory, so it may overlap the previous grid)
   if (warp == kWarpMma) {
@@ -126,6 +138,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       mbar_init(acc_empty(b), kEpiWarps);  // drained and zeroed by every epilogue warp
     }
     mbar_init(done_bar, 2);
+    if constexpr (KS > 1) {
+      mbar_init(recv_full, (KS - 1) * kEpiWarps * 32);   // every epilogue thread of every partner
+      mbar_init(send_ok, (KS - 1) * kEpiWarps * 32);
+    }
     fence_mbar_init();
   }
   if (warp == kWarpTma && lane == 0) prefetch_tmap(&tmap_w);
@@ -146,6 +162,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
+  // the partners' barriers are initialised before any CTA of the cluster reaches them
+  if constexpr (KS > 1) cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   grid_dep_launch();
@@ -161,17 +179,17 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     // load cursor over this group's stages it = group + 4*j: tile l_tile, K stage l_k
     int l_tile = 0, l_k = group;
     while (l_k >= nk) { l_k -= nk; ++l_tile; }
-    RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r
+    RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)(cid + l_tile * G), args.div_nt) * kBM + r
                                                 : args.M);
     // packed codes of kAh of this group's stages in registers (16 registers either way)
     constexpr int kAh = SB == 2 ? kAhead : 1;
     auto next_load = [&](uint4 (&u)[kU]) {
 #pragma unroll
-      for (int q = 0; q < kU; ++q) u[q] = load_unit<GB>(sTab, g, l_k * kU + q);
+      for (int q = 0; q < kU; ++q) u[q] = load_unit<GB>(sTab, g, (kb + l_k) * kU + q);
       l_k += kGatherGroups;
       if (l_k >= nk) {
         do { l_k -= nk; ++l_tile; } while (l_k >= nk);
-        if (l_tile < n_local) g = row_geom(args, (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), args.div_nt) * kBM + r);
+        if (l_tile < n_local) g = row_geom(args, (int)fdiv((uint32_t)(cid + l_tile * G), args.div_nt) * kBM + r);
       }
     };
     uint4 ring[kAh][kU];
@@ -197,14 +215,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           const uint32_t ph = (uint32_t)(it / kS) & 1u;
           if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
           tc_fence_after();
-          if constexpr (SB == 2) {
-            expand_tmem_store(tA + (uint32_t)(s * 32), cur[0]);
-            expand_tmem_store(tA + (uint32_t)(s * 32 + 16), cur[kU - 1]);
-          } else {
-            expand4_tmem_store(tA + (uint32_t)(s * 32), cur[0], cur[1]);
-            expand4_tmem_store(tA + (uint32_t)(s * 32 + 16), cur[kU - 2], cur[kU - 1]);
-          }
-          asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+          uint32_t o[16];
+          if constexpr (SB == 2) expand2(cur[0], o);
+          else expand4(cur[0], cur[1], o);
+          tmem_st16_sync(tA + (uint32_t)(s * 32), o);
+          if constexpr (SB == 2) expand2(cur[kU - 1], o);
+          else expand4(cur[kU - 2], cur[kU - 1], o);
+          tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(full(s));
@@ -218,7 +235,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     bool ok = true;
 #pragma unroll 1
     for (int jt = 0; jt < n_local && ok; ++jt) {
-      const int t = (int)blockIdx.x + jt * G;
+      const int t = cid + jt * G;
       const int n0 = (t - (int)fdiv((uint32_t)t, args.div_nt) * args.nt) * BN;
 #pragma unroll 1
       for (int k = 0; k < nk; ++k, ++it) {
@@ -227,7 +244,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
         if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
         if (elect_one()) {
           mbar_arrive_expect_tx(full(s), (uint32_t)L::kB);
-          tma_load_2d(sB + (uint32_t)(s * L::kB), &tmap_w, full(s), k * kBK, n0);
+          tma_load_2d(sB + (uint32_t)(s * L::kB), &tmap_w, full(s), (kb + k) * kBK, n0);
         }
         __syncwarp();
       }
@@ -293,22 +310,26 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     __syncwarp();
   } else {
     // =================== epilogue ===================
-    // warp pair e, e+4 covers lane quarter (warp % 4), column halves 0 and 1
-    constexpr int CW = BN / 2;                  // columns per thread
+    // warp pair e, e+4 covers lane quarter (warp % 4), halves 0 and 1 of every column block (the
+    // whole tile for KS = 1; with KS > 1 the block of CTA r is columns [r BN/KS, (r+1) BN/KS))
+    constexpr int CB = BN / KS;                 // columns of a block
+    constexpr int CW = CB / 2;                  // columns per thread in a block
     const int e = warp - kWarpEpi0;             // 0..7
     const int et = tid - kWarpEpi0 * 32;        // 0..255
     const int quarter = warp & 3;
-    const int c_lo = (e >> 2) * CW;
+    const int c_in = (e >> 2) * CW;             // this thread's first column within a block
+    const int c_lo = (int)crank * CB + c_in;    // ... within this CTA's own block
     const int row = quarter * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     bool ok = true;   // after a timed-out wait, keep only the named barriers (uniform over the 8 warps)
     // both accumulator buffers start at zero: every MMA accumulates
     {
-      const uint32_t tz = tmem + (uint32_t)c_lo + ((uint32_t)(quarter * 32) << 16);
 #pragma unroll
       for (int b2 = 0; b2 < 2; ++b2)
 #pragma unroll
-        for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16(tz + (uint32_t)(b2 * BN + c0));
-      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        for (int p = 0; p < KS; ++p)
+#pragma unroll
+          for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16_sync(tmem + lane_off + (uint32_t)(b2 * BN + p * CB + c_in + c0));
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -318,7 +339,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
 #pragma unroll 1
     for (int jt = 0; jt < n_local; ++jt) {
-      const int t = (int)blockIdx.x + jt * G;
+      const int t = cid + jt * G;
       const int mt = (int)fdiv((uint32_t)t, args.div_nt);
       const int n0 = (t - mt * args.nt) * BN;
       const int m = mt * kBM + row;
@@ -350,20 +371,56 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait_backoff(acc_full(ab), (uint32_t)(jt >> 1) & 1u, 64));
       if (!ok) continue;
       tc_fence_after();
-      const uint32_t tacc = tmem + (uint32_t)(ab * BN + c_lo) + ((uint32_t)(quarter * 32) << 16);
+      const uint32_t tbuf = tmem + (uint32_t)(ab * BN) + lane_off;   // this row of accumulator buffer ab
+      const uint32_t tacc = tbuf + (uint32_t)c_lo;
+      if constexpr (KS > 1) {
+        // send the partners' blocks of this partial sum to their receive slots (slot s of CTA p
+        // holds the partial of the s-th other CTA in rank order), once p has read the last tile's
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait_cluster(send_ok, ((uint32_t)jt & 1u) ^ 1u));
+        if (ok) {
+#pragma unroll 1
+          for (int pp = 1; pp < KS; ++pp) {
+            const uint32_t p = (crank + (uint32_t)pp) % KS;
+            const uint32_t slot = crank < p ? crank : crank - 1u;
+            const uint32_t dst = mapa_shared(
+                sbase + (uint32_t)L::offRecv + slot * (uint32_t)L::kRecvSlot + (uint32_t)(row * L::kRecvRow + c_in) * 4u, p);
+#pragma unroll
+            for (int c0 = 0; c0 < CW; c0 += 16) {
+              uint32_t v[16];
+              tmem_ld16_sync(tbuf + (uint32_t)(p * CB + c_in + c0), v);
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                st_cluster_v4(dst + (uint32_t)(c0 + 4 * q) * 4u, v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            }
+          }
+#pragma unroll 1
+          for (int pp = 1; pp < KS; ++pp) mbar_arrive_remote(mapa_shared(recv_full, (crank + (uint32_t)pp) % KS));
+          ok = __all_sync(0xffffffffu, mbar_wait_cluster(recv_full, (uint32_t)jt & 1u));
+        }
+        if (!ok) continue;
+      }
       const float4* th = sThr + (size_t)(tb * BN + c_lo) * (SBO == 2 ? 1 : 5);
       constexpr int kPW = CW * SBO / 32;          // 32-bit words of packed codes per thread
       uint32_t packed[kPW];
 #pragma unroll
       for (int c0 = 0; c0 < CW; c0 += 16) {
         uint32_t v[16];
-        asm volatile(
-            "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-            : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-              "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
-            : "r"(tacc + c0)
-            : "memory");
-        tmem_ld_wait();
+        tmem_ld16_sync(tacc + c0, v);
+        if constexpr (KS > 1) {   // + the partners' partial sums of these 16 columns
+#pragma unroll
+          for (int sl = 0; sl < KS - 1; ++sl) {
+            const float4* src =
+                (const float4*)(smem + L::offRecv + (size_t)sl * L::kRecvSlot) + (row * L::kRecvRow + c_in + c0) / 4;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const float4 f = src[q];
+              v[4 * q] = __float_as_uint(__uint_as_float(v[4 * q]) + f.x);
+              v[4 * q + 1] = __float_as_uint(__uint_as_float(v[4 * q + 1]) + f.y);
+              v[4 * q + 2] = __float_as_uint(__uint_as_float(v[4 * q + 2]) + f.z);
+              v[4 * q + 3] = __float_as_uint(__uint_as_float(v[4 * q + 3]) + f.w);
+            }
+          }
+        }
         // Fused pool (Sec. 2.1: the pool acts on Y^conv, before BN and the quantizer): the window
         // maximum of A over the window's consecutive lanes, then the thresholds.
         if (args.lpool == 1) {
@@ -445,10 +502,16 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           }
         }
       }
+      // the partners may store the next tile's partials into this CTA's slots
+      if constexpr (KS > 1) {
+#pragma unroll 1
+        for (int pp = 1; pp < KS; ++pp) mbar_arrive_remote(mapa_shared(send_ok, (crank + (uint32_t)pp) % KS));
+      }
       // the accumulator buffer may be refilled once every epilogue warp has read and zeroed it
 #pragma unroll
-      for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16(tacc + c0);
-      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      for (int p = 0; p < KS; ++p)
+#pragma unroll
+        for (int c0 = 0; c0 < CW; c0 += 16) tmem_zero16_sync(tbuf + (uint32_t)(p * CB + c_in + c0));
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty(ab));
@@ -481,6 +544,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   // ---- teardown: every MMA has completed (done_bar) before TMEM is released
   tc_fence_before();
   __syncthreads();
+  // no CTA leaves while a partner may still store into its receive slots or arrive on its barriers
+  if constexpr (KS > 1) cluster_sync_all();
   if (warp == kWarpMma) {
     tc_fence_after();
     mbar_wait(done_bar, 0);

@@ -84,29 +84,87 @@ cudaError_t launch_k(void (*kern)(Exp...), dim3 grid, dim3 block, size_t smem, c
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
 }
 
-template <int BN, int GB, int SB, int SBO>
+// A launch in clusters of `cluster` CTAs along x (grid.x a multiple of it), with programmatic
+// dependent launch as in launch_k.
+template <typename... Exp, typename... Act>
+cudaError_t launch_k_cluster(void (*kern)(Exp...), int cluster, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                             Act&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = (unsigned)cluster;
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Act>(args)...);
+}
+
+// One instance of the tensor-core kernel.  KS > 1 (split K over clusters of KS CTAs): the grid is
+// as many clusters as can be resident at once (cudaOccupancyMaxActiveClusters), at most one per
+// tile.
+template <int BN, int GB, int SB, int SBO, int KS = 1>
 struct TcInst {
-  using L = TcSmem<BN, SBO>;
+  using L = TcSmem<BN, SBO, KS>;
   static_assert(L::bytes <= 232448, "shared memory budget");
+  static constexpr auto kern = conv_tc_kernel<BN, GB, SB, SBO, KS>;
   static cudaError_t set_attr() {
-    return cudaFuncSetAttribute(conv_tc_kernel<BN, GB, SB, SBO>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                L::bytes);
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
+  }
+  // clusters of this instance that fit on the device at once (0: none)
+  static int max_clusters(int nsm) {
+    static int cached = -1;
+    if (cached < 0) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3((unsigned)(nsm / KS * KS));
+      cfg.blockDim = dim3(kConvThreads);
+      cfg.dynamicSmemBytes = L::bytes;
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = KS;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      int n = 0;
+      cached = cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess ? n : 0;
+      cudaGetLastError();
+    }
+    return cached;
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
-    const int grid = a.ntiles < nsm ? a.ntiles : nsm;
-    return launch_k(conv_tc_kernel<BN, GB, SB, SBO>, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
+    if constexpr (KS == 1) {
+      const int grid = a.ntiles < nsm ? a.ntiles : nsm;
+      return launch_k(kern, dim3(grid), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
+    } else {
+      const int mc = max_clusters(nsm);
+      if (mc < 1) return cudaErrorInvalidConfiguration;
+      const int nc = a.ntiles < mc ? a.ntiles : mc;
+      return launch_k_cluster(kern, KS, dim3(nc * KS), dim3(kConvThreads), (size_t)L::bytes, st, tm, a);
+    }
   }
 };
 
-// The output-channel tile widths of the tensor-core kernel.
-#define IFQ_TC_VARIANTS(X, GB, SB, SBO) X(128, GB, SB, SBO) X(64, GB, SB, SBO) X(32, GB, SB, SBO)
+// The (output-channel tile width, K split) instances of the tensor-core kernel; the split ones
+// exist for 16-byte granules (every layer with 64 or more 2-bit, or 32 or more 4-bit, channels).
+#define IFQ_TC_VARIANTS(X, GB, SB, SBO) X(128, GB, SB, SBO, 1) X(64, GB, SB, SBO, 1) X(32, GB, SB, SBO, 1)
+#define IFQ_TC_SPLIT_VARIANTS(X, GB, SB, SBO) X(64, GB, SB, SBO, 2)
 
 template <int GB, int SB, int SBO>
 cudaError_t set_attrs_gb() {
   cudaError_t e = cudaSuccess;
-#define IFQ_SET(BN, G, S, SO) \
-  if (e == cudaSuccess) e = TcInst<BN, G, S, SO>::set_attr();
+#define IFQ_SET(BN, G, S, SO, KS) \
+  if (e == cudaSuccess) e = TcInst<BN, G, S, SO, KS>::set_attr();
   IFQ_TC_VARIANTS(IFQ_SET, GB, SB, SBO)
+  if constexpr (GB == 16) {
+    IFQ_TC_SPLIT_VARIANTS(IFQ_SET, GB, SB, SBO)
+  }
 #undef IFQ_SET
   return e;
 }
@@ -311,10 +369,49 @@ int choose_bn(const ConvGeom& g, int cout, int nsm) {
 }
 
 template <int GB, int SB, int SBO>
-cudaError_t launch_tc_gb(int bn, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
-#define IFQ_LAUNCH(BN, G, S, SO) \
-  if (bn == BN) return TcInst<BN, G, S, SO>::launch(tm, a, nsm, st);
+int tc_max_clusters(int bn, int ks, int nsm) {
+  if constexpr (GB == 16) {
+#define IFQ_MC(BN, G, S, SO, KS) \
+  if (bn == BN && ks == KS) return TcInst<BN, G, S, SO, KS>::max_clusters(nsm);
+    IFQ_TC_SPLIT_VARIANTS(IFQ_MC, GB, SB, SBO)
+#undef IFQ_MC
+  }
+  return 0;
+}
+
+// K split of the tensor-core kernel (1: none).  Splitting K over a cluster of two CTAs halves each
+// CTA's K stages but adds the exchange of partial sums, and with as many tiles as SMs it leaves the
+// per-CTA work unchanged.  Measured on GB300: AlexNet FC6 (one 128-row tile, K = 9216) 20.6 -> 16.5
+// us at BN = 64; every ResNet-18 layer at batch 32 slower (the 7x7 512-channel layers have 104
+// tiles at BN = 64, so a split would need 208 CTAs).  So the split is taken only where the unsplit
+// layer would leave more than half of the SMs idle, the split grid fits in one wave of clusters and
+// every CTA keeps at least eight K stages.  IFQ_TC_KS = 1 / 2 forbids / forces it where eligible.
+template <int GB, int SB, int SBO>
+void choose_split(const ConvGeom& g, int cout, int nsm, int* bn, int* ks) {
+  *ks = 1;
+  if constexpr (GB == 16) {
+    const int forced = env_int("IFQ_TC_KS", 0);
+    if (forced == 1) return;
+    const int nk = g.Kpad / kBK;
+    if (cout <= 32 || nk < 4) return;   // the split instance is BN = 64, KS = 2
+    const long long tiles = (long long)ceil_div(g.M, kBM) * ceil_div(cout, 64);
+    const int mc = tc_max_clusters<GB, SB, SBO>(64, 2, nsm);
+    if (mc < 1) return;
+    if (forced == 2 || (nk >= 16 && 2 * tiles <= nsm && tiles <= mc)) {
+      *bn = 64;
+      *ks = 2;
+    }
+  }
+}
+
+template <int GB, int SB, int SBO>
+cudaError_t launch_tc_gb(int bn, int ks, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
+#define IFQ_LAUNCH(BN, G, S, SO, KS) \
+  if (bn == BN && ks == KS) return TcInst<BN, G, S, SO, KS>::launch(tm, a, nsm, st);
   IFQ_TC_VARIANTS(IFQ_LAUNCH, GB, SB, SBO)
+  if constexpr (GB == 16) {
+    IFQ_TC_SPLIT_VARIANTS(IFQ_LAUNCH, GB, SB, SBO)
+  }
 #undef IFQ_LAUNCH
   return cudaErrorInvalidValue;
 }
@@ -429,22 +526,27 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     else if (d->cout <= 16) e = launch_k(conv_direct_kernel<8>, grid, block, 0, st, a);
     else e = launch_k(conv_direct_kernel<16>, grid, block, 0, st, a);
   } else if (path == IFQ_PATH_TC) {
-    const int bn = choose_bn(g, d->cout, nsm);
+    int bn = choose_bn(g, d->cout, nsm), ks = 1;
+    const int gb = granule_bytes(d, g);
+    if (gb == 16) {
+      if (g.sbi == 2) choose_split<16, 2, 2>(g, d->cout, nsm, &bn, &ks);
+      else if (g.sb == 4) choose_split<16, 4, 4>(g, d->cout, nsm, &bn, &ks);
+      else choose_split<16, 4, 2>(g, d->cout, nsm, &bn, &ks);
+    }
     CUtensorMap tm;
     if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
-    const int gb = granule_bytes(d, g);
     if (g.sbi == 2) {
-      if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, tm, a, nsm, st);
-      else if (gb == 4) e = launch_tc_gb<4, 2, 2>(bn, tm, a, nsm, st);
-      else e = launch_tc_gb<1, 2, 2>(bn, tm, a, nsm, st);
+      if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st);
+      else if (gb == 4) e = launch_tc_gb<4, 2, 2>(bn, ks, tm, a, nsm, st);
+      else e = launch_tc_gb<1, 2, 2>(bn, ks, tm, a, nsm, st);
     } else if (g.sb == 4) {
-      if (gb == 16) e = launch_tc_gb<16, 4, 4>(bn, tm, a, nsm, st);
-      else e = launch_tc_gb<4, 4, 4>(bn, tm, a, nsm, st);
+      if (gb == 16) e = launch_tc_gb<16, 4, 4>(bn, ks, tm, a, nsm, st);
+      else e = launch_tc_gb<4, 4, 4>(bn, ks, tm, a, nsm, st);
     } else {   // 8-bit input values, 2-bit output codes
-      if (gb == 16) e = launch_tc_gb<16, 4, 2>(bn, tm, a, nsm, st);
-      else e = launch_tc_gb<4, 4, 2>(bn, tm, a, nsm, st);
+      if (gb == 16) e = launch_tc_gb<16, 4, 2>(bn, ks, tm, a, nsm, st);
+      else e = launch_tc_gb<4, 4, 2>(bn, ks, tm, a, nsm, st);
     }
   } else if (narrow_supported(d, g)) {
     NarrowArgs a;

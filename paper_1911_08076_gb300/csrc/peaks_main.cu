@@ -83,8 +83,7 @@ __global__ void __launch_bounds__(128) tc_rate(int N, int iters, float* sink) {
   asm volatile("tcgen05.fence::after_thread_sync;");
   if (warp == 0) {
     uint32_t r;
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(r) : "r"(tm));
-    asm volatile("tcgen05.wait::ld.sync.aligned;");
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];\n\ttcgen05.wait::ld.sync.aligned;" : "=r"(r) : "r"(tm));
     if (tid == 0) sink[blockIdx.x] = __uint_as_float(r);
   }
   asm volatile("tcgen05.fence::before_thread_sync;");

@@ -164,6 +164,10 @@ __device__ __forceinline__ bool wait_deps(const StackLayer* sL, unsigned int* cn
   return ok;
 }
 
+// Own K stages of packed codes a gather thread of the stack kernel keeps in registers (one: the
+// stack kernel's extra state leaves no room for a second at 72 registers).
+constexpr int kStackAhead = 1;
+
 // One gather group's share of one layer: its own K stages q = q0, q0+4, ... of
 // the layer's local stage sequence (stage index it_base + q in the CTA ring).
 template <int GB>
@@ -189,28 +193,30 @@ __device__ __forceinline__ bool stack_gather_layer(const ConvArgs& a, const int2
       if (l_tile < nl) g = row_geom(a, (int)fdiv((uint32_t)((int)blockIdx.x + l_tile * G), a.div_nt) * kBM + r);
     }
   };
-  uint4 ring_lo[kAhead], ring_hi[kAhead];
+  uint4 ring_lo[kStackAhead], ring_hi[kStackAhead];
 #pragma unroll
-  for (int d = 0; d < kAhead; ++d) {
+  for (int d = 0; d < kStackAhead; ++d) {
     ring_lo[d] = ring_hi[d] = make_uint4(0u, 0u, 0u, 0u);
     if (d < own) next_load(ring_lo[d], ring_hi[d]);
   }
 #pragma unroll 1
-  for (int base = 0; base < own; base += kAhead) {
+  for (int base = 0; base < own; base += kStackAhead) {
 #pragma unroll
-    for (int d = 0; d < kAhead; ++d) {
+    for (int d = 0; d < kStackAhead; ++d) {
       const int j = base + d;
       if (j < own) {
         const uint4 lo = ring_lo[d], hi = ring_hi[d];
-        if (j + kAhead < own) next_load(ring_lo[d], ring_hi[d]);
+        if (j + kStackAhead < own) next_load(ring_lo[d], ring_hi[d]);
         const int it = it_base + q0 + kGatherGroups * j;
         const int s = it % kStages;
         const uint32_t ph = (uint32_t)(it / kStages) & 1u;
         if (!__all_sync(0xffffffffu, ok && mbar_wait_backoff(barBase + 8u * (kStages + s), ph ^ 1u, 64))) return false;   // empty(s)
         tc_fence_after();
-        expand_tmem_store(tA + (uint32_t)(s * 32), lo);
-        expand_tmem_store(tA + (uint32_t)(s * 32 + 16), hi);
-        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+        uint32_t o[16];
+        expand2(lo, o);
+        tmem_st16_sync(tA + (uint32_t)(s * 32), o);
+        expand2(hi, o);
+        tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(barBase + 8u * s);   // full(s)
@@ -232,13 +238,7 @@ __device__ __forceinline__ void stack_epi_tile(const ConvArgs& a, uint32_t tacc,
 #pragma unroll
   for (int c0 = 0; c0 < CW; c0 += 16) {
     uint32_t v[16];
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
-        : "r"(tacc + c0)
-        : "memory");
-    tmem_ld_wait();
+    tmem_ld16_sync(tacc + c0, v);
     uint32_t wd = 0;
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
