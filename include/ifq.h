@@ -373,6 +373,29 @@ int ifq_graph_launch(ifq_graph* g, void* stream);
 int ifq_graph_destroy(ifq_graph* g);
 
 /*
+ * ifq_graph_create_io -- ifq_graph_create whose graph also moves the stack's
+ * input in and its results out, so that one ifq_graph_launch serves a request
+ * end to end.  The paper has no counterpart; this is a serving convenience.
+ *   x_src, x_bytes: when x_src is not NULL, the graph first copies x_bytes from
+ *     x_src to x.  x_bytes must equal the bytes of packed input that the layers
+ *     with src = -1 read (n * h * w * c * field bits / 8; IFQ_ESHAPE otherwise).
+ *   y_codes_dst, y_acc_dst: NULL, or arrays of nlayers destinations.  When entry
+ *     i is not NULL, the graph copies layer i's y_codes (y_acc) buffer, all of
+ *     it, to that address right after layer i, on layer i's branch of the graph.
+ *     The results of a side branch are then copied while the main chain runs.
+ *     A destination for a buffer that layer i does not have is IFQ_EINVAL.
+ * The addresses are part of the graph: every launch copies from and to the same
+ * buffers.  A copy between buffers the device addresses directly (device
+ * memory, or pinned host memory under unified addressing), 16-byte aligned and
+ * a multiple of 16 bytes, runs on the SMs as in ifq_copy_bytes; any other is a
+ * cudaMemcpyAsync node.  Argument errors are returned before anything is
+ * captured.
+ */
+int ifq_graph_create_io(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes,
+                        const void* x_src, size_t x_bytes, void* const* y_codes_dst, void* const* y_acc_dst,
+                        void* stream, ifq_graph** out);
+
+/*
  * Codes <-> packed format helpers (device buffers; n % 4 == 0 codes, one code
  * per byte on the unpacked side).  The _kbits forms take the code width
  * (0, 2, 3, 4; a code keeps its low f bits); the plain forms are kbits = 2.

@@ -933,6 +933,99 @@ int run_stack(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t 
   return IFQ_OK;
 }
 
+// Whether the device addresses p directly at the same address: device or managed memory, or
+// pinned host memory under unified addressing.
+bool device_addressable(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();   // an unregistered pointer is not an error to keep
+    return false;
+  }
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) return true;
+  return at.type == cudaMemoryTypeHost && at.devicePointer == p;
+}
+
+// One copy of a graph's input or of a layer's result; `sm`: on the SMs (copy16_kernel), else
+// cudaMemcpyAsync.
+struct IoCopy {
+  void* dst;
+  const void* src;
+  size_t bytes;
+  bool sm;
+};
+
+IoCopy make_copy(void* dst, const void* src, size_t n) {
+  const bool sm = aligned16(dst) && aligned16(src) && n % 16 == 0 && device_addressable(dst) && device_addressable(src);
+  return IoCopy{dst, src, n, sm};
+}
+
+int enqueue_copy(const IoCopy& c, int nsm, cudaStream_t st) {
+  if (c.bytes == 0) return IFQ_OK;
+  if (!c.sm) return cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyDefault, st) == cudaSuccess ? IFQ_OK : IFQ_ECUDA;
+  const size_t n16 = c.bytes / 16;
+  size_t blocks = (n16 + 255) / 256;
+  if (blocks > (size_t)nsm * 8) blocks = (size_t)nsm * 8;
+  return launch_k(copy16_kernel, dim3((unsigned)blocks), dim3(256), 0, st, (const uint4*)c.src, (uint4*)c.dst, n16) ==
+                 cudaSuccess
+             ? IFQ_OK
+             : IFQ_ECUDA;
+}
+
+// The copies a graph makes around the stack: the input before the first layer, and after layer
+// i the results of layer i.
+struct IoPlan {
+  IoCopy in{nullptr, nullptr, 0, false};
+  std::vector<std::vector<IoCopy>> after;
+  int nsm = 0;
+  int copies_after(int i, cudaStream_t st) const {
+    if (after.empty()) return IFQ_OK;
+    for (const IoCopy& c : after[i]) {
+      const int rc = enqueue_copy(c, nsm, st);
+      if (rc) return rc;
+    }
+    return IFQ_OK;
+  }
+};
+
+// Bytes of layer i's code and accumulator buffers (0 where it has none).
+int layer_buffer_bytes(const ifq_layer* layers, int i, size_t* codes, size_t* acc) {
+  int n, h, w, c, kb;
+  bool has_codes;
+  const int rc = layer_out(layers, i, &n, &h, &w, &c, &has_codes, &kb);
+  if (rc) return rc;
+  int k, f, lvl;
+  if (code_width(kb, &k, &f, &lvl)) f = 2;
+  const size_t px = (size_t)n * h * w;
+  const ifq_layer& l = layers[i];
+  *codes = has_codes ? px * c * f / 8 : 0;
+  *acc = (l.kind == IFQ_LAYER_FIXED || (l.kind == IFQ_LAYER_CONV && (l.conv.out_mode & IFQ_OUT_ACC))) ? px * c * 4 : 0;
+  return IFQ_OK;
+}
+
+// Bytes of packed input read by the layers with src = -1 (they must agree).
+int stack_input_bytes(const ifq_layer* layers, int nlayers, size_t* bytes) {
+  *bytes = 0;
+  for (int i = 0; i < nlayers; ++i) {
+    const ifq_layer& l = layers[i];
+    if (l.src >= 0 || l.kind == IFQ_LAYER_FIXED) continue;
+    size_t b;
+    if (l.kind == IFQ_LAYER_CONV) {
+      ConvGeom g;
+      const int rc = check_conv(&l.conv, &g);
+      if (rc) return rc;
+      b = (size_t)l.conv.n * l.conv.h * l.conv.w * pixel_bytes(&l.conv, g);
+    } else {
+      int k, f, lvl;
+      const int rc = code_width(l.pool.kbits, &k, &f, &lvl);
+      if (rc) return rc;
+      b = (size_t)l.pool.n * l.pool.h * l.pool.w * l.pool.c * f / 8;
+    }
+    if (*bytes && *bytes != b) return IFQ_ESHAPE;
+    *bytes = b;
+  }
+  return IFQ_OK;
+}
+
 // Stream capture of a stack with its side branches: a layer whose output no later layer reads (a
 // ResNet shortcut conv), other than the last, does not hold up the layers after it, so it runs on a
 // second stream that forks from the main stream when its source layer has run and joins it at the
@@ -943,7 +1036,9 @@ struct BranchedCapture {
   cudaStream_t side = nullptr;
   std::vector<cudaEvent_t> events;
 
-  int run(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t main) {
+  int run(const ifq_layer* layers, int nlayers, const void* x, cudaStream_t main, const IoPlan& io) {
+    int rc;
+    if ((rc = enqueue_copy(io.in, io.nsm, main))) return rc;
     std::vector<char> read(nlayers, 0);
     for (int i = 0; i < nlayers; ++i)
       if (layers[i].src >= 0) read[layers[i].src] = 1;
@@ -952,21 +1047,25 @@ struct BranchedCapture {
     for (int i = 0; i + 1 < nlayers; ++i)
       if (!read[i]) is_side[i] = 1, ++nside;
     const char* v = getenv("IFQ_GRAPH_BRANCH");
-    if (nside == 0 || (v && v[0] == '0')) return run_stack(layers, nlayers, x, main);
+    if (nside == 0 || (v && v[0] == '0')) {
+      for (int i = 0; i < nlayers; ++i)
+        if ((rc = run_layer(layers, i, x, main)) || (rc = io.copies_after(i, main))) return rc;
+      return IFQ_OK;
+    }
     if (cudaStreamCreateWithFlags(&side, cudaStreamNonBlocking) != cudaSuccess) return IFQ_ECUDA;
     auto fork = [&](int s) -> int {   // side layer s after everything issued so far on main
       cudaEvent_t e;
       if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return IFQ_ECUDA;
       events.push_back(e);
       if (cudaEventRecord(e, main) != cudaSuccess || cudaStreamWaitEvent(side, e, 0) != cudaSuccess) return IFQ_ECUDA;
-      return run_layer(layers, s, x, side);
+      const int r = run_layer(layers, s, x, side);
+      return r ? r : io.copies_after(s, side);
     };
-    int rc;
     for (int s = 0; s < nlayers; ++s)   // side layers on the stack input fork before anything runs
       if (is_side[s] && layers[s].src < 0 && (rc = fork(s))) return rc;
     for (int i = 0; i < nlayers; ++i) {
       if (is_side[i]) continue;
-      if ((rc = run_layer(layers, i, x, main))) return rc;
+      if ((rc = run_layer(layers, i, x, main)) || (rc = io.copies_after(i, main))) return rc;
       for (int s = i + 1; s < nlayers; ++s)
         if (is_side[s] && layers[s].src == i && (rc = fork(s))) return rc;
     }
@@ -1082,14 +1181,12 @@ int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, voi
   return run_stack(layers, nlayers, x, S(stream));
 }
 
-int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream,
-                     ifq_graph** out) {
-  if (!out) return IFQ_EINVAL;
-  *out = nullptr;
-  int rc = check_stack(layers, nlayers, x);
-  if (rc) return rc;
-  if ((rc = ensure_init(nullptr))) return rc;
-  if (!get_encode()) return IFQ_ECUDA;
+}  // extern "C"
+
+namespace {
+
+int graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, const IoPlan& io,
+                 void* stream, ifq_graph** out) {
   cudaStream_t cap = S(stream);
   bool own = false;
   if (cap == nullptr) {
@@ -1097,12 +1194,21 @@ int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* 
     own = true;
   }
   ifq_graph* g = new ifq_graph();
-  rc = IFQ_OK;
+  int rc = IFQ_OK;
   if (cudaStreamBeginCapture(cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) rc = IFQ_ECUDA;
   if (!rc) {
     BranchedCapture bc;
-    int frc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, cap);
-    if (frc == IFQ_EUNSUPPORTED) frc = bc.run(layers, nlayers, x, cap);
+    int frc = enqueue_copy(io.in, io.nsm, cap);
+    if (!frc) {
+      frc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, cap);
+      if (!frc) {   // the whole stack in one launch: every result copy after it
+        for (int i = 0; i < nlayers && !frc; ++i) frc = io.copies_after(i, cap);
+      } else if (frc == IFQ_EUNSUPPORTED) {
+        IoPlan rest = io;
+        rest.in = IoCopy{nullptr, nullptr, 0, false};   // enqueued above
+        frc = bc.run(layers, nlayers, x, cap, rest);
+      }
+    }
     const cudaError_t e = cudaStreamEndCapture(cap, &g->graph);
     bc.release();
     if (frc) rc = frc;
@@ -1116,6 +1222,49 @@ int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* 
   }
   *out = g;
   return IFQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int ifq_graph_create(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes, void* stream,
+                     ifq_graph** out) {
+  return ifq_graph_create_io(layers, nlayers, x, ws, ws_bytes, nullptr, 0, nullptr, nullptr, stream, out);
+}
+
+int ifq_graph_create_io(const ifq_layer* layers, int nlayers, const void* x, void* ws, size_t ws_bytes,
+                        const void* x_src, size_t x_bytes, void* const* y_codes_dst, void* const* y_acc_dst,
+                        void* stream, ifq_graph** out) {
+  if (!out) return IFQ_EINVAL;
+  *out = nullptr;
+  int rc = check_stack(layers, nlayers, x);
+  if (rc) return rc;
+  int nsm = 0;
+  if ((rc = ensure_init(&nsm))) return rc;
+  if (!get_encode()) return IFQ_ECUDA;
+  // the copies are planned (sizes checked, device addressability looked up) before the capture
+  IoPlan io;
+  io.nsm = nsm;
+  if (x_src) {
+    size_t need = 0;
+    if ((rc = stack_input_bytes(layers, nlayers, &need))) return rc;
+    if (x_bytes != need) return IFQ_ESHAPE;
+    io.in = make_copy(const_cast<void*>(x), x_src, x_bytes);
+  }
+  if (y_codes_dst || y_acc_dst) {
+    io.after.resize(nlayers);
+    for (int i = 0; i < nlayers; ++i) {
+      size_t cb = 0, ab = 0;
+      if ((rc = layer_buffer_bytes(layers, i, &cb, &ab))) return rc;
+      void* dc = y_codes_dst ? y_codes_dst[i] : nullptr;
+      void* da = y_acc_dst ? y_acc_dst[i] : nullptr;
+      if ((dc && (!cb || !layers[i].y_codes)) || (da && (!ab || !layers[i].y_acc))) return IFQ_EINVAL;
+      if (dc) io.after[i].push_back(make_copy(dc, layers[i].y_codes, cb));
+      if (da) io.after[i].push_back(make_copy(da, layers[i].y_acc, ab));
+    }
+  }
+  return graph_create(layers, nlayers, x, ws, ws_bytes, io, stream, out);
 }
 
 int ifq_graph_launch(ifq_graph* g, void* stream) {
@@ -1184,15 +1333,6 @@ int ifq_fixed_output(const int32_t* acc, int rows, int cout, const int64_t* mul,
 
 // Whether the device can dereference p as is: device or managed memory, or host memory that
 // cudaHostAlloc / cudaHostRegister mapped at the same address (unified addressing).
-bool device_addressable(const void* p) {
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
-    cudaGetLastError();   // an unregistered pointer is not an error to keep
-    return false;
-  }
-  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) return true;
-  return at.type == cudaMemoryTypeHost && at.devicePointer == p;
-}
 
 int ifq_copy_bytes(void* dst, const void* src, size_t n, void* stream) {
   if ((!dst || !src) && n) return IFQ_EINVAL;

@@ -23,7 +23,7 @@ extern "C" const char* ifq_status_str(int s) {
   }
 }
 
-extern "C" int ifq_version(void) { return 300; }   // 3.0: in_bits, fixed-point output layers
+extern "C" int ifq_version(void) { return 301; }   // 3.1: graphs with the input and result copies
 
 // Eq. (3)'s uniform level i (1-based) in the compact form of Sec. 3.2.
 static inline double level(int i, double q_base, double q_offset) { return (double)i * q_base + q_offset; }

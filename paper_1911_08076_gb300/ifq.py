@@ -78,6 +78,8 @@ _SIGS = {
     "ifq_forward": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P], _I),
     "ifq_forward_noalloc": ([ctypes.POINTER(Layer), _I, _P, _P], _I),
     "ifq_graph_create": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, ctypes.POINTER(_P)], _I),
+    "ifq_graph_create_io": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, _SZ, ctypes.POINTER(_P), ctypes.POINTER(_P),
+                             _P, ctypes.POINTER(_P)], _I),
     "ifq_graph_launch": ([_P, _P], _I),
     "ifq_graph_destroy": ([_P], _I),
     "ifq_pack_codes": ([_P, _P, _SZ, _P], _I),
@@ -289,6 +291,26 @@ def ifq_graph_create(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, str
     g = _P()
     _ok(lib().ifq_graph_create(arr, n, _ptr(x), _ptr(ws), ws_bytes, _stream(stream), ctypes.byref(g)),
         "ifq_graph_create")
+    return g.value
+
+
+def ifq_graph_create_io(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, x_src=None, x_bytes: int = 0,
+                        y_codes_dst: Optional[Sequence] = None, y_acc_dst: Optional[Sequence] = None,
+                        stream=None) -> int:
+    """ifq_graph_create with the input copy (x_src -> x, x_bytes) and per-layer result copies
+    (y_codes_dst[i] / y_acc_dst[i]: a tensor, an address or None) inside the graph."""
+    arr, n = _layer_array(layers)
+
+    def dsts(seq):
+        if seq is None:
+            return None
+        if len(seq) != n:
+            raise ValueError("one destination (or None) per layer")
+        return (_P * n)(*[_ptr(t) for t in seq])
+
+    g = _P()
+    _ok(lib().ifq_graph_create_io(arr, n, _ptr(x), _ptr(ws), ws_bytes, _ptr(x_src), x_bytes, dsts(y_codes_dst),
+                                  dsts(y_acc_dst), _stream(stream), ctypes.byref(g)), "ifq_graph_create_io")
     return g.value
 
 

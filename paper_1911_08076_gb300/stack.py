@@ -167,6 +167,41 @@ class DeviceStack:
         self._graph = ifq.ifq_graph_create(self.layers, x, self.ws, self.ws_bytes, stream)
         return self._graph
 
+    def leaf_spans(self):
+        """(byte offset, bytes) of every leaf output buffer within leaf_block (the block pads each
+        buffer to 256 bytes; the padding is not part of any result)."""
+        base = self.leaf_block.data_ptr()
+        spans = []
+        for li in self.leaf_layers():
+            for t in (self.y_codes.get(li), self.y_acc.get(li)):
+                if t is not None:
+                    spans.append((t.data_ptr() - base, t.numel() * t.element_size()))
+        return spans
+
+    def leaf_results_equal(self, leaf_host: torch.Tensor, other: Optional[torch.Tensor] = None) -> bool:
+        """Whether the host copy of the leaf block holds the same results as this stack's device block
+        (or as `other`, a block of the same layout), buffer by buffer."""
+        dev = (self.leaf_block if other is None else other).cpu()
+        return all(torch.equal(leaf_host[o:o + n], dev[o:o + n]) for o, n in self.leaf_spans())
+
+    def capture_io(self, x: torch.Tensor, x_host: torch.Tensor, leaf_host: torch.Tensor, stream=None) -> int:
+        """Capture ifq_forward on input buffer x into a CUDA graph that also copies x_host (pinned)
+        into x first and every leaf layer's outputs into leaf_host (pinned, the size of leaf_block,
+        the same layout) right after that layer (replaced on each call)."""
+        assert leaf_host.numel() * leaf_host.element_size() == self.leaf_block.numel()
+        base_d, base_h = self.leaf_block.data_ptr(), leaf_host.data_ptr()
+        n = len(self.layers)
+        codes_dst, acc_dst = [None] * n, [None] * n
+        for li in self.leaf_layers():
+            if li in self.y_codes:
+                codes_dst[li] = base_h + (self.y_codes[li].data_ptr() - base_d)
+            if li in self.y_acc:
+                acc_dst[li] = base_h + (self.y_acc[li].data_ptr() - base_d)
+        self.release()
+        self._graph = ifq.ifq_graph_create_io(self.layers, x, self.ws, self.ws_bytes, x_host,
+                                              x_host.numel() * x_host.element_size(), codes_dst, acc_dst, stream)
+        return self._graph
+
     def replay(self, stream=None):
         ifq.ifq_graph_launch(self._graph, stream)
 

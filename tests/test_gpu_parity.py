@@ -552,3 +552,54 @@ def test_bounded_wait_reports_timeout_and_the_context_survives():
     T, sg = _fold_gpu(prm, 576)
     codes, acc = _run_conv(x, w, T, sg, 1, 1, ifq.IFQ_OUT_BOTH, ifq.IFQ_PATH_TC)
     assert (acc == O.conv_acc(x, w, 1, 1)).all()
+
+
+@pytest.mark.parametrize("name,batch", [("resnet18", 4), ("alexnet", 2), ("tinieryolo_full", 2)])
+def test_graph_with_copies_serves_requests_end_to_end(name, batch):
+    """ifq_graph_create_io: one graph launch copies the pinned host input in, runs the stack and copies
+    every result out (the side branch's right after its layer).  The host results equal the device
+    buffers and a plain forward's, and a new input written into the same host buffer gives the new
+    results on the next launch (the copies are part of the graph)."""
+    wl = synth.get(name, batch=batch)
+    x, params = synth.draw_workload(wl, batch=batch)
+    fb = 8 if wl.in_bits == 8 else wl.kbits
+    st = DeviceStack(wl, params, batch=batch, device=DEV)
+    ref = DeviceStack(wl, params, batch=batch, device=DEV)
+    x_host = torch.from_numpy(synth.pack_codes(x, fb)).pin_memory()
+    leaf_host = torch.zeros(st.leaf_block.shape, dtype=torch.uint8).pin_memory()
+    xd = st.input_buffer()
+    stream = torch.cuda.Stream()
+    st.capture_io(xd, x_host, leaf_host, stream)
+    rng = np.random.default_rng(3)
+    for trial in range(2):
+        if trial:   # a new request in the same pinned buffer
+            x2 = rng.integers(0, 256 if wl.in_bits == 8 else 1 << wl.kbits, x.shape, dtype=np.uint8)
+            if wl.in_bits == 8:
+                x2[..., 3:] = 0
+            x_host.copy_(torch.from_numpy(synth.pack_codes(x2, fb)))
+        st.replay(stream)
+        stream.synchronize()
+        assert ifq.ifq_device_status() == ifq.IFQ_OK
+        ref.forward(x_host.to(DEV))
+        torch.cuda.synchronize()
+        assert st.leaf_results_equal(leaf_host)
+        assert st.leaf_results_equal(leaf_host, ref.leaf_block)
+    st.release()
+
+
+def test_graph_with_copies_rejects_bad_io():
+    wl = synth.get("resnet18", batch=2)
+    x, params = synth.draw_workload(wl, batch=2)
+    st = DeviceStack(wl, params, batch=2, device=DEV)
+    xd = st.input_buffer()
+    x_host = torch.empty(xd.numel(), dtype=torch.uint8).pin_memory()
+    with pytest.raises(ifq.IfqError) as e:   # one byte short of the stack's input
+        ifq.ifq_graph_create_io(st.layers, xd, st.ws, st.ws_bytes, x_host, xd.numel() - 1)
+    assert e.value.status == ifq.IFQ_ESHAPE
+    acc_dst = [None] * len(st.layers)
+    acc_dst[0] = torch.empty(16, dtype=torch.int32, device=DEV)   # layer 0 writes no accumulators
+    with pytest.raises(ifq.IfqError) as e:
+        ifq.ifq_graph_create_io(st.layers, xd, st.ws, st.ws_bytes, None, 0, None, acc_dst)
+    assert e.value.status == ifq.IFQ_EINVAL
+    with pytest.raises(ValueError):
+        ifq.ifq_graph_create_io(st.layers, xd, st.ws, st.ws_bytes, None, 0, [None])
