@@ -135,6 +135,11 @@ __device__ __forceinline__ uint4 ld_codes16(const uint8_t* p) {
   else return __ldg((const uint4*)p);
 }
 template <bool COHERENT>
+__device__ __forceinline__ uint2 ld_codes8(const uint8_t* p) {
+  if constexpr (COHERENT) return *(const uint2*)p;
+  else return __ldg((const uint2*)p);
+}
+template <bool COHERENT>
 __device__ __forceinline__ uint32_t ld_codes4(const uint8_t* p) {
   if constexpr (COHERENT) return *(const uint32_t*)p;
   else return __ldg((const uint32_t*)p);
@@ -147,13 +152,18 @@ __device__ __forceinline__ uint32_t ld_codes1(const uint8_t* p) {
 
 // 16 packed bytes of row g: unit u of the row's K sequence (bytes 16u .. 16u+15 of the packed
 // K codes, 64 two-bit or 32 four-bit codes), zero outside the image.  The table has one entry
-// per GB bytes, so unit u starts at entry u * 16 / GB.
+// per GB bytes (GB = 16, 8, 4 or 1), so unit u starts at entry u * 16 / GB.
 template <int GB, bool COHERENT = false>
 __device__ __forceinline__ uint4 load_unit(const int2* tab, const RowGeom& g, int u) {
   uint4 v = make_uint4(0u, 0u, 0u, 0u);
   if constexpr (GB == 16) {
     const int2 e = tab[u];
     if (tap_ok(g, e)) v = ld_codes16<COHERENT>(g.base + e.x);
+  } else if constexpr (GB == 8) {
+    const int2 e0 = tab[u * 2], e1 = tab[u * 2 + 1];
+    const uint2 lo = tap_ok(g, e0) ? ld_codes8<COHERENT>(g.base + e0.x) : make_uint2(0u, 0u);
+    const uint2 hi = tap_ok(g, e1) ? ld_codes8<COHERENT>(g.base + e1.x) : make_uint2(0u, 0u);
+    v = make_uint4(lo.x, lo.y, hi.x, hi.y);
   } else if constexpr (GB == 4) {
     uint32_t w[4];
 #pragma unroll

@@ -68,7 +68,7 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
   return 4u * q + (uint32_t)(sv > g.x) + (uint32_t)(sv > g.y) + (uint32_t)(sv > g.z);
 }
 
-// GB: bytes per gathered granule: 16, 4 or 1 (the largest that divides the packed bytes of a
+// GB: bytes per gathered granule: 16, 8, 4 or 1 (the largest that divides the packed bytes of a
 // pixel); SB: bits per stored input code (2 for k = 2, 4 for k = 3 and 4 and for the two nibbles of
 // an 8-bit input value); SBO: bits per stored output code (2 or 4).
 //

@@ -184,10 +184,11 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   std::lock_guard<std::mutex> lk(g_dev_mu);
   DevState& d = g_dev[dev];
   if (!d.init) {
-    if (set_attrs_gb<16, 2, 2>() != cudaSuccess || set_attrs_gb<4, 2, 2>() != cudaSuccess ||
-        set_attrs_gb<1, 2, 2>() != cudaSuccess || set_attrs_gb<16, 4, 4>() != cudaSuccess ||
+    if (set_attrs_gb<16, 2, 2>() != cudaSuccess || set_attrs_gb<8, 2, 2>() != cudaSuccess ||
+        set_attrs_gb<4, 2, 2>() != cudaSuccess || set_attrs_gb<1, 2, 2>() != cudaSuccess ||
+        set_attrs_gb<16, 4, 4>() != cudaSuccess || set_attrs_gb<8, 4, 4>() != cudaSuccess ||
         set_attrs_gb<4, 4, 4>() != cudaSuccess || set_attrs_gb<16, 4, 2>() != cudaSuccess ||
-        set_attrs_gb<4, 4, 2>() != cudaSuccess)
+        set_attrs_gb<8, 4, 2>() != cudaSuccess || set_attrs_gb<4, 4, 2>() != cudaSuccess)
       return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
     if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
@@ -419,10 +420,11 @@ cudaError_t launch_tc_gb(int bn, int ks, const CUtensorMap& tm, const ConvArgs& 
 // Bytes of packed codes per input pixel.
 int pixel_bytes(const ifq_conv_desc* d, const ConvGeom& g) { return g.cink * g.sbi / 8; }
 
-// Bytes of packed codes per gathered granule: the largest of 16, 4, 1 that divides a pixel's bytes.
-int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
+// Bytes of packed codes per gathered granule: the largest of 16, 8, 4, 1 that divides a pixel's
+// bytes (the persistent stack kernel has no 8-byte instance: 16, 4, 1 there).
+int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g, bool stack = false) {
   const int pb = pixel_bytes(d, g);
-  return pb % 16 == 0 ? 16 : (pb % 4 == 0 ? 4 : 1);
+  return pb % 16 == 0 ? 16 : (pb % 8 == 0 && !stack ? 8 : (pb % 4 == 0 ? 4 : 1));
 }
 
 // Whether the tensor-core kernel supports this shape: an accumulator magnitude inside the
@@ -431,7 +433,7 @@ int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
 bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
   const long long amax = (long long)(g.in8 ? 255 : g.lvl) * g.K;   // largest |A|
   if (amax > kTcMaxAcc || d->kh > 32 || d->kw > 32) return false;
-  const int gb = granule_bytes(d, g);
+  const int gb = granule_bytes(d, g, true);   // the smaller granule of the two kernels: the larger table
   if (g.sbi == 4 && gb == 1) return false;
   if ((long long)g.Kpad * g.sbi / 8 / gb > kMaxTab) return false;
   const long long pb = pixel_bytes(d, g);
@@ -452,7 +454,7 @@ bool encode_wmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, 
 }
 
 void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const void* x, const int32_t* thr,
-                    const int8_t* sign, uint8_t* yc, int32_t* ya, ConvArgs* a) {
+                    const int8_t* sign, uint8_t* yc, int32_t* ya, ConvArgs* a, bool stack = false) {
   a->x = (const uint8_t*)x;
   a->thr = thr;
   a->sign = sign;
@@ -467,7 +469,7 @@ void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const voi
   a->nk = g.Kpad / kBK;
   a->nt = ceil_div(d->cout, bn);
   a->ntiles = ceil_div(g.M, kBM) * a->nt;
-  a->ntab = g.Kpad * g.sbi / 8 / granule_bytes(d, g);
+  a->ntab = g.Kpad * g.sbi / 8 / granule_bytes(d, g, stack);
   a->div_hw = make_fastdiv((uint32_t)(g.ho * g.wo));
   a->div_wo = make_fastdiv((uint32_t)g.wo);
   a->div_nt = make_fastdiv((uint32_t)a->nt);
@@ -539,13 +541,16 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
     if (g.sbi == 2) {
       if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st);
+      else if (gb == 8) e = launch_tc_gb<8, 2, 2>(bn, ks, tm, a, nsm, st);
       else if (gb == 4) e = launch_tc_gb<4, 2, 2>(bn, ks, tm, a, nsm, st);
       else e = launch_tc_gb<1, 2, 2>(bn, ks, tm, a, nsm, st);
     } else if (g.sb == 4) {
       if (gb == 16) e = launch_tc_gb<16, 4, 4>(bn, ks, tm, a, nsm, st);
+      else if (gb == 8) e = launch_tc_gb<8, 4, 4>(bn, ks, tm, a, nsm, st);
       else e = launch_tc_gb<4, 4, 4>(bn, ks, tm, a, nsm, st);
     } else {   // 8-bit input values, 2-bit output codes
       if (gb == 16) e = launch_tc_gb<16, 4, 2>(bn, ks, tm, a, nsm, st);
+      else if (gb == 8) e = launch_tc_gb<8, 4, 2>(bn, ks, tm, a, nsm, st);
       else e = launch_tc_gb<4, 4, 2>(bn, ks, tm, a, nsm, st);
     }
   } else if (narrow_supported(d, g)) {
@@ -773,7 +778,7 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     if (g.pool > 1 || g.kb != 2 || g.in8) return false;   // the persistent kernel: 2-bit codes, no fused pool
     if (g.M == 0) return false;                           // an empty batch runs (as nothing) layer by layer
     if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
-    tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g));
+    tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g, true));
   }
   if (tab > kMaxStackTab) return false;
   if (bytes) *bytes = round_up(stack_counters(layers, nlayers) * sizeof(unsigned int), 256);
@@ -866,9 +871,9 @@ int launch_stack_kernel(const ifq_layer* layers, int nlayers, const void* x, voi
     uint8_t* yc = (l.conv.out_mode & IFQ_OUT_CODES) ? (uint8_t*)l.y_codes : nullptr;
     int32_t* ya = (l.conv.out_mode & IFQ_OUT_ACC) ? l.y_acc : nullptr;
     StackLayer& S = P.L[i];
-    fill_conv_args(&l.conv, g, bn, l.src < 0 ? x : layers[l.src].y_codes, l.thr, l.sign, yc, ya, &S.a);
+    fill_conv_args(&l.conv, g, bn, l.src < 0 ? x : layers[l.src].y_codes, l.thr, l.sign, yc, ya, &S.a, true);
     S.bn = bn;
-    S.gb = granule_bytes(&l.conv, g);
+    S.gb = granule_bytes(&l.conv, g, true);
     S.tab_off = tab;
     S.dep = l.src;
     S.cnt_off = cnt;

@@ -86,6 +86,8 @@ CONV_CASES = [
     (2, 13, 13, 1024, 30, 1, 1, 0, 2),    # accumulators only, cout = 30
     (1, 14, 14, 256, 512, 3, 2, 1, 1),    # stride 2, codes only
     (1, 5, 5, 64, 64, 3, 1, 0, 1),        # no padding
+    (2, 14, 14, 32, 64, 3, 1, 1, 3),      # 8-byte pixels: 8-byte gather granules
+    (2, 15, 13, 160, 128, 3, 2, 1, 3),    # 40-byte pixels, stride 2, ragged M
 ]
 
 
@@ -118,6 +120,7 @@ POOL_FUSED_CASES = [
     (2, 12, 12, 8, 16, 3, 1, 1, 2, None),       # 1-byte granules
     (2, 16, 16, 128, 256, 3, 1, 1, 4, None),    # 4x4 windows, 16 lanes each
     (1, 28, 28, 64, 128, 3, 2, 1, 2, None),     # strided convolution, then the pool
+    (2, 16, 16, 32, 64, 3, 1, 1, 2, None),      # 8-byte pixels (8-byte granules), then the pool
     (2, 16, 16, 64, 200, 3, 1, 1, 2, 32),       # every channel-tile width
     (2, 16, 16, 64, 200, 3, 1, 1, 2, 64),
     (2, 16, 16, 64, 200, 3, 1, 1, 2, 128),
