@@ -41,6 +41,10 @@ struct ConvArgs {
   // that a window's rows sit in consecutive lanes of one epilogue warp.
   int lpool;
   FastDiv div_phw, div_pwo;         // by (ho/p)*(wo/p), wo/p
+  // 1: the kernels before this one in the stream write neither its filters nor its thresholds (a
+  // layer of a stack after the first), so only the warps that read the previous layer's codes wait
+  // for them; the filter and threshold loads start at once
+  int early;
 };
 
 constexpr int kBM = 128;         // output pixels per tile (MMA M)

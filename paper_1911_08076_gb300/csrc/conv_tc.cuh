@@ -167,7 +167,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   grid_dep_launch();
-  grid_dep_wait();
+  // The gather warps read the previous layer's codes: they wait for the kernels before this one.
+  // With args.early the TMA warp (filters) and the epilogue warps (thresholds) start at once; the
+  // epilogue's stores come after accumulators that the gathered codes fed, so after that wait too.
+  if (!args.early || warp < kGatherWarps) grid_dep_wait();
 
   if (warp < kGatherWarps) {
     // =================== gather: packed codes -> registers -> tensor memory ===================

@@ -474,12 +474,15 @@ void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const voi
   a->div_wo = make_fastdiv((uint32_t)g.wo);
   a->div_nt = make_fastdiv((uint32_t)a->nt);
   a->lpool = g.pool == 4 ? 2 : (g.pool == 2 ? 1 : 0);
+  a->early = 0;
   a->div_phw = make_fastdiv((uint32_t)(g.pho * g.pwo));
   a->div_pwo = make_fastdiv((uint32_t)g.pwo);
 }
 
+// early: the kernels before this one in the stream write neither w_prep nor thr / sign (a layer of a
+// stack after the first), so the tensor-core kernel may load them before its dependency wait.
 int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr, const int8_t* sign,
-             void* y_codes, int32_t* y_acc, cudaStream_t st) {
+             void* y_codes, int32_t* y_acc, cudaStream_t st, bool early = false) {
   ConvGeom g;
   int rc = check_conv(d, &g);
   if (rc) return rc;
@@ -539,6 +542,7 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
+    a.early = early ? 1 : 0;
     if (g.sbi == 2) {
       if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st);
       else if (gb == 8) e = launch_tc_gb<8, 2, 2>(bn, ks, tm, a, nsm, st);
@@ -921,7 +925,8 @@ int noalloc_counters(void** out) {
 int run_layer(const ifq_layer* layers, int i, const void* x, cudaStream_t st) {
   const ifq_layer& l = layers[i];
   const void* in = l.src < 0 ? x : layers[l.src].y_codes;
-  if (l.kind == IFQ_LAYER_CONV) return run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st);
+  // every kernel of a stack before layer i is a layer of the stack or a copy of its input or results
+  if (l.kind == IFQ_LAYER_CONV) return run_conv(&l.conv, in, l.w_prep, l.thr, l.sign, l.y_codes, l.y_acc, st, i > 0);
   if (l.kind == IFQ_LAYER_POOL) return run_pool(&l.pool, in, l.sign, l.y_codes, st);
   const ifq_layer& sl = layers[l.src];
   ConvGeom g;
