@@ -167,12 +167,14 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   grid_dep_launch();
-  // The gather warps read the previous layer's codes: they wait for the kernels before this one.
-  // With args.early the TMA warp (filters) and the epilogue warps (thresholds) start at once; the
-  // epilogue's stores come after accumulators that the gathered codes fed, so after that wait too.
-  if (!args.early || warp < kGatherWarps) grid_dep_wait();
+  // Each role waits for the kernels before this one (griddepcontrol.wait) where it first needs
+  // them.  The gather warps read the previous layer's codes and always wait.  With args.early the
+  // TMA warp (filters) and the epilogue warps (thresholds) start at once: the epilogue's stores
+  // come after accumulators that the gathered codes fed, so after the gather's wait too.  The MMA
+  // warps touch no global memory and never wait.
 
   if (warp < kGatherWarps) {
+    grid_dep_wait();
     // =================== gather: packed codes -> registers -> tensor memory ===================
     const int group = warp >> 2, quarter = warp & 3;
     const int r = quarter * 32 + lane;                       // A row = tensor-memory lane
@@ -232,6 +234,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       }
     }
   } else if (warp == kWarpTma) {
+    if (!args.early) grid_dep_wait();
     // =================== TMA producer (filters) ===================
     // the whole warp runs the loop; one elected lane issues
     int it = 0;
@@ -313,6 +316,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     __syncwarp();
   } else {
     // =================== epilogue ===================
+    if (!args.early) grid_dep_wait();
     // warp pair e, e+4 covers lane quarter (warp % 4), halves 0 and 1 of every column block (the
     // whole tile for KS = 1; with KS > 1 the block of CTA r is columns [r BN/KS, (r+1) BN/KS))
     constexpr int CB = BN / KS;                 // columns of a block
