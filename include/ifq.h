@@ -231,8 +231,8 @@ int ifq_conv_workspace_bytes(const ifq_conv_desc* d, size_t* bytes);
 int ifq_conv2bit(const ifq_conv_desc* d, const void* x, const void* w_prep, const int32_t* thr,
                  const int8_t* sign, void* y_codes, int32_t* y_acc, void* ws, size_t ws_bytes, void* stream);
 
-/* Pooling descriptor (geometry in the header comment); c % 4 == 0. */
-/* Pooling descriptor; kbits is the code width as in ifq_conv_desc (0 means 2). */
+/* Pooling descriptor (geometry in the header comment); c % 4 == 0; kbits is the code width as in
+ * ifq_conv_desc (0 means 2). */
 typedef struct {
   int n, h, w, c;
   int k, stride, pad;
