@@ -223,3 +223,22 @@ def test_separated_fold_refusals():
         ifq.ifq_fold_layer_separated(64, 21, one, one, one * 0, one * 0, one)      # m beyond 20
     with pytest.raises(ifq.IfqError):                                                # sigma floors to 0
         ifq.ifq_fold_layer_separated(64, 4, one, one * 1e4, one * 0, one * 0, one)
+
+
+def test_build_refuses_spilling_tensor_core_kernels():
+    """build() rejects a library in which a warp-specialised tensor-core kernel spills registers to
+    local memory; other kernels may spill."""
+    from paper_1911_08076_gb300 import build as B
+    log = """ptxas info    : Compiling entry function '_ZN3ifq14conv_tc_kernelILi128ELi16ELi2ELi2ELi1EEEv' for 'sm_103a'
+ptxas info    : Function properties for _ZN3ifq14conv_tc_kernelILi128ELi16ELi2ELi2ELi1EEEv
+    24 bytes stack frame, 24 bytes spill stores, 68 bytes spill loads
+ptxas info    : Compiling entry function '_ZN3ifq26maxpool_codes_bytes_kernelILi4EEEvNS_8PoolArgsE' for 'sm_103a'
+    8 bytes stack frame, 8 bytes spill stores, 8 bytes spill loads
+ptxas info    : Compiling entry function '_ZN3ifq17conv_stack_kernelENS_11StackParamsE' for 'sm_103a'
+    16 bytes stack frame, 0 bytes spill stores, 0 bytes spill loads
+ptxas info    : Compiling entry function '_ZN3ifq14conv_tc_kernelILi64ELi16ELi2ELi2ELi1EEEv' for 'sm_103a'
+    0 bytes stack frame, 0 bytes spill stores, 4 bytes spill loads
+"""
+    assert B.spilling_kernels(log) == ["_ZN3ifq14conv_tc_kernelILi128ELi16ELi2ELi2ELi1EEEv",
+                                       "_ZN3ifq14conv_tc_kernelILi64ELi16ELi2ELi2ELi1EEEv"]
+    assert B.spilling_kernels("") == []
