@@ -454,3 +454,29 @@ def test_fold_for_8bit_input_covers_the_whole_range():
     T, s = O.fold(p, O.fold_k(layer))
     codes, ties = O.check_chains(A, p, T, s)
     assert ties == 0 and codes.min() == 0 and codes.max() == 3
+
+
+@pytest.mark.parametrize("h,k,s,p,want", [
+    (227, 11, 4, 0, 55),   # AlexNet conv1
+    (56, 3, 2, 1, 28),     # a ResNet stride-2 3x3
+    (56, 1, 2, 0, 28),     # its 1x1 shortcut
+    (13, 3, 1, 1, 13),     # AlexNet conv3-5 ("same" 3x3)
+    (27, 5, 1, 2, 27),     # AlexNet conv2
+    (7, 3, 1, 0, 5),       # no padding
+])
+def test_conv_out_known_shapes(h, k, s, p, want):
+    """Output size floor((h + 2p - k) / s) + 1 on the shapes of well-known networks."""
+    assert O.conv_out(h, k, s, p) == want
+
+
+@pytest.mark.parametrize("h,k,s,p,want", [
+    (55, 3, 2, 0, 27),     # AlexNet pool1 (overlapping 3x3 / 2)
+    (27, 3, 2, 0, 13),     # pool2
+    (13, 3, 2, 0, 6),      # pool5
+    (416, 2, 2, 0, 208),   # Tiny-YOLO 2x2 / 2
+    (13, 2, 1, 1, 13),     # Tiny-YOLO's last pool: 2x2 / 1 with one padded cell at the right and bottom
+])
+def test_pool_out_known_shapes(h, k, s, p, want):
+    """Pool output size with `p` padded cells at the bottom / right only (Darknet's 2x2 / 1 pool keeps
+    13 x 13)."""
+    assert O.pool_out(h, k, s, p) == want
