@@ -79,3 +79,27 @@ def test_profiled_traffic_is_keyed_by_workload_and_kernel_source(tmp_path, monke
     assert bench.profiled_traffic("wl_a") == 123.0
     assert bench.profiled_traffic("wl_b") is None        # taken on another kernel source
     assert bench.profiled_traffic("wl_c") is None        # no summary for this workload
+
+
+def test_bench_counts_the_resnet18_step_ops_and_algorithmic_bytes():
+    """bench.py's ops (2 per MAC) and algorithmic bytes of the ResNet-18 body at batch 32, against
+    the network written out layer by layer here: 108.5 GOP and 31.2 MB per step."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_1911_08076_gb300 import synth
+    B = 32
+    # (input size, cin, cout, k, stride) of the 19 convs
+    layers = [(56, 64, 64, 3, 1)] * 4
+    for c_in, c, h in ((64, 128, 56), (128, 256, 28), (256, 512, 14)):
+        layers += [(h, c_in, c, 3, 2), (h, c_in, c, 1, 2)] + [(h // 2, c, c, 3, 1)] * 3
+    ops = nbytes = 0
+    for h, cin, cout, k, s in layers:
+        ho = h // s
+        ops += 2 * B * ho * ho * cout * k * k * cin
+        nbytes += B * h * h * cin / 4 + k * k * cin * cout / 8 + 13 * cout + B * ho * ho * cout / 4
+    wl = synth.get("resnet18")
+    convs = [l for l in wl.layers if l.kind == "conv"]
+    assert len(convs) == 19
+    assert abs(sum(bench.conv_ops(l, B) for l in convs) - ops) < 1
+    assert abs(sum(bench.alg_bytes(l, B, 2) for l in convs) - nbytes) < 1
+    assert round(ops / 1e9, 1) == 108.5 and round(nbytes / 1e6, 1) == 31.2
