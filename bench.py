@@ -5,7 +5,11 @@ A step is one pass of the layer stack over one batch: for the default workload,
 the ResNet-18 body (16 3x3 + 3 1x1 binary x 2-bit convs, batch 32) through
 ifq_forward, replayed as a CUDA graph.  Inputs are seeded synthetic 2-bit codes
 already resident in HBM; L2 is flushed (a 256 MB write) between timed steps
-and the flush is outside the per-step CUDA events.
+and the flush is outside the per-step CUDA events.  The end-to-end figure (`e2e`)
+replays a graph from ifq_graph_create_io that also copies the pinned host input
+in and every result out, one launch per step; `roofline` is the conv kernel's
+share of the step against the measured tensor peak, with the DRAM traffic of the
+committed ncu summary of the same workload and kernel source.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload NAME]
 
