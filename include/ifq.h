@@ -84,6 +84,20 @@ const char* ifq_status_str(int status);
 int ifq_version(void);
 
 /*
+ * Environment switches, read on every call that uses them (for experiments; the defaults are the
+ * measured best):
+ *   IFQ_FORCE_PATH   = 1 / 2 / 3: request IFQ_PATH_TC / IFQ_PATH_BITSERIAL / IFQ_PATH_DIRECT
+ *                      where a descriptor says IFQ_PATH_AUTO (ifq_conv_plan reports the result).
+ *   IFQ_TC_BN        = 32 / 64 / 128: the tensor-core kernel's output-channel tile width.
+ *   IFQ_TC_KS        = 1 / 2: forbid / force splitting K over clusters of two CTAs (by default only
+ *                      layers that would leave more than half of the SMs idle are split).
+ *   IFQ_PDL          = 0: launch without programmatic dependent launch.
+ *   IFQ_GRAPH_BRANCH = 0: capture stacks as one chain, without side branches.
+ *   IFQ_STACK        = 1: run qualifying stacks as one persistent launch (ifq_forward).
+ * None changes a result; all change only how it is computed.
+ */
+
+/*
  * ifq_fold_layer -- integrated fixed-point conversion of one quantized
  * substructure (Sec. 3.2, Eq. (6)-(7), floor of the composed thresholds).
  * Host only, pure, thread-safe; nothing is launched.
