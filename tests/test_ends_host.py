@@ -119,3 +119,29 @@ def test_empty_batch_is_a_validated_no_op():
 def test_wait_selftest_refuses_bad_limits():
     assert _status(ifq.ifq_wait_selftest, 0, stream=0) == ifq.IFQ_EINVAL
     assert _status(ifq.ifq_wait_selftest, 2000000, stream=0) == ifq.IFQ_EINVAL
+
+
+def test_synthetic_draws_follow_the_stated_recipe():
+    """The benchmark inputs follow the recipe of the design notes (all workloads seeded): codes
+    uniform on {0..2^k-1}, filters uniform +-1, alpha ~ U(0.5, 1.5), gamma ~ N(1, 0.3), beta ~
+    N(0, 0.5), mean ~ N(0, 2), var ~ U(0.5, 2); the seed is 1911_08076 + the workload index, so two
+    draws are identical.  N(1, 0.3) puts 0.04 % of the channels at a negative BN scale (the parity
+    tests draw their own parameters with many more)."""
+    from paper_1911_08076_gb300 import synth
+    wl = synth.get("resnet18")
+    assert wl.seed == synth.SEED_BASE + wl.index
+    x, params = synth.draw_workload(wl)
+    x2, params2 = synth.draw_workload(wl)
+    assert np.array_equal(x, x2) and np.array_equal(params[0].w, params2[0].w)
+    counts = np.bincount(x.ravel(), minlength=4) / x.size
+    assert np.allclose(counts, 0.25, atol=0.002)
+    convs = [p for l, p in zip(wl.layers, params) if l.kind == "conv"]
+    w = np.concatenate([p.w.ravel() for p in convs])
+    assert set(np.unique(w)) == {-1, 1} and abs(w.mean()) < 0.002
+    cat = lambda f: np.concatenate([getattr(p, f) for p in convs]).astype(np.float64)
+    alpha, gamma, beta, mean, var = map(cat, ("alpha", "gamma", "beta", "mean", "var"))
+    assert alpha.min() >= 0.5 and alpha.max() <= 1.5 and abs(alpha.mean() - 1.0) < 0.03
+    assert abs(gamma.mean() - 1.0) < 0.03 and abs(gamma.std() - 0.3) < 0.02
+    assert (gamma < 0).mean() < 0.002                 # P(N(1, 0.3) < 0) = 0.0004
+    assert abs(beta.std() - 0.5) < 0.03 and abs(mean.std() - 2.0) < 0.1
+    assert var.min() >= 0.5 and var.max() <= 2.0
