@@ -242,3 +242,21 @@ ptxas info    : Compiling entry function '_ZN3ifq14conv_tc_kernelILi64ELi16ELi2E
     assert B.spilling_kernels(log) == ["_ZN3ifq14conv_tc_kernelILi128ELi16ELi2ELi2ELi1EEEv",
                                        "_ZN3ifq14conv_tc_kernelILi64ELi16ELi2ELi2ELi1EEEv"]
     assert B.spilling_kernels("") == []
+
+
+def test_graph_with_copies_validates_the_stack_before_any_capture():
+    """ifq_graph_create_io checks the stack (and a missing output handle) on the host first, like
+    ifq_graph_create (works without a GPU)."""
+    fake = 1 << 20
+    L0 = ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=-1, conv=ifq.conv_desc(1, 8, 8, 64, 32, 3, 1, 1), w_prep=fake,
+                   thr=fake, sign=fake, y_codes=fake)
+    L1 = ifq.Layer(kind=ifq.IFQ_LAYER_CONV, src=0, conv=ifq.conv_desc(1, 8, 8, 16, 32, 3, 1, 1), w_prep=fake,
+                   thr=fake, sign=fake, y_codes=fake)
+    with pytest.raises(ifq.IfqError) as e:   # layer 1 reads 16 channels, layer 0 writes 32
+        ifq.ifq_graph_create_io([L0, L1], fake, None, 0, fake, 1024, [None, fake], None, stream=0)
+    assert e.value.status == ifq.IFQ_ESHAPE
+    with pytest.raises(ifq.IfqError) as e:   # no input buffer
+        ifq.ifq_graph_create_io([L0], None, None, 0, fake, 1024, None, None, stream=0)
+    assert e.value.status == ifq.IFQ_EINVAL
+    arr = (ifq.Layer * 1)(L0)
+    assert ifq.lib().ifq_graph_create_io(arr, 1, fake, None, 0, None, 0, None, None, None, None) == ifq.IFQ_EINVAL
