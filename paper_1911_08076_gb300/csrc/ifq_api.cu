@@ -418,7 +418,7 @@ cudaError_t launch_tc_gb(int bn, int ks, const CUtensorMap& tm, const ConvArgs& 
 }
 
 // Bytes of packed codes per input pixel.
-int pixel_bytes(const ifq_conv_desc* d, const ConvGeom& g) { return g.cink * g.sbi / 8; }
+int pixel_bytes(const ifq_conv_desc*, const ConvGeom& g) { return g.cink * g.sbi / 8; }
 
 // Bytes of packed codes per gathered granule: the largest of 16, 8, 4, 1 that divides a pixel's
 // bytes (the persistent stack kernel has no 8-byte instance: 16, 4, 1 there).
