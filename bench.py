@@ -1,17 +1,26 @@
 #!/usr/bin/env python
 """Throughput benchmark of the quantized-substructure path on GB300.
 
-A step is one pass of the layer stack over one batch: for the default workload,
-the ResNet-18 body (16 3x3 + 3 1x1 binary x 2-bit convs, batch 32) through
-ifq_forward, replayed as a CUDA graph.  Inputs are seeded synthetic 2-bit codes
-already resident in HBM; L2 is flushed (a 256 MB write) between timed steps
-and the flush is outside the per-step CUDA events.  The end-to-end figure (`e2e`)
-replays a graph from ifq_graph_create_io that also copies the pinned host input
-in and every result out, one launch per step; `roofline` is the conv kernel's
-share of the step against the measured tensor peak, with the DRAM traffic of the
-committed ncu summary of the same workload and kernel source.
+A step is one pass of a layer stack over one batch through ifq_forward, replayed
+as a CUDA graph.  The headline workload is the largest single-GPU configuration:
+the 3x3 256->256 binary x 2-bit conv at 56x56, batch 256 (GEMM M = 802816,
+N = 256, K = 2304, 947 GOP).  The same JSON line carries a sub-record for every
+other configuration (the single PR1 layer, the ResNet-18 body b32, AlexNet
+conv2-FC7 b128, Tiny-YOLO and Tinier-YOLO b64 with fused pools, IFQ-Tinier-YOLO
+end to end from 8-bit pixels, the 1x1 512->512 layer b256), each with its step
+time, TOPS, images/s, roofline fraction, per-layer times, end-to-end figure and
+the oracle's CPU baseline.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload NAME]
+Inputs are seeded synthetic codes already resident in HBM; L2 is flushed (a
+256 MB write) between timed steps, outside the per-step CUDA events.  `e2e`
+replays a graph from ifq_graph_create_io that also copies the pinned host input
+in and every result out, one launch per step.  `roofline` is the conv kernel
+against the measured tensor peak (MEASURED_PEAKS.json bf16 x 2), with the DRAM
+traffic of the committed ncu summary of the same workload and kernel source;
+beside it, fractions against the e4m3 tcgen05 and the s8 mma.sync rates
+measured in the same process.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--workload NAME] [--no-sub]
 
 Rank 0 prints one JSON line.  Under torchrun each rank runs an independent
 replica (no data-path collective; a barrier and a max over ranks time the job).
@@ -21,6 +30,8 @@ of the same workload.
 from __future__ import annotations
 
 import argparse
+import ctypes
+import glob
 import hashlib
 import json
 import os
@@ -40,13 +51,15 @@ from paper_1911_08076_gb300 import synth  # noqa: E402
 
 METRIC = "binary×2-bit conv TOPS and images/s at 1 GB300; % of dense INT8 peak"
 UNIT = "TOPS"
-# mma.sync.m16n8k32 s8 rate measured on this machine's GB300 (sm_103a has no tcgen05 integer MMA);
-# see profiles/tensor_peaks_gb300.md.
-INT8_PEAK_TOPS = 151.4
+HEADLINE = "roofline3x3"
+SUB_WORKLOADS = ["pr1", "resnet18", "alexnet", "tinyyolo_fused", "tinieryolo_fused", "tinieryolo_full_fused",
+                 "roofline1x1"]
 FP8_PER_BF16 = 2.0          # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK_BF16_TFLOPS = 1900.0
 PROFILES = os.path.join(ROOT, "profiles")
 KERNEL_SRC = [os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", f) for f in ("conv_tc.cuh", "conv_common.cuh", "ptx.cuh")]
+RATES_SRC = os.path.join(ROOT, "bench_rates.cu")
+RATES_LIB = os.path.join(ROOT, "_build", "libbench_rates.so")
 
 
 def log(*a):
@@ -76,6 +89,19 @@ def alg_bytes(layer, batch, kbits=2):
     return inp + wts + thr + out
 
 
+def layer_alg_bytes(wl, li, batch):
+    """Algorithmic bytes of any layer of a stack: a conv as alg_bytes; a code pool reads its input
+    and writes its output once; a fixed-point output reads and writes one int32 per value."""
+    l = wl.layers[li]
+    if l.kind == "conv":
+        return alg_bytes(l, batch, wl.kbits)
+    cb = synth.field_bits(wl.kbits) / 8
+    if l.kind == "pool":
+        return batch * l.c * (l.h * l.w + l.ho * l.wo) * cb
+    s = wl.layers[l.src]
+    return 2 * 4 * batch * s.out_h * s.out_w * s.cout
+
+
 def read_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -99,8 +125,7 @@ def kernel_sha():
 def profiled_traffic(workload: str):
     """DRAM bytes per conv launch from the committed ncu summary of this workload, if it was taken
     on this kernel source (a summary names its `workload:` and `kernel_sha:`)."""
-    import glob
-    for path in sorted(glob.glob(os.path.join(PROFILES, "conv_tc_*.md"))):
+    for path in sorted(glob.glob(os.path.join(PROFILES, "*.md"))):
         try:
             txt = open(path).read()
         except OSError:
@@ -111,6 +136,44 @@ def profiled_traffic(workload: str):
         if wl and sha and tb and wl.group(1) == workload and sha.group(1) == kernel_sha():
             return float(tb.group(1))
     return None
+
+
+def build_rates(force: bool = False) -> str:
+    """Compile bench_rates.cu (the instruction-rate probes) into _build/libbench_rates.so."""
+    if not force and os.path.exists(RATES_LIB) and os.path.getmtime(RATES_LIB) >= os.path.getmtime(RATES_SRC):
+        return RATES_LIB
+    from paper_1911_08076_gb300 import build as B
+    os.makedirs(os.path.dirname(RATES_LIB), exist_ok=True)
+    tmp = RATES_LIB + f".{os.getpid()}.tmp"
+    nvcc = B._nvcc()
+    cudalib = os.path.join(os.path.dirname(os.path.dirname(nvcc)), "lib64")
+    subprocess.check_call([nvcc, *B.ARCH, "-O3", "-std=c++17", "-Xcompiler", "-fPIC", "-shared", "-cudart", "shared",
+                           RATES_SRC, "-Xlinker", f"-rpath={cudalib}", "-o", tmp])
+    os.replace(tmp, RATES_LIB)
+    return RATES_LIB
+
+
+def measure_rates(stream):
+    """Tensor rates measured now, on this GPU: tcgen05 e4m3 at N = 128 and 256 (the conv's
+    instruction) and mma.sync s8 (the dense INT8 path)."""
+    try:
+        L = ctypes.CDLL(build_rates())
+    except Exception as e:  # no nvcc or no library: report the reason, not a guess
+        return {"error": f"rate probes unavailable: {e}"}
+    dbl = ctypes.c_double
+    L.bench_tc_e4m3_tops.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.POINTER(dbl)]
+    L.bench_mma_s8_tops.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.POINTER(dbl)]
+    out = {}
+    for n in (128, 256):
+        v = dbl(0.0)
+        rc = L.bench_tc_e4m3_tops(n, 8192, 5, ctypes.c_void_p(stream.cuda_stream), ctypes.byref(v))
+        out[f"tcgen05_e4m3_n{n}_tops"] = v.value if rc == 0 else None
+    v = dbl(0.0)
+    rc = L.bench_mma_s8_tops(4096, 3, ctypes.c_void_p(stream.cuda_stream), ctypes.byref(v))
+    out["mma_sync_s8_tops"] = v.value if rc == 0 else None
+    out["how"] = ("same process, before the timed regions: one CTA per SM issuing M128xNxK32 e4m3 tcgen05 MMAs "
+                  "back to back; 4 CTAs x 8 warps per SM issuing m16n8k32 s8 mma.sync; 2 ops per MAC")
+    return out
 
 
 class ClockSampler:
@@ -166,23 +229,36 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def cpu_baseline(wl, x, params):
-    """The oracle as it stands (float and integer chains, naive loops) on the host cores, over the
-    whole batch of the workload, images split across threads."""
+def line_config(wl, args):
+    """The `config` object of both arms' JSON lines (identical for the same workload)."""
+    convs = [l for l in wl.layers if l.kind == "conv"]
+    return {"workload": wl.name, "batch_per_gpu": wl.batch, "layers": len(wl.layers),
+            "ops_per_step": sum(conv_ops(l, wl.batch) for l in convs),
+            "parallelism": f"replicas x{args.gpus}" if args.gpus > 1 else "single GPU",
+            "l2": "flushed between steps (256 MB write outside the step events)", "path": args.path}
+
+
+def cpu_baseline(wl, x, params, seconds: float):
+    """The oracle as it stands (float and integer chains, naive loops) on the host cores, on whole
+    images of the workload, images split across threads: as many images as fit in about
+    `seconds` of host time (at least one), scaled to the workload's metric."""
     from oracle import oracle as O
     O.build()
     threads = len(os.sched_getaffinity(0))
-    n = wl.batch
-    passes, dt = 0, 0.0
-    while passes == 0 or (dt < 10.0 and passes < 50):   # about 10 s of host work, at most 50 passes
+    per_img = sum(conv_ops(l, 1) for l in wl.layers if l.kind == "conv")
+    n_done, dt, n = 0, 0.0, 1
+    while dt < seconds and n_done < wl.batch:
+        n = min(n, wl.batch - n_done)
         t0 = time.perf_counter()
-        O.forward(wl, x[:n], params, images=list(range(n)), threads=threads)
+        O.forward(wl, x[n_done:n_done + n], params, threads=threads)
         dt += time.perf_counter() - t0
-        passes += 1
-    ops = passes * sum(conv_ops(l, n) for l in wl.layers if l.kind == "conv")
+        n_done += n
+        rate = n_done / dt if dt > 0 else 1.0
+        n = max(1, min(4 * n, int(rate * max(seconds - dt, 0.0))))
+    ops = n_done * per_img
     return {"value": ops / dt / 1e12, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"{passes} passes of all {n} images of the batch through all {len(wl.layers)} layers, "
-                      f"float and integer chains, {dt:.2f} s wall", "images_per_s": passes * n / dt}
+            "sample": f"{n_done} of the {wl.batch} images of the batch through all {len(wl.layers)} layers, "
+                      f"float and integer chains, {dt:.2f} s wall", "images_per_s": n_done / dt}
 
 
 def run_reference(args):
@@ -196,7 +272,7 @@ def run_reference(args):
     from oracle import oracle as O
     O.build()
     wl = synth.get(args.workload, args.batch)
-    x, params = synth.draw_workload(wl)
+    x, params = synth.draw_workload(wl, batch=1)
     outs = O.forward(wl, x, params, images=[0], check_float=False)
     convs = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
     threads = len(os.sched_getaffinity(0))
@@ -244,12 +320,10 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32 (naive loops) + f64",
-            "data": "synthetic",
-            "config": {"workload": wl.name, "batch": wl.batch,
-                       "sample": "per step: a slice of the output channels of one conv layer for one image"},
+            "data": "synthetic", "config": line_config(wl, args),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                             "sample": f"{args.steps} steps of one conv layer's channel slice for image 0 "
-                                       f"(cycling over {len(convs)} layers), both chains"},
+                             "sample": f"each of {args.steps} steps: a slice of the output channels of one conv "
+                                       f"layer for image 0 (cycling over {len(convs)} layers), both chains"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -257,7 +331,7 @@ def run_reference(args):
 POOL_HBM_SHAPE = (512, 208, 208, 32)   # Tiny-YOLO pool2 (2x2 / 2 on 208x208x32 codes) at batch 512
 
 
-def measure_pool_hbm(ifq, torch, dev, stream, flush, reps=20):
+def measure_pool_hbm(ifq, torch, dev, stream, reps=20):
     """HBM throughput of the code max-pool (an HBM-bound step of the path) on a map larger than L2:
     2x2 / stride 2 on 512 x 208 x 208 x 32 packed 2-bit codes (177 MB in, 44 MB out), channel
     signs with negatives.  Launches back to back, each between CUDA events; the input is larger
@@ -307,27 +381,32 @@ def job_throughput(ops_per_rank_step: float, world: int, step_ms_max: float) -> 
     return world * ops_per_rank_step / (step_ms_max * 1e-3) / 1e12
 
 
-def run_ours(args):
-    import torch
-    import torch.distributed as dist
+PATH_NAMES = {0: "auto", 1: "conv_tc_kernel", 2: "bitserial", 3: "conv_direct_kernel"}
 
-    from paper_1911_08076_gb300 import ifq
+
+def kernel_of(ifq, st, li):
+    """Name of the kernel family a layer launches (the planner's choice for convs)."""
+    rec = st.layers[li]
+    if rec.kind == ifq.IFQ_LAYER_CONV:
+        p = ifq.ifq_conv_plan(rec.conv)
+        if p == ifq.IFQ_PATH_BITSERIAL:
+            l = st.wl.layers[li]
+            narrow = l.kind == "conv" and l.cin in (4, 8, 16) and l.k == 3 and l.stride == 1 and l.cout <= 32
+            return "conv_bitserial_narrow_kernel" if narrow else "conv_bitserial_kernel"
+        return PATH_NAMES.get(p, str(p))
+    if rec.kind == ifq.IFQ_LAYER_POOL:
+        return "maxpool_codes"
+    return "fixed_output_kernel"
+
+
+def measure_workload(name, args, ifq, torch, dev, stream, flush, K, W, world, barrier, max_over_ranks,
+                     peaks, e2e_separate=False, clocks=False):
+    """Time one workload: K graph replays of the step (L2 flushed between steps, outside the
+    step events), per-launch durations from a graph with external event nodes, the end-to-end
+    step through ifq_graph_create_io from pinned host buffers, and the per-layer roofline.
+    Returns (record, workload, inputs, params)."""
     from paper_1911_08076_gb300.stack import DeviceStack
-
-    rank, world, local = dist_info()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
-    def max_over_ranks(v):
-        return reduce_max(v, world, dev)
-
-    wl = synth.get(args.workload, args.batch)
+    wl = synth.get(name, args.batch if name == args.workload else None)
     B = wl.batch
     x, params = synth.draw_workload(wl)
     path = {"auto": ifq.IFQ_PATH_AUTO, "tc": ifq.IFQ_PATH_TC, "bitserial": ifq.IFQ_PATH_BITSERIAL}[args.path]
@@ -335,26 +414,22 @@ def run_ours(args):
     x_host = torch.from_numpy(synth.pack_codes(x, 8 if wl.in_bits == 8 else wl.kbits)).pin_memory()
     xd = st.input_buffer()
     xd.copy_(x_host)
-    stream = torch.cuda.Stream(device=dev)
     torch.cuda.synchronize()
     st.capture(xd, stream)
-    n_kernels = len(wl.layers)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
     convs = [l for l in wl.layers if l.kind == "conv"]
     ops = sum(conv_ops(l, B) for l in convs)
-    K, W = args.steps, args.warmup
-
+    rec = {"workload": wl.name, "batch": B, "layers": len(wl.layers), "ops_per_step": ops}
+    sampler = None
     with torch.cuda.stream(stream):
-        # ---------------- timed region: graph replays, L2 flushed between steps
         for i in range(W):
             st.replay(stream)
             flush.fill_(i & 0xFF)
         torch.cuda.synchronize()
         starts = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
         ends = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
-        gid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
-        sampler = ClockSampler(gid)
-        sampler.start()
+        if clocks:
+            sampler = ClockSampler("GPU-" + str(torch.cuda.get_device_properties(dev).uuid))
+            sampler.start()
         barrier()
         torch.cuda.synchronize()
         wall0 = time.perf_counter()
@@ -366,16 +441,16 @@ def run_ours(args):
         torch.cuda.synchronize()
         wall = time.perf_counter() - wall0
         barrier()
-        clocks = sampler.stop()
-        step_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / K
-        step_ms = max_over_ranks(step_ms)
+        if sampler is not None:
+            rec["clocks"] = sampler.stop()
+        step_ms = max_over_ranks(sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / K)
         status = ifq.ifq_device_status(stream)
         if status != ifq.IFQ_OK:
-            raise RuntimeError(f"device status after timed region: {ifq.ifq_status_str(status)}")
+            raise RuntimeError(f"{wl.name}: device status after timed region: {ifq.ifq_status_str(status)}")
 
-        # ---------------- per-launch durations: the step's launches captured in a graph with an
-        # external event record node around each kernel, replayed with an L2 flush before each step
-        KR = min(K, 300)
+        # per-launch durations: the step's launches captured in a graph with an external event
+        # record node around each kernel, replayed with an L2 flush before each step
+        KR = max(3, min(K, 300))
         try:
             ev = [(torch.cuda.Event(enable_timing=True, external=True),
                    torch.cuda.Event(enable_timing=True, external=True)) for _ in wl.layers]
@@ -405,22 +480,17 @@ def run_ours(args):
             torch.cuda.synchronize()
             per_layer_ms = [sum(evl[i][li][0].elapsed_time(evl[i][li][1]) for i in range(KR)) / KR
                             for li in range(len(wl.layers))]
-        conv_idx = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
-        conv_ms = sum(per_layer_ms[i] for i in conv_idx)
-        conv_ops_total = sum(conv_ops(wl.layers[i], B) for i in conv_idx)
-        conv_bytes_total = sum(alg_bytes(wl.layers[i], B, wl.kbits) for i in conv_idx)
 
-        # ---------------- end to end through the C ABI with host buffers: one graph launch per step
-        # that copies the pinned host input in first and every result (the leaf layers' outputs) out
-        # right after its layer (ifq_graph_create_io); the shortcut results leave while the main
-        # chain still runs
+        # end to end through the C ABI with host buffers: one graph launch per step that copies the
+        # pinned host input in first and every result (the leaf layers' outputs) out right after its
+        # layer (ifq_graph_create_io)
         leaf_host = torch.empty(st.leaf_block.shape, dtype=torch.uint8).pin_memory()
         h2d = x_host.numel() * x_host.element_size()
         d2h = sum(n for _, n in st.leaf_spans())
-        KE = min(K, 1000)
+        KE = max(3, min(K, 1000))
 
         def timed_steps(step):
-            for i in range(min(W, 20)):
+            for i in range(max(3, min(W, 20))):
                 step()
             torch.cuda.synchronize()
             barrier()
@@ -437,65 +507,142 @@ def run_ours(args):
         st.capture_io(xd, x_host, leaf_host, stream)
         e2e_ms = timed_steps(lambda: st.replay(stream))
         if not st.leaf_results_equal(leaf_host):
-            raise RuntimeError("end-to-end results differ from the device results")
-        # the same copies as three launches per step (input copy, step graph, result copy)
-        st.capture(xd, stream)
-        e2e_sep_ms = timed_steps(lambda: (ifq.ifq_copy_bytes(xd, x_host, h2d, stream), st.replay(stream),
-                                          ifq.ifq_copy_bytes(leaf_host, st.leaf_block, leaf_host.numel(), stream)))
+            raise RuntimeError(f"{wl.name}: end-to-end results differ from the device results")
+        e2e = {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+               "sequence": "per step (L2 flushed, untimed, between steps): one graph launch that copies the "
+                           "pinned input in, runs the step and copies each result out after its layer"}
+        if e2e_separate:
+            st.capture(xd, stream)
+            e2e_sep_ms = timed_steps(lambda: (ifq.ifq_copy_bytes(xd, x_host, h2d, stream), st.replay(stream),
+                                              ifq.ifq_copy_bytes(leaf_host, st.leaf_block, leaf_host.numel(), stream)))
+            e2e["separate_copies"] = {"value": world * ops / (e2e_sep_ms * 1e-3) / 1e12, "unit": UNIT,
+                                      "ms_per_step": e2e_sep_ms,
+                                      "sequence": "input copy, step graph, result copy: three launches"}
 
-    pool_hbm = measure_pool_hbm(ifq, torch, dev, stream, flush)
-    value = job_throughput(ops, world, step_ms)
-    imgs = world * B / (step_ms * 1e-3)
-    bf16, bf16_sus, hbm, src = read_peaks()
-    peak = bf16 * FP8_PER_BF16
-    # The dominant kernel's launch duration inside the timed region: the step's launches run back to
-    # back (programmatic dependent launch overlaps each one's prologue with its predecessor's tail),
-    # so a conv launch's in-step duration is the step time times the conv share of the step (from
-    # the serialised per-launch pass), divided by the conv launches per step.
+    # per-layer roofline: each launch timed alone against the tensor peak and the HBM copy rate
+    peak, hbm = peaks["tensor_tops"], peaks["hbm_gbs"]
+    layers = []
+    for li, l in enumerate(wl.layers):
+        us = 1e3 * per_layer_ms[li]
+        b = layer_alg_bytes(wl, li, B)
+        o = conv_ops(l, B) if l.kind == "conv" else 0.0
+        t_tensor = o / (peak * 1e12) * 1e6
+        t_hbm = b / (hbm * 1e9) * 1e6
+        bound = "tensor" if t_tensor >= t_hbm else "hbm"
+        layers.append({"name": l.name, "kernel": kernel_of(ifq, st, li), "us": round(us, 3),
+                       "gop": round(o / 1e9, 4), "alg_mb": round(b / 1e6, 4),
+                       "tops": round(o / (us * 1e-6) / 1e12, 2) if us > 0 else None,
+                       "alg_gbs": round(b / (us * 1e-6) / 1e9, 1) if us > 0 else None,
+                       "bound": bound, "roofline_us": round(max(t_tensor, t_hbm), 3),
+                       "frac": round(max(t_tensor, t_hbm) / us, 4) if us > 0 else None})
+    conv_idx = [i for i, l in enumerate(wl.layers) if l.kind == "conv"]
+    conv_ms = sum(per_layer_ms[i] for i in conv_idx)
     total_ms = sum(per_layer_ms)
     conv_share = conv_ms / total_ms if total_ms > 0 else 1.0
+    # A conv launch's in-step duration: the step's launches run back to back (programmatic dependent
+    # launch overlaps each one's prologue with its predecessor's tail), so the convs' share of the
+    # step time (from the serialised per-launch pass), divided by the conv launches per step.
     conv_in_step_ms = step_ms * conv_share
-    achieved = conv_ops_total / (conv_in_step_ms * 1e-3) / 1e12
-    achieved_serial = conv_ops_total / (conv_ms * 1e-3) / 1e12
-    traffic = profiled_traffic(wl.name)
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
-        "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": f"e4m3xe4m3->f32 (exact integer: u{wl.kbits} codes x +-1 signs)", "data": "synthetic",
-        "config": {"workload": wl.name, "batch_per_gpu": B, "layers": len(wl.layers),
-                   "ops_per_step": ops, "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "l2": "flushed between steps (256 MB write outside the step events)",
-                   "path": args.path},
-        "images_per_s": imgs,
-        "pct_of_int8_peak": 100.0 * value / (world * INT8_PEAK_TOPS),
-        "int8_peak_tops": INT8_PEAK_TOPS,
+    achieved = ops / (conv_in_step_ms * 1e-3) / 1e12
+    achieved_serial = ops / (conv_ms * 1e-3) / 1e12
+    rec.update({
+        "ms_per_step": step_ms, "value": job_throughput(ops, world, step_ms), "unit": UNIT,
+        "images_per_s": world * B / (step_ms * 1e-3),
         "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                     "frac": achieved / peak, "traffic": traffic,
-                     "kernel": "conv_tc_kernel (all conv launches of a step)",
-                     "peak_source": f"{src} bf16 burst {bf16} x {FP8_PER_BF16} (fp8/bf16 nominal)",
-                     "algorithmic_bytes_per_launch": conv_bytes_total / len(conv_idx),
-                     "ops_per_launch": conv_ops_total / len(conv_idx),
+                     "frac": achieved / peak, "traffic": profiled_traffic(wl.name),
+                     "kernel": "conv launches of a step" if len(conv_idx) > 1 else layers[conv_idx[0]]["kernel"],
+                     "peak_source": peaks["tensor_source"],
+                     "algorithmic_bytes_per_launch": sum(layer_alg_bytes(wl, i, B) for i in conv_idx) / len(conv_idx),
+                     "ops_per_launch": ops / len(conv_idx),
                      "avg_launch_us": 1e3 * conv_in_step_ms / len(conv_idx),
                      "timing": "timed region: step time x conv share / conv launches per step",
                      "serialized": {"achieved": achieved_serial, "frac": achieved_serial / peak,
                                     "avg_launch_us": 1e3 * conv_ms / len(conv_idx),
                                     "timing": f"each launch alone between CUDA events ({timing_mode})"}},
-        "e2e": {"value": world * ops / (e2e_ms * 1e-3) / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-                "sequence": "per step (L2 flushed, untimed, between steps): one graph launch that copies the "
-                            "pinned input in, runs the step and copies each result out after its layer",
-                "separate_copies": {"value": world * ops / (e2e_sep_ms * 1e-3) / 1e12, "unit": UNIT,
-                                    "ms_per_step": e2e_sep_ms,
-                                    "sequence": "input copy, step graph, result copy: three launches"}},
-        "pool_hbm": pool_hbm,
-        "gpu_launches": K * n_kernels,
-        "clocks": clocks,
-        "timed_wall_s": wall,
-    }
-    log("per-layer us:", ", ".join(f"{l.name}={1e3 * t:.2f}" for l, t in zip(wl.layers, per_layer_ms)))
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, x, params)
+        "e2e": e2e, "gpu_launches": K * len(wl.layers), "timed_wall_s": wall, "layers_timed_alone": layers,
+    })
+    log(f"{wl.name}: {step_ms * 1e3:.2f} us/step, {rec['value']:.1f} TOPS; per-layer us: " +
+        ", ".join(f"{l['name']}={l['us']:.2f}" for l in layers))
     st.release()
+    del st, xd
+    torch.cuda.empty_cache()
+    return rec, wl, x, params
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_1911_08076_gb300 import ifq
+
+    rank, world, local = dist_info()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(v):
+        return reduce_max(v, world, dev)
+
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    bf16, bf16_sus, hbm, src = read_peaks()
+    peaks = {"tensor_tops": bf16 * FP8_PER_BF16, "hbm_gbs": hbm,
+             "tensor_source": f"{src} bf16 burst {bf16} x {FP8_PER_BF16} (fp8/bf16 nominal)"}
+    rates = measure_rates(stream)
+    K, W = args.steps, args.warmup
+
+    head, wl, x, params = measure_workload(args.workload, args, ifq, torch, dev, stream, flush, K, W, world,
+                                           barrier, max_over_ranks, peaks, e2e_separate=True, clocks=True)
+    value = head["value"]
+    r = head["roofline"]
+    ach = r["achieved"]
+
+    def frac(v):
+        return ach / v if v else None
+
+    r["vs_measured_rates"] = {
+        "tcgen05_e4m3_n128": frac(rates.get("tcgen05_e4m3_n128_tops")),
+        "tcgen05_e4m3_n256": frac(rates.get("tcgen05_e4m3_n256_tops")),
+        "note": "achieved / the e4m3 tcgen05 rate measured in this process (the conv's own instruction)"}
+    s8 = rates.get("mma_sync_s8_tops")
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": f"e4m3xe4m3->f32 (exact integer: u{wl.kbits} codes x +-1 signs)", "data": "synthetic",
+        "config": line_config(wl, args),
+        "images_per_s": head["images_per_s"],
+        "pct_of_int8_peak": 100.0 * value / (world * s8) if s8 else None,
+        "int8_peak": {"tops": s8, "source": "mma.sync.m16n8k32 s8 rate measured in this process (sm_103a has no "
+                                            "tcgen05 integer MMA; the exact binary x 2-bit product runs on e4m3)"},
+        "rates_measured": rates,
+        "roofline": r,
+        "e2e": head["e2e"],
+        "gpu_launches": head["gpu_launches"],
+        "clocks": head.get("clocks"),
+        "timed_wall_s": head["timed_wall_s"],
+        "layers_timed_alone": head["layers_timed_alone"],
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, x, params, 12.0)
+    del x, params
+    subs = {}
+    if not args.no_sub:
+        for name in SUB_WORKLOADS:
+            if name == args.workload:
+                continue
+            rec, swl, sx, sp = measure_workload(name, args, ifq, torch, dev, stream, flush, K, W, world, barrier,
+                                                max_over_ranks, peaks)
+            if rank == 0 and world == 1 and not args.no_cpu_baseline:
+                rec["cpu_baseline"] = cpu_baseline(swl, sx, sp, 3.0)
+            subs[name] = rec
+    line["configs"] = subs
+    line["pool_hbm"] = measure_pool_hbm(ifq, torch, dev, stream)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -505,13 +652,14 @@ def run_ours(args):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=3000)
-    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="resnet18", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--workload", default=HEADLINE, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--path", default="auto", choices=["auto", "tc", "bitserial"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sub", action="store_true", help="time the headline workload only")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")

@@ -367,7 +367,10 @@ int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, s
  * should come before any stream capture.  All calls on one device share the
  * array, so calls whose executions overlap in time (on other streams or from
  * other host threads) race on it and must be serialised by the caller.
- * Results are identical to ifq_forward's.
+ * The looked-up address is kept for the life of the process: after
+ * cudaDeviceReset (or anything else that destroys the device's primary
+ * context) it is stale, so a process that resets a device must not call this
+ * entry point on that device again.  Results are identical to ifq_forward's.
  */
 int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, void* stream);
 

@@ -39,6 +39,10 @@ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 inline size_t round_up(size_t a, size_t b) { return (a + b - 1) / b * b; }
 inline cudaStream_t S(void* s) { return (cudaStream_t)s; }
 
+// Guards the per-device state below (kernel attributes, SM count, occupancy lookups, the address
+// of the no-allocation scratch array).
+std::mutex g_dev_mu;
+
 // ---------------------------------------------------------------- driver entry point for TMA descriptors
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -117,10 +121,15 @@ struct TcInst {
   static cudaError_t set_attr() {
     return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
   }
-  // clusters of this instance that fit on the device at once (0: none)
+  // clusters of this instance that fit on the current device at once (0: none), looked up once per
+  // device under the device-state lock
   static int max_clusters(int nsm) {
-    static int cached = -1;
-    if (cached < 0) {
+    static int cached[kMaxDevices];
+    static bool known[kMaxDevices];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    if (!known[dev]) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3((unsigned)(nsm / KS * KS));
       cfg.blockDim = dim3(kConvThreads);
@@ -133,10 +142,11 @@ struct TcInst {
       cfg.attrs = at;
       cfg.numAttrs = 1;
       int n = 0;
-      cached = cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess ? n : 0;
+      cached[dev] = cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess ? n : 0;
       cudaGetLastError();
+      known[dev] = true;
     }
-    return cached;
+    return cached[dev];
   }
   static cudaError_t launch(const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
     if constexpr (KS == 1) {
@@ -175,7 +185,6 @@ struct DevState {
   bool stack_ok = false;   // the stack kernel fits one CTA per SM (cooperative launch possible)
 };
 DevState g_dev[kMaxDevices];
-std::mutex g_dev_mu;
 
 // Per-device one-time setup (shared-memory limits of the kernels, SM count).
 int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {

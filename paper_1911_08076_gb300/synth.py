@@ -331,11 +331,25 @@ def draw_codes(rng: np.random.Generator, shape, kbits: int = 2) -> np.ndarray:
 PIXEL_STEP = 1.0 / 255.0   # input step of a layer on 8-bit image values (pixels scaled to [0, 1])
 
 
-def draw_workload(wl: Workload, batch: Optional[int] = None):
+NEG_GAMMA_SEED = 77   # offset of the generator that picks the channels whose BN scale is negated
+
+
+def draw_workload(wl: Workload, batch: Optional[int] = None, neg_gamma: float = 0.0):
     """Input [B][H][W][C] (uint8: k-bit codes, or 8-bit pixels with a zero 4th channel for an image
-    input) and per-layer ConvParams (None for pools and fixed-point outputs)."""
+    input) and per-layer ConvParams (None for pools and fixed-point outputs).
+
+    neg_gamma > 0: after the standard draw, each channel's BN scale gamma is negated with that
+    probability, picked by a second generator (seed + NEG_GAMMA_SEED), so every other value equals
+    the standard draw's.  The configurations call for about 10 % of channels with a negative BN
+    scale, which gamma ~ N(1, 0.3) alone gives only 0.04 % of the time."""
     rng = np.random.default_rng(wl.seed)
     params = [draw_conv_params(rng, l) if l.kind == "conv" else None for l in wl.layers]
+    if neg_gamma > 0:
+        flip = np.random.default_rng(wl.seed + NEG_GAMMA_SEED)
+        for p in params:
+            if p is not None:
+                neg = flip.random(p.gamma.shape[0]) < neg_gamma
+                p.gamma = np.where(neg, -np.abs(p.gamma), np.abs(p.gamma)).astype(np.float32)
     for l, p in zip(wl.layers, params):
         if l.kind == "conv" and l.in_bits == 8:
             p.delta_in = PIXEL_STEP

@@ -4,6 +4,7 @@ fixed-point output of the detection conv (Sec. 2.2), alone and in the whole IFQ-
 import numpy as np
 import pytest
 import torch
+from stack_parity import compare_stack_with_oracle
 
 from oracle import oracle as O
 from paper_1911_08076_gb300 import ifq, synth
@@ -88,24 +89,11 @@ def test_fixed_output_matches_oracle(m):
     assert (y.cpu().numpy() == O.fixed_output(A, p, m)).all()
 
 
-@pytest.mark.parametrize("name", ["tinieryolo_full", "tinieryolo_full_fused"])
-def test_tinier_yolo_full_matches_oracle(name):
-    """The whole IFQ-Tinier-YOLO stack from 8-bit pixels to fixed-point detection outputs; the oracle
-    recomputes the first and last image through every layer."""
-    wl = synth.get(name, 3)
+@pytest.mark.parametrize("name,batch", [("tinieryolo_full", 3), ("tinieryolo_full", 64)])
+def test_tinier_yolo_full_matches_oracle(name, batch):
+    """The whole IFQ-Tinier-YOLO stack with separate pool launches from 8-bit pixels to fixed-point
+    detection outputs (the fused form is in the full-size workload tests); the oracle recomputes
+    every image through every layer."""
+    wl = synth.get(name, batch)
     x, params = synth.draw_workload(wl)
-    st = DeviceStack(wl, params)
-    xd = st.input_buffer()
-    xd.copy_(torch.from_numpy(synth.pack_codes(x, 8)))
-    st.forward(xd)
-    torch.cuda.synchronize()
-    assert ifq.ifq_device_status() == ifq.IFQ_OK
-    imgs = [0, 2]
-    ref = O.forward(wl, x, params, images=imgs)
-    for li, l in enumerate(wl.layers):
-        out = st.output(li)
-        if l.kind == "fixed" or (l.kind == "conv" and l.out == "acc"):
-            assert (out["acc"][imgs] == ref[li]).all(), l.name
-        else:
-            c = l.cout if l.kind == "conv" else l.c
-            assert (synth.unpack_codes(out["codes"][imgs], c) == ref[li]).all(), l.name
+    compare_stack_with_oracle(wl, x, params)

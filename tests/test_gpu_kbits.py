@@ -5,6 +5,7 @@ largest admitted magnitude, and whole k-bit stacks."""
 import numpy as np
 import pytest
 import torch
+from stack_parity import compare_stack_with_oracle
 
 from oracle import oracle as O
 from paper_1911_08076_gb300 import ifq, synth
@@ -209,26 +210,9 @@ def test_tc_accumulation_exact_at_the_admitted_bound(kbits, K):
     assert (codes.reshape(B, cout) == O.int_chain(A.astype(np.int32), *O.fold(prm, K))).all()
 
 
-@pytest.mark.parametrize("name,batch", [("alexnet_k3", 16), ("alexnet_k4", 16), ("resnet18_k4", 8),
-                                        ("tinyyolo_fused_k4", 4)])
-def test_kbit_workload_matches_oracle(name, batch):
-    """Whole k-bit stacks through ifq_forward; the oracle recomputes the first and last image."""
-    wl = synth.get(name, batch)
+@pytest.mark.parametrize("name", ["alexnet_k3", "alexnet_k4", "resnet18_k4", "tinyyolo_fused_k4"])
+def test_kbit_workload_matches_oracle(name):
+    """Whole k-bit stacks at full size through ifq_forward; the oracle recomputes every image."""
+    wl = synth.get(name)
     x, params = synth.draw_workload(wl)
-    st = DeviceStack(wl, params)
-    xd = torch.from_numpy(synth.pack_codes(x, wl.kbits)).to(DEV)
-    st.forward(xd)
-    torch.cuda.synchronize()
-    assert ifq.ifq_device_status() == ifq.IFQ_OK
-    imgs = [0, batch - 1]
-    ref = O.forward(wl, x, params, images=imgs)
-    for li, l in enumerate(wl.layers):
-        out = st.output(li)
-        r = ref[li]
-        if l.kind == "conv" and l.out == "acc":
-            assert (out["acc"][imgs] == r).all(), l.name
-        elif l.kind == "conv" and l.out == "both":
-            assert (synth.unpack_codes(out["codes"][imgs], l.cout, wl.kbits) == r["codes"]).all(), l.name
-        else:
-            c = l.cout if l.kind == "conv" else l.c
-            assert (synth.unpack_codes(out["codes"][imgs], c, wl.kbits) == r).all(), l.name
+    compare_stack_with_oracle(wl, x, params)

@@ -14,6 +14,7 @@ import torch
 from oracle import oracle as O
 from paper_1911_08076_gb300 import ifq, synth
 from paper_1911_08076_gb300.stack import DeviceStack
+from stack_parity import compare_stack_with_oracle
 
 pytestmark = [pytest.mark.gpu,
               pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
@@ -254,33 +255,31 @@ def test_pack_helpers_match_formats():
 
 # ----------------------------------------------------------------------------- whole workloads
 
-WORKLOADS = ["pr1", "resnet18", "alexnet", "tinyyolo", "tinieryolo", "roofline3x3", "roofline1x1"]
+# Every configuration at full size: the single PR1 layer, the ResNet-18 body b32, AlexNet conv2-FC7
+# b128, Tiny-YOLO and Tinier-YOLO b64 (separate and fused pools; Tinier also end to end from 8-bit
+# pixels to fixed-point detections), and the two roofline layers b256.
+WORKLOADS = ["pr1", "resnet18", "alexnet", "tinyyolo", "tinyyolo_fused", "tinieryolo", "tinieryolo_fused",
+             "tinieryolo_full_fused", "roofline3x3", "roofline1x1"]
 
 
 @pytest.mark.parametrize("name", WORKLOADS)
 def test_workload_matches_oracle(name):
-    """Full-size workload on the GPU; the oracle recomputes the first and last image through
-    every layer (all images for the single-image workload)."""
+    """Full-size workload on the GPU; the oracle recomputes every image through every layer."""
     wl = synth.get(name)
     x, params = synth.draw_workload(wl)
-    st = DeviceStack(wl, params)
-    xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
-    st.forward(xd)
-    torch.cuda.synchronize()
-    assert ifq.ifq_device_status() == ifq.IFQ_OK
-    imgs = [0] if wl.batch == 1 else [0, wl.batch - 1]
-    ref = O.forward(wl, x, params, images=imgs)
-    for li, l in enumerate(wl.layers):
-        out = st.output(li)
-        r = ref[li]
-        if l.kind == "conv" and l.out == "both":
-            assert (synth.unpack_codes(out["codes"][imgs], l.cout) == r["codes"]).all(), l.name
-            assert (out["acc"][imgs] == r["acc"]).all(), l.name
-        elif l.kind == "conv" and l.out == "acc":
-            assert (out["acc"][imgs] == r).all(), l.name
-        else:
-            c = l.cout if l.kind == "conv" else l.c
-            assert (synth.unpack_codes(out["codes"][imgs], c) == r).all(), l.name
+    compare_stack_with_oracle(wl, x, params)
+
+
+@pytest.mark.parametrize("name", WORKLOADS)
+def test_workload_with_negative_bn_scales_matches_oracle(name):
+    """The same full-size workloads with about 10 % of channels drawn with a negative BN scale (the
+    sign-flipped thresholds of Eq. (7) and the min-pool of those channels), every image."""
+    wl = synth.get(name)
+    x, params = synth.draw_workload(wl, neg_gamma=0.1)
+    negs = sum(int((p.gamma < 0).sum()) for p in params if p is not None)
+    chans = sum(p.gamma.shape[0] for p in params if p is not None)
+    assert 0.05 * chans <= negs <= 0.2 * chans or chans < 100, (negs, chans)
+    compare_stack_with_oracle(wl, x, params)
 
 
 @pytest.mark.parametrize("persistent", ["0", "1"], ids=["per_layer", "persistent"])
