@@ -375,6 +375,18 @@ int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, s
 int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, void* stream);
 
 /*
+ * ifq_last_forward_mode -- how the calling host thread's last successful
+ * ifq_forward or ifq_forward_noalloc call ran its stack: IFQ_FORWARD_LAYERS
+ * (one launch per layer) or IFQ_FORWARD_PERSISTENT (the whole stack as one
+ * persistent launch).  The paper has no counterpart; this is a diagnostic for
+ * callers and tests that need to know which launch served a request (results
+ * are identical either way).  Host only, thread-local; IFQ_EINVAL if `mode` is
+ * NULL or the thread has made no successful forward call.
+ */
+enum { IFQ_FORWARD_LAYERS = 1, IFQ_FORWARD_PERSISTENT = 2 };
+int ifq_last_forward_mode(int* mode);
+
+/*
  * CUDA-graph form of ifq_forward: ifq_graph_create captures the launches of
  * ifq_forward(layers, nlayers, x, ws, ws_bytes) on `stream` into a graph that
  * ifq_graph_launch replays on any stream with the same buffers.  The graph is

@@ -931,6 +931,14 @@ int noalloc_counters(void** out) {
   return IFQ_OK;
 }
 
+// Launch mode of this host thread's last successful ifq_forward / ifq_forward_noalloc (0: none yet).
+thread_local int t_last_forward = 0;
+
+int note_forward(int rc, int mode) {
+  if (rc == IFQ_OK) t_last_forward = mode;
+  return rc;
+}
+
 int run_layer(const ifq_layer* layers, int i, const void* x, cudaStream_t st) {
   const ifq_layer& l = layers[i];
   const void* in = l.src < 0 ? x : layers[l.src].y_codes;
@@ -1183,21 +1191,28 @@ int ifq_forward(const ifq_layer* layers, int nlayers, const void* x, void* ws, s
   int rc = check_stack(layers, nlayers, x);
   if (rc) return rc;
   rc = run_stack_kernel(layers, nlayers, x, ws, ws_bytes, S(stream));
-  if (rc != IFQ_EUNSUPPORTED) return rc;
-  return run_stack(layers, nlayers, x, S(stream));
+  if (rc != IFQ_EUNSUPPORTED) return note_forward(rc, IFQ_FORWARD_PERSISTENT);
+  return note_forward(run_stack(layers, nlayers, x, S(stream)), IFQ_FORWARD_LAYERS);
 }
 
 int ifq_forward_noalloc(const ifq_layer* layers, int nlayers, const void* x, void* stream) {
   int rc = check_stack(layers, nlayers, x);
   if (rc) return rc;
   size_t need = 0;
-  if (!stack_eligible(layers, nlayers, &need)) return run_stack(layers, nlayers, x, S(stream));
+  if (!stack_eligible(layers, nlayers, &need))
+    return note_forward(run_stack(layers, nlayers, x, S(stream)), IFQ_FORWARD_LAYERS);
   if (need > kNoallocCounterBytes) return IFQ_EWORKSPACE;
   void* ws = nullptr;
   if ((rc = noalloc_counters(&ws))) return rc;
   rc = launch_stack_kernel(layers, nlayers, x, ws, need, S(stream));
-  if (rc != IFQ_EUNSUPPORTED) return rc;
-  return run_stack(layers, nlayers, x, S(stream));
+  if (rc != IFQ_EUNSUPPORTED) return note_forward(rc, IFQ_FORWARD_PERSISTENT);
+  return note_forward(run_stack(layers, nlayers, x, S(stream)), IFQ_FORWARD_LAYERS);
+}
+
+int ifq_last_forward_mode(int* mode) {
+  if (!mode || t_last_forward == 0) return IFQ_EINVAL;
+  *mode = t_last_forward;
+  return IFQ_OK;
 }
 
 }  // extern "C"

@@ -23,6 +23,7 @@ IFQ_OK, IFQ_EINVAL, IFQ_ESHAPE, IFQ_EALIGN, IFQ_ERANGE, IFQ_ECUDA, IFQ_ETIMEOUT,
 IFQ_OUT_CODES, IFQ_OUT_ACC, IFQ_OUT_BOTH = 1, 2, 3
 IFQ_PATH_AUTO, IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT = 0, 1, 2, 3
 IFQ_LAYER_CONV, IFQ_LAYER_POOL, IFQ_LAYER_FIXED = 1, 2, 3
+IFQ_FORWARD_LAYERS, IFQ_FORWARD_PERSISTENT = 1, 2
 
 
 class IfqError(RuntimeError):
@@ -77,6 +78,7 @@ _SIGS = {
     "ifq_forward_workspace_bytes": ([ctypes.POINTER(Layer), _I, ctypes.POINTER(_SZ)], _I),
     "ifq_forward": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P], _I),
     "ifq_forward_noalloc": ([ctypes.POINTER(Layer), _I, _P, _P], _I),
+    "ifq_last_forward_mode": ([ctypes.POINTER(_I)], _I),
     "ifq_graph_create": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, ctypes.POINTER(_P)], _I),
     "ifq_graph_create_io": ([ctypes.POINTER(Layer), _I, _P, _P, _SZ, _P, _SZ, ctypes.POINTER(_P), ctypes.POINTER(_P),
                              _P, ctypes.POINTER(_P)], _I),
@@ -284,6 +286,13 @@ def ifq_forward(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=N
 def ifq_forward_noalloc(layers: Sequence[Layer], x, stream=None):
     arr, n = _layer_array(layers)
     _ok(lib().ifq_forward_noalloc(arr, n, _ptr(x), _stream(stream)), "ifq_forward_noalloc")
+
+
+def ifq_last_forward_mode() -> int:
+    """IFQ_FORWARD_LAYERS or IFQ_FORWARD_PERSISTENT for this thread's last forward call."""
+    m = ctypes.c_int(0)
+    _ok(lib().ifq_last_forward_mode(ctypes.byref(m)), "ifq_last_forward_mode")
+    return m.value
 
 
 def ifq_graph_create(layers: Sequence[Layer], x, ws=None, ws_bytes: int = 0, stream=None) -> int:

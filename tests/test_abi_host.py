@@ -260,3 +260,20 @@ def test_graph_with_copies_validates_the_stack_before_any_capture():
     assert e.value.status == ifq.IFQ_EINVAL
     arr = (ifq.Layer * 1)(L0)
     assert ifq.lib().ifq_graph_create_io(arr, 1, fake, None, 0, None, 0, None, None, None, None) == ifq.IFQ_EINVAL
+
+
+def test_last_forward_mode_before_any_forward_is_einval():
+    """A host thread that has made no forward call has no launch mode to report."""
+    import threading
+    out = {}
+
+    def probe():
+        try:
+            ifq.ifq_last_forward_mode()
+        except ifq.IfqError as e:
+            out["status"] = e.status
+
+    t = threading.Thread(target=probe)
+    t.start()
+    t.join()
+    assert out.get("status") == ifq.IFQ_EINVAL

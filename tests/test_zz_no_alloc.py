@@ -3,9 +3,9 @@
 Its persistent launch keeps completion counters in a file-scope device array
 instead of a caller's workspace, so the checks here are that two calls in a
 row give exactly what ifq_forward gives (the counters are re-zeroed on every
-call), both for a stack that takes the persistent launch (checked in the
-profiler's kernel list: the persistent kernel ran, no per-layer conv kernel
-did) and for one that runs layer by layer, and that a stack needing more
+call), both for a stack that takes the persistent launch (checked with
+ifq_last_forward_mode: the one persistent launch is what ran) and for one that
+runs layer by layer, and that a stack needing more
 counters than the array holds is refused before anything runs.
 """
 import numpy as np
@@ -16,17 +16,6 @@ from paper_1911_08076_gb300 import ifq, synth
 from paper_1911_08076_gb300.stack import DeviceStack
 
 DEV = "cuda"
-
-
-def _kernels_launched(fn):
-    """Names of the GPU kernels that fn launches (CUDA activity of the torch profiler)."""
-    from torch.profiler import ProfilerActivity, profile
-    with profile(activities=[ProfilerActivity.CUDA]) as prof:
-        fn()
-        torch.cuda.synchronize()
-    names = [e.name for e in prof.events() if e.device_type == torch.autograd.DeviceType.CUDA]
-    assert names, "the profiler recorded no GPU kernel"
-    return names
 
 
 def _outputs(st):
@@ -46,19 +35,17 @@ def test_noalloc_forward_equals_forward_on_two_calls_in_a_row(name, monkeypatch)
     xd = torch.from_numpy(synth.pack_codes(x)).to(DEV)
     ifq.ifq_forward(st.layers, xd)        # reference: the default entry point, one launch per layer
     torch.cuda.synchronize()
+    assert ifq.ifq_last_forward_mode() == ifq.IFQ_FORWARD_LAYERS
     ref = _outputs(st)
     for call in range(2):
         for t in list(st.y_codes.values()) + list(st.y_acc.values()):
             t.fill_(-1)                   # every output element must be written again
+        ifq.ifq_forward_noalloc(st.layers, xd)
         torch.cuda.synchronize()
-        kernels = _kernels_launched(lambda: ifq.ifq_forward_noalloc(st.layers, xd))
         assert ifq.ifq_device_status() == ifq.IFQ_OK, call
-        # the persistent launch (the one that uses the device counter array) really ran, and only it
-        stack = [k for k in kernels if "conv_stack_kernel" in k]
-        if persistent:
-            assert stack and not any("conv_tc_kernel" in k for k in kernels), (call, kernels)
-        else:
-            assert not stack and any("conv_tc_kernel" in k for k in kernels), (call, kernels)
+        # the persistent launch (the one that uses the device counter array) is what ran
+        expect = ifq.IFQ_FORWARD_PERSISTENT if persistent else ifq.IFQ_FORWARD_LAYERS
+        assert ifq.ifq_last_forward_mode() == expect, call
         got = _outputs(st)
         for li in ref:
             for k in ref[li]:
