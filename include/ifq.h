@@ -72,7 +72,7 @@ typedef enum {
 enum { IFQ_OUT_CODES = 1, IFQ_OUT_ACC = 2, IFQ_OUT_BOTH = 3 };
 
 /* Kernel path of a convolution (ifq_conv_desc.path). */
-enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2, IFQ_PATH_DIRECT = 3 };
+enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2, IFQ_PATH_DIRECT = 3, IFQ_PATH_WIN = 4 };
 
 /* Layer kinds of ifq_forward. */
 enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2, IFQ_LAYER_FIXED = 3 };
@@ -86,8 +86,10 @@ int ifq_version(void);
 /*
  * Environment switches, read on every call that uses them (for experiments; the defaults are the
  * measured best):
- *   IFQ_FORCE_PATH   = 1 / 2 / 3: request IFQ_PATH_TC / IFQ_PATH_BITSERIAL / IFQ_PATH_DIRECT
- *                      where a descriptor says IFQ_PATH_AUTO (ifq_conv_plan reports the result).
+ *   IFQ_FORCE_PATH   = 1 / 2 / 3 / 4: request IFQ_PATH_TC / IFQ_PATH_BITSERIAL / IFQ_PATH_DIRECT /
+ *                      IFQ_PATH_WIN where a descriptor says IFQ_PATH_AUTO (ifq_conv_plan reports the
+ *                      result).
+ *   IFQ_WIN          = 0: never take the window path (IFQ_PATH_WIN requests take the tensor-core path).
  *   IFQ_TC_BN        = 32 / 64 / 128: the tensor-core kernel's output-channel tile width.
  *   IFQ_TC_KS        = 1 / 2: forbid / force splitting K over clusters of two CTAs (by default only
  *                      layers that would leave more than half of the SMs idle are split).
@@ -213,7 +215,13 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
 
 /*
  * The kernel path ifq_conv2bit takes for `d` (host; reads IFQ_FORCE_PATH as
- * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL or IFQ_PATH_DIRECT.  The
+ * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT or
+ * IFQ_PATH_WIN.  The window path (the default where it applies) serves
+ * stride-1 k x k layers with "same" padding (k odd, <= 7) on 2-bit codes with
+ * cin 16 or a multiple of 32, cout 32, 64 or a multiple of 128, no pool or a
+ * 2 x 2 pool on even sizes, output rows of at most 256 pixels, and a filter
+ * bank that stays resident in one CTA's shared memory; a request for it
+ * elsewhere takes the tensor-core path.  The
  * tensor-core path needs (2^k - 1)*K <= 196608 (the accumulator range checked
  * exact on the fp8 tensor cores; 255*K for 8-bit inputs), kh, kw <= 32, and
  * for k = 3, 4 cin % 8 == 0; a request for it outside that range takes the

@@ -1,0 +1,464 @@
+// Window path of the quantized convolution (Eq. (1) integer core, Eq. (7)
+// thresholds fused as the epilogue) for stride-1 k x k layers with "same"
+// padding, on the sm_103a tensor cores.
+//
+// GEMM view with the output pixels on the MMA's N side:
+//   D[m][j] = sum_K A[m][K] * B[j][K],   m = (sy, n): output row offset sy and
+//   output channel n of the tile; j = an anchor pixel of the tile's band.
+//
+// B is the input itself.  A tile's band of input rows is expanded once into
+// shared memory as e4m3 bytes (a 2-bit code c is the e4m3 byte c, c * 2^-9),
+// one 16-byte slot per pixel and 16-channel plane, rows `pitch` slots apart
+// with zero slots for the padding.  The MMA's B operand for one tap (dy, dx)
+// is that band read at an offset of dy * pitch + dx slots: in the
+// non-swizzled K-major layout a core matrix is 8 rows of 16 bytes, 16 bytes
+// apart, so consecutive anchors are consecutive slots and every tap is just
+// another descriptor over the same bytes.  No im2col copy is ever made.
+//
+// A is the filter bank, made resident in shared memory once per CTA as a
+// block-Toeplitz matrix: row (sy, n) holds w[n][iy - sy][ix][c] at K position
+// (iy, ix, c) for 0 <= iy - sy < k, zero elsewhere.  So one accumulator row
+// computes output row y0 + sy of channel n, and with 128 / cout output rows
+// stacked along M a layer with few channels still fills the 128 lanes of the
+// MMA.  The prepared filter rows (ifq_pack_weights: e4m3 +-1, natural
+// (dy, dx, c) order with the intra-word order of the code expansion) are its
+// source, 16 bytes at a time.
+//
+// Exactness is that of the main path: every product is +-c * 2^-9 and every
+// partial sum an integer multiple of 2^-9 far inside the fp32 significand
+// (the planner admits 3 K <= 196608), so D = A_int / 512 exactly.
+//
+// Epilogue: tensor-memory lane m is one output channel of one output row, so
+// its three thresholds are per-thread constants.  A channel with a negative
+// BN scale compares against a' = (-T - 1) / 512 in ascending order and flips
+// its code (c ^ 3): sign * A > T  <=>  A < -T  <=>  not (A > -T - 1).  The
+// codes of 32 channels of one pixel are gathered with two warp ballots (bit 1
+// and the parity of the three compares) and packed into the 8 bytes those
+// channels occupy in the NHWC output.  The fused 2 x 2 pool (Sec. 2.1: on
+// Y^conv, before BN and the quantizer) takes the max of A over the
+// horizontal pair in registers; the vertical pair is either two anchor rows
+// of the same thread (one output row per tile row) or two warps (stacked
+// output rows), combined as codes: code(max A) is the max of the codes for a
+// positive BN scale and the min for a negative one.
+//
+// Warps: 0-3 epilogue (lane quadrant = warp), 4 TMEM allocation and MMA
+// issue, 5-8 band producers.  Two band buffers and two accumulators, so the
+// expansion of tile i+1, the MMAs of tile i and the epilogue of tile i-1 run
+// at once.  Every wait is bounded (IFQ_ETIMEOUT, then every role leaves its
+// loop; epilogue pairs keep their named barriers).
+#pragma once
+#include "conv_common.cuh"
+
+namespace ifq {
+
+constexpr int kWinEpiWarps = 4;
+constexpr int kWinMmaWarp = 4;
+constexpr int kWinProd0 = 5;
+constexpr int kWinProdWarps = 4;
+constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 288
+constexpr int kWinXchgBytes = 4096;    // pooled codes passed between the two warps of a row pair
+constexpr int kWinMaxSmem = 232448;    // dynamic shared memory per CTA
+
+struct WinArgs {
+  const uint8_t* x;        // packed 2-bit NHWC input codes
+  const uint8_t* w_prep;   // prepared e4m3 filter rows [cout][Kpad]
+  const int32_t* thr;      // [cout][3]
+  const int8_t* sign;      // [cout]
+  uint8_t* y_codes;        // packed 2-bit output codes (after the fused pool) or nullptr
+  int32_t* y_acc;          // int32 accumulators or nullptr (never with a fused pool)
+  int n, h, w, cin, cout, k, pad, Kpad;
+  int planes;       // cin / 16
+  int ct;           // output channels of a tile; M = ry * ct = 128
+  int ry;           // output rows stacked along M
+  int nct;          // channel tiles, cout / ct
+  int R;            // anchor rows of a tile (1 when ry > 1)
+  int rows;         // output rows a tile covers: ry * R
+  int pitch;        // slots per band row
+  int N;            // MMA N: anchors per tile, a multiple of 16, <= 256
+  int rb;           // band rows: rows + k - 1
+  int kc;           // 16-byte core columns of the Toeplitz K (even)
+  int kc_real;      // of which carry filter bytes: (ry + k - 1) * k * planes
+  int bands;        // tiles per image and channel tile
+  int ntiles;       // n * bands (per channel tile)
+  int lpool;        // 1: fused 2 x 2 / stride 2 max pool
+  uint32_t plane_stride;   // bytes between the planes of a band buffer
+  uint32_t band_bytes;     // bytes of one band buffer
+  uint32_t a_bytes;        // bytes of the resident A operand (kc * 2048)
+  FastDiv div_planes, div_pitch, div_bands;
+};
+
+// Shared-memory descriptor of a K-major operand in the non-swizzled layout: core matrices of
+// 8 rows x 16 bytes, `lbo` bytes apart along K and `sbo` bytes apart along M/N.
+__device__ __forceinline__ uint64_t sdesc_none(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+         ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
+}
+
+// 32 bits -> 64 bits with bit i at bit 2i.
+__device__ __forceinline__ uint64_t spread_bits(uint32_t x) {
+  uint64_t v = x;
+  v = (v | (v << 16)) & 0x0000FFFF0000FFFFull;
+  v = (v | (v << 8)) & 0x00FF00FF00FF00FFull;
+  v = (v | (v << 4)) & 0x0F0F0F0F0F0F0F0Full;
+  v = (v | (v << 2)) & 0x3333333333333333ull;
+  v = (v | (v << 1)) & 0x5555555555555555ull;
+  return v;
+}
+
+// Field-wise max of two words of 32 two-bit codes, after flipping (c ^ 3) the fields set in `flip`
+// and flipping the result back: the max for plain fields, the min for flipped ones.
+__device__ __forceinline__ uint64_t pool_codes2(uint64_t a, uint64_t b, uint64_t flip) {
+  constexpr uint64_t H = 0xAAAAAAAAAAAAAAAAull, L = 0x5555555555555555ull;
+  a ^= flip;
+  b ^= flip;
+  const uint64_t ha = a & H, hb = b & H;
+  const uint64_t only_a = (ha & ~hb) >> 1, only_b = (hb & ~ha) >> 1;
+  const uint64_t lo = ((a & L) & ~only_b) | ((b & L) & ~only_a);
+  return (ha | hb | lo) ^ flip;
+}
+
+// Byte address in a band buffer of 16-byte core column c = (iy, ix, p) of the Toeplitz K, for
+// anchor 0.
+__device__ __forceinline__ uint32_t win_col_addr(const WinArgs& a, int c) {
+  const int p = c % a.planes, t = c / a.planes;
+  const int iy = t / a.k, ix = t - iy * a.k;
+  return (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.pitch + ix);
+}
+
+template <int POOL>
+__global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs a) {
+  extern __shared__ uint8_t smem_raw_[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t sA = sbase;
+  const uint32_t sBand = sbase + a.a_bytes;
+  uint64_t* xchg = (uint64_t*)(smem + a.a_bytes + 2 * a.band_bytes);
+  const uint32_t barBase = sbase + a.a_bytes + 2 * a.band_bytes + kWinXchgBytes;
+  auto band_full = [&](int b) { return barBase + 8u * b; };
+  auto band_empty = [&](int b) { return barBase + 16u + 8u * b; };
+  auto acc_full = [&](int b) { return barBase + 32u + 8u * b; };
+  auto acc_empty = [&](int b) { return barBase + 48u + 8u * b; };
+  const uint32_t done_bar = barBase + 64u;
+  uint32_t* tmem_slot = (uint32_t*)(smem + a.a_bytes + 2 * a.band_bytes + kWinXchgBytes + 80);
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  // CTA c takes channel tile c % nct and the band tiles c / nct, c / nct + G / nct, ... of it
+  const int ctile = (int)blockIdx.x % a.nct;
+  const int first = (int)blockIdx.x / a.nct, step = (int)gridDim.x / a.nct;
+  const int n_local = first < a.ntiles ? (a.ntiles - first + step - 1) / step : 0;
+
+  if (warp == kWinMmaWarp) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
+    tmem_relinquish();
+  }
+  if (tid == 0) {
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(band_full(b), kWinProdWarps);
+      mbar_init(band_empty(b), 1);
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), kWinEpiWarps);
+    }
+    mbar_init(done_bar, 1);
+    fence_mbar_init();
+  }
+  grid_dep_wait();
+  // The resident A operand: row m = (sy, nl) at 16-byte core column c = (iy, ix, p) holds bytes
+  // [16p, 16p + 16) of tap (iy - sy, ix) of filter n, or zeros.  Layout: core column c, row group
+  // m / 8, row m % 8 -> c * 2048 + (m / 8) * 128 + (m % 8) * 16.
+  for (int it = tid; it < 128 * a.kc; it += kWinThreads) {
+    const int c = it >> 7, m = it & 127;
+    const int sy = m / a.ct, nl = m - sy * a.ct;
+    const int n = ctile * a.ct + nl;
+    const uint8_t* src = a.w_prep;
+    uint32_t bytes = 0;
+    if (c < a.kc_real) {
+      const int p = c % a.planes, t = c / a.planes;
+      const int iy = t / a.k, ix = t - iy * a.k, dy = iy - sy;
+      if (dy >= 0 && dy < a.k) {
+        src = a.w_prep + (size_t)n * a.Kpad + (size_t)((dy * a.k + ix) * a.cin + 16 * p);
+        bytes = 16;
+      }
+    }
+    cp_async_16(sA + (uint32_t)c * 2048u + (uint32_t)(m >> 3) * 128u + (uint32_t)(m & 7) * 16u, src, bytes);
+  }
+  cp_async_commit();
+  // both band buffers start as zeros: padding slots and the tail past the band stay zero
+  for (uint32_t o = (uint32_t)tid * 16u; o < 2u * a.band_bytes; o += kWinThreads * 16u)
+    *(uint4*)(smem + a.a_bytes + o) = make_uint4(0u, 0u, 0u, 0u);
+  cp_async_wait<0>();
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  grid_dep_launch();
+
+  if (warp >= kWinProd0) {
+    // =================== producers: packed input rows -> e4m3 band in shared memory ===================
+    const int pt = tid - kWinProd0 * 32;   // 0..127
+    const int cinb = a.cin >> 2;           // packed bytes per pixel
+    const int items = a.rb * a.pitch * a.planes;
+    bool ok = true;
+#pragma unroll 1
+    for (int i = 0; i < n_local && ok; ++i) {
+      const int bb = i & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait_backoff(band_empty(bb), ((uint32_t)(i >> 1) & 1u) ^ 1u, 64))) {
+        ok = false;
+        break;
+      }
+      const int t = first + i * step;
+      const int b = (int)fdiv((uint32_t)t, a.div_bands);
+      const int y0 = (t - b * a.bands) * a.rows;
+      const uint8_t* img = a.x + (size_t)b * a.h * a.w * cinb;
+      const uint32_t dst0 = sBand + (uint32_t)bb * a.band_bytes;
+#pragma unroll 1
+      for (int base = pt; base < items; base += 4 * 128) {
+        uint32_t v[4];
+        uint32_t dst[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int it = base + u * 128;
+          v[u] = 0u;
+          dst[u] = 0xFFFFFFFFu;
+          if (it < items) {
+            const int rest = (int)fdiv((uint32_t)it, a.div_planes);
+            const int p = it - rest * a.planes;
+            const int iy = (int)fdiv((uint32_t)rest, a.div_pitch);
+            const int slot = rest - iy * a.pitch;
+            const int xx = slot - a.pad, yy = y0 - a.pad + iy;
+            if (xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
+              v[u] = ld_codes4<false>(img + ((size_t)yy * a.w + xx) * cinb + 4 * p);
+            dst[u] = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.pitch + slot);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          if (dst[u] != 0xFFFFFFFFu) {
+            const uint32_t w = v[u];
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst[u]), "r"(w & 0x03030303u),
+                         "r"((w >> 2) & 0x03030303u), "r"((w >> 4) & 0x03030303u), "r"((w >> 6) & 0x03030303u)
+                         : "memory");
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(band_full(bb));
+    }
+  } else if (warp == kWinMmaWarp) {
+    // =================== MMA issue (one elected lane; the warp runs the loop) ===================
+    const uint32_t idesc = idesc_e4m3_f32(128, a.N);
+    const int nmma = a.kc >> 1;
+    bool ok = true;
+#pragma unroll 1
+    for (int i = 0; i < n_local && ok; ++i) {
+      const int bb = i & 1;
+      const uint32_t ph = (uint32_t)(i >> 1) & 1u;
+      bool got = mbar_wait(band_full(bb), ph);
+      got = got && mbar_wait(acc_empty(bb), ph ^ 1u);
+      if (!__all_sync(0xffffffffu, got)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (elect_one()) {
+        const uint32_t band = sBand + (uint32_t)bb * a.band_bytes;
+        const uint32_t dacc = tmem + (uint32_t)(bb * 256);
+#pragma unroll 1
+        for (int q = 0; q < nmma; ++q) {
+          const int c0 = 2 * q;
+          const uint32_t b0 = win_col_addr(a, c0);
+          // the second core column: the next K column, or (past the filter bytes, where A is zero)
+          // the slot after the first
+          const uint32_t b1 = c0 + 1 < a.kc_real ? win_col_addr(a, c0 + 1) : b0 + 16u;
+          const uint64_t ad = sdesc_none(sA + (uint32_t)c0 * 2048u, 2048u, 128u);
+          const uint64_t bd = sdesc_none(band + b0, b1 - b0, 128u);
+          mma_e4m3(dacc, ad, bd, idesc, q > 0 ? 1u : 0u);
+        }
+        mma_commit(band_empty(bb));
+        mma_commit(acc_full(bb));
+      }
+      __syncwarp();
+    }
+    if (elect_one()) mma_commit(done_bar);
+    __syncwarp();
+  } else {
+    // =================== epilogue: thresholds, code packing, fused pool, stores ===================
+    const int q = warp;                          // lane quadrant
+    const int sy = (32 * q) / a.ct;              // output row offset of this quadrant
+    const int cg = ((32 * q) % a.ct) >> 5;       // 32-channel group within the channel tile
+    const int n = ctile * a.ct + cg * 32 + lane;
+    // thresholds in the fp32 domain of D = A / 512; negative scale: ascending (-T - 1) / 512
+    float t1 = 0.f, t2 = 0.f, t3 = 0.f;
+    bool neg = false;
+    if (a.thr) {
+      const int32_t T0 = a.thr[3 * n], T1 = a.thr[3 * n + 1], T2 = a.thr[3 * n + 2];
+      neg = a.sign[n] < 0;
+      if (!neg) {
+        t1 = (float)T0 * (1.0f / 512.0f);
+        t2 = (float)T1 * (1.0f / 512.0f);
+        t3 = (float)T2 * (1.0f / 512.0f);
+      } else {
+        t1 = (float)(-T2 - 1) * (1.0f / 512.0f);
+        t2 = (float)(-T1 - 1) * (1.0f / 512.0f);
+        t3 = (float)(-T0 - 1) * (1.0f / 512.0f);
+      }
+    }
+    const uint32_t negmask = __ballot_sync(0xffffffffu, neg);
+    const uint64_t flip = spread_bits(negmask) * 3ull;
+    const int rowb = a.cout >> 2;                                  // output bytes per pixel
+    const int chb = (ctile * a.ct + cg * 32) >> 2;                 // this warp's byte within a pixel
+    const uint32_t lane_off = (uint32_t)(32 * q) << 16;
+    // row pairs of stacked output rows (ry > 1, pooled): the odd row's warp hands its codes over
+    const int partner_off = a.ct / 32;                             // quadrant distance of sy and sy + 1
+    const int pair = a.ct == 32 ? (q >> 1) : (q & 1);
+    const bool odd_row = (sy & 1) != 0;
+    bool ok = true;
+#pragma unroll 1
+    for (int i = 0; i < n_local; ++i) {
+      const int ab = i & 1;
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait_backoff(acc_full(ab), (uint32_t)(i >> 1) & 1u, 64));
+      const int t = first + i * step;
+      const int b = (int)fdiv((uint32_t)t, a.div_bands);
+      const int y0 = (t - b * a.bands) * a.rows;
+      const uint32_t tacc = tmem + (uint32_t)(ab * 256) + lane_off;
+      if (ok) tc_fence_after();
+      if constexpr (POOL == 0) {
+        if (ok) {
+#pragma unroll 1
+          for (int g = 0; g * 32 < a.N; ++g) {
+            uint32_t k0 = 0, k1 = 0;
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              uint32_t v[16];
+              tmem_ld16_sync(tacc + (uint32_t)(32 * g + 16 * h), v);
+#pragma unroll
+              for (int c = 0; c < 16; ++c) {
+                const float f = __uint_as_float(v[c]);
+                const bool p1 = f > t1, p2 = f > t2, p3 = f > t3;
+                const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
+                const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
+                if (lane == 16 * h + c) {
+                  k0 = m0;
+                  k1 = m1;
+                }
+                if (a.y_acc) {
+                  const int j = 32 * g + 16 * h + c;
+                  const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
+                  const int yy = y0 + r + sy;
+                  if (j < a.N && r < a.R && xx < a.w && yy < a.h)
+                    a.y_acc[(((size_t)b * a.h + yy) * a.w + xx) * a.cout + n] = __float2int_rn(f * 512.0f);
+                }
+              }
+            }
+            const int j = 32 * g + lane;
+            const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
+            const int yy = y0 + r + sy;
+            if (a.y_codes && j < a.N && r < a.R && xx < a.w && yy < a.h) {
+              const uint64_t codes = (spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1));
+              *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = codes;
+            }
+          }
+        }
+      } else {
+        // pooled output map: (h / 2) x (w / 2)
+        const int pw = a.w >> 1, ph = a.h >> 1;
+        uint64_t own[4] = {0ull, 0ull, 0ull, 0ull};
+        const int npool = a.ry > 1 ? (a.N >> 1) : (a.R >> 1) * (a.pitch >> 1);
+        if (ok) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            if (32 * g < npool) {
+              uint32_t k0 = 0, k1 = 0;
+#pragma unroll
+              for (int h = 0; h < 4; ++h) {
+                // 8 pooled columns from 16 accumulator columns of a row (and of the next row when
+                // one output row per tile row: pitch % 16 == 0)
+                uint32_t v[16];
+                float mx[8];
+                const int pi0 = 32 * g + 8 * h;   // first pooled index of this chunk
+                if (pi0 >= npool) {
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) mx[e] = 0.f;
+                } else if (a.ry > 1) {
+                  tmem_ld16_sync(tacc + (uint32_t)(2 * pi0), v);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) mx[e] = fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                } else {
+                  const int half = a.pitch >> 1;
+                  const int pr = pi0 / half, px0 = pi0 - pr * half;
+                  const uint32_t col = (uint32_t)(2 * pr * a.pitch + 2 * px0);
+                  tmem_ld16_sync(tacc + col, v);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e) mx[e] = fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                  tmem_ld16_sync(tacc + col + (uint32_t)a.pitch, v);
+#pragma unroll
+                  for (int e = 0; e < 8; ++e)
+                    mx[e] = fmaxf(mx[e], fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1])));
+                }
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                  const bool p1 = mx[e] > t1, p2 = mx[e] > t2, p3 = mx[e] > t3;
+                  const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
+                  const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
+                  if (lane == 8 * h + e) {
+                    k0 = m0;
+                    k1 = m1;
+                  }
+                }
+              }
+              own[g] = spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1);
+            }
+          }
+        }
+        if (a.ry > 1) {
+          // rows sy (even) and sy + 1 of the window live in two warps: the odd one hands over
+          uint64_t* xc = xchg + (size_t)((i & 1) * 2 + pair) * 128;
+          if (odd_row) {
+#pragma unroll
+            for (int g = 0; g < 4; ++g)
+              if (32 * g < npool) xc[32 * g + lane] = own[g];
+          }
+          named_bar(1 + pair, 64);
+          if (!odd_row && ok) {
+            const int py = (y0 + sy) >> 1;
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              const int px = 32 * g + lane;
+              if (32 * g < npool && px < pw && py < ph && a.y_codes) {
+                const uint64_t c = pool_codes2(own[g], xc[px], flip);
+                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = c;
+              }
+            }
+          }
+        } else if (ok) {
+          const int half = a.pitch >> 1;
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            const int pi = 32 * g + lane;
+            const int pr = pi / half, px = pi - pr * half;
+            const int py = (y0 >> 1) + pr;
+            if (pi < npool && px < pw && py < ph && a.y_codes)
+              *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = own[g];
+          }
+        }
+      }
+      if (ok) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty(ab));
+      }
+    }
+  }
+
+  // ---- teardown: every MMA has completed (done_bar) before tensor memory is released
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWinMmaWarp) {
+    tc_fence_after();
+    mbar_wait(done_bar, 0);
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+}  // namespace ifq

@@ -17,6 +17,7 @@
 #include "conv_bitserial.cuh"
 #include "conv_direct.cuh"
 #include "conv_tc.cuh"
+#include "conv_win.cuh"
 #include "ifq.h"
 #include "pool_pack.cuh"
 #include "selftest.cuh"
@@ -199,6 +200,11 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
         set_attrs_gb<4, 4, 4>() != cudaSuccess || set_attrs_gb<16, 4, 2>() != cudaSuccess ||
         set_attrs_gb<8, 4, 2>() != cudaSuccess || set_attrs_gb<4, 4, 2>() != cudaSuccess)
       return IFQ_ECUDA;
+    if (cudaFuncSetAttribute(conv_win_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(conv_win_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
+            cudaSuccess)
+      return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
     if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
         cudaSuccess)
@@ -276,7 +282,7 @@ int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if (d->cin % 4 != 0) return IFQ_ESHAPE;
   if (d->out_mode < IFQ_OUT_CODES || d->out_mode > IFQ_OUT_BOTH) return IFQ_EINVAL;
   if ((d->out_mode & IFQ_OUT_CODES) && d->cout % 4 != 0) return IFQ_ESHAPE;
-  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_DIRECT) return IFQ_EINVAL;
+  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_WIN) return IFQ_EINVAL;
   const long long K = (long long)d->kh * d->kw * d->cin;
   const long long M = (long long)d->n * g->ho * g->wo;
   if (K > kMaxK || d->cout > 65536 || M >= (1LL << 31)) return IFQ_ERANGE;
@@ -341,13 +347,93 @@ cudaError_t launch_narrow(int cin, int pool, int cout, dim3 grid, dim3 block, co
   return pool == 2 ? launch_narrow_cp<16, 2>(cout, grid, block, a, st) : launch_narrow_cp<16, 1>(cout, grid, block, a, st);
 }
 
+// Geometry of the window kernel (conv_win.cuh) for a layer, or false where it does not apply:
+// 2-bit codes in and out, stride 1, k x k with "same" padding (k odd, <= 7), cin 16 or a multiple of
+// 32, cout 32, 64 or a multiple of 128 (at most one channel tile per SM), a fused pool of 2 on even
+// sizes or none, an output row of at most 256 anchors, and the resident filters plus two band
+// buffers within the shared memory of one CTA.  Fills every field but the pointers.
+bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, size_t* smem) {
+  if (env_int("IFQ_WIN", 1) == 0) return false;
+  if (g.in8 || g.kb != 2) return false;
+  const int k = d->kh;
+  if (d->stride != 1 || d->kw != k || (k & 1) == 0 || k > 7 || 2 * d->pad != k - 1) return false;
+  if (!(d->cin == 16 || d->cin % 32 == 0)) return false;
+  int ct;
+  if (d->cout == 32 || d->cout == 64) ct = d->cout;
+  else if (d->cout % 128 == 0) ct = 128;
+  else return false;
+  const int nct = d->cout / ct;
+  if (nct > nsm) return false;
+  if (g.pool != 1 && g.pool != 2) return false;
+  const bool pool = g.pool == 2;
+  const int H = g.ho, W = g.wo;
+  if (pool && ((H & 1) || (W & 1))) return false;
+  const int ry = 128 / ct, planes = d->cin / 16;
+  int pitch, R, N;
+  if (ry > 1) {
+    pitch = W + k - 1;
+    R = 1;
+    N = (int)round_up((size_t)W, 16);
+    if (N > 256) return false;
+  } else {
+    pitch = W + k - 1;
+    if (pool) pitch = (int)round_up((size_t)pitch, 16);   // row pairs of the pool at aligned columns
+    if (pitch > 256) return false;
+    R = std::min(H, 256 / pitch);
+    if (pool) R &= ~1;
+    if (R < 1) return false;
+    N = (int)round_up((size_t)(R * pitch), 16);
+  }
+  const int rows = ry > 1 ? ry : R;
+  const int rb = rows + k - 1;
+  const int kc_real = (ry + k - 1) * k * planes;
+  const int kc = (int)round_up((size_t)kc_real, 2);
+  // slots a plane needs: the band rows, and what the MMAs read past them (N anchors from the
+  // farthest tap, and the slot after the last core column), with slack
+  const int iy_max = ry + k - 2;
+  const int slots = std::max(rb * pitch, iy_max * pitch + (k - 1) + N + 2) + 4;
+  const uint32_t ps = (uint32_t)round_up((size_t)slots * 16, 128) + (planes > 1 ? 16u : 0u);
+  const uint32_t band_bytes = (uint32_t)round_up((size_t)planes * ps, 1024);
+  const uint32_t a_bytes = (uint32_t)kc * 2048u;
+  const size_t need = 1024 + (size_t)a_bytes + 2 * (size_t)band_bytes + kWinXchgBytes + 128;
+  if (need > (size_t)kWinMaxSmem) return false;
+  if (wa) {
+    memset(wa, 0, sizeof(*wa));
+    wa->n = d->n; wa->h = H; wa->w = W; wa->cin = d->cin; wa->cout = d->cout; wa->k = k; wa->pad = d->pad;
+    wa->Kpad = g.Kpad;
+    wa->planes = planes; wa->ct = ct; wa->ry = ry; wa->nct = nct; wa->R = R; wa->rows = rows; wa->pitch = pitch;
+    wa->N = N; wa->rb = rb; wa->kc = kc; wa->kc_real = kc_real;
+    wa->bands = ceil_div(H, rows);
+    wa->ntiles = d->n * wa->bands;
+    wa->lpool = pool ? 1 : 0;
+    wa->plane_stride = ps;
+    wa->band_bytes = band_bytes;
+    wa->a_bytes = a_bytes;
+    wa->div_planes = make_fastdiv((uint32_t)planes);
+    wa->div_pitch = make_fastdiv((uint32_t)pitch);
+    wa->div_bands = make_fastdiv((uint32_t)wa->bands);
+  }
+  if (smem) *smem = need;
+  return true;
+}
+
+bool win_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  int nsm = 0;
+  if (ensure_init(&nsm)) nsm = 148;   // no device: plan as for a full GB300
+  return win_plan(d, g, nsm, nullptr, nullptr);
+}
+
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
     path = forced ? forced
-                  : (direct_supported(d, g) ? IFQ_PATH_DIRECT : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL : IFQ_PATH_TC));
+                  : (direct_supported(d, g) ? IFQ_PATH_DIRECT
+                                            : (win_supported(d, g) ? IFQ_PATH_WIN
+                                                                   : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL
+                                                                                        : IFQ_PATH_TC)));
   }
+  if (path == IFQ_PATH_WIN && !win_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_DIRECT && !direct_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
   // the fused pool has a bit-serial form only in the narrow kernel; 8-bit inputs have none
@@ -539,6 +625,21 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     else if (d->cout <= 8) e = launch_k(conv_direct_kernel<4>, grid, block, 0, st, a);
     else if (d->cout <= 16) e = launch_k(conv_direct_kernel<8>, grid, block, 0, st, a);
     else e = launch_k(conv_direct_kernel<16>, grid, block, 0, st, a);
+  } else if (path == IFQ_PATH_WIN) {
+    WinArgs wa;
+    size_t smem = 0;
+    if (!win_plan(d, g, nsm, &wa, &smem)) return IFQ_EUNSUPPORTED;
+    wa.x = (const uint8_t*)x;
+    wa.w_prep = (const uint8_t*)w_prep;
+    wa.thr = thr;
+    wa.sign = sign;
+    wa.y_codes = yc;
+    wa.y_acc = ya;
+    // CTAs come in groups of nct, one per channel tile, each group sharing the band tiles
+    const int per = std::max(1, std::min(wa.ntiles, nsm / wa.nct));
+    const dim3 grid((unsigned)(per * wa.nct)), block(kWinThreads);
+    e = wa.lpool ? launch_k(conv_win_kernel<1>, grid, block, smem, st, wa)
+                 : launch_k(conv_win_kernel<0>, grid, block, smem, st, wa);
   } else if (path == IFQ_PATH_TC) {
     int bn = choose_bn(g, d->cout, nsm), ks = 1;
     const int gb = granule_bytes(d, g);
@@ -790,7 +891,10 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     if (check_conv(&layers[i].conv, &g)) return false;
     if (g.pool > 1 || g.kb != 2 || g.in8) return false;   // the persistent kernel: 2-bit codes, no fused pool
     if (g.M == 0) return false;                           // an empty batch runs (as nothing) layer by layer
-    if (choose_path(&layers[i].conv, g) != IFQ_PATH_TC) return false;
+    // the persistent kernel computes every layer with the tensor-core data path: layers whose own
+    // launch would take that path or the window path qualify
+    const int p = choose_path(&layers[i].conv, g);
+    if (!(p == IFQ_PATH_TC || (p == IFQ_PATH_WIN && tc_supported(&layers[i].conv, g)))) return false;
     tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g, true));
   }
   if (tab > kMaxStackTab) return false;

@@ -605,3 +605,51 @@ def test_graph_with_copies_rejects_bad_io():
     assert e.value.status == ifq.IFQ_EINVAL
     with pytest.raises(ValueError):
         ifq.ifq_graph_create_io(st.layers, xd, st.ws, st.ws_bytes, None, 0, [None])
+
+
+# ----------------------------------------------------------------------------- window path
+
+WIN_CASES = [
+    # B, H, W, C, cout, k, pool, out_mode
+    (1, 4, 16, 16, 32, 3, 1, 3),          # smallest: one tile of 4 rows x 16 anchors, 4 rows stacked on M
+    (2, 10, 10, 16, 32, 3, 1, 3),         # ragged band (10 rows in tiles of 4), N = 16 > w
+    (2, 12, 20, 16, 32, 3, 2, 1),         # fused pool, row pairs across warps
+    (2, 9, 13, 32, 64, 3, 1, 3),          # 2 planes, 2 rows stacked on M, odd sizes
+    (3, 14, 18, 32, 64, 3, 2, 1),         # fused pool over warp pairs (sy, sy + 1)
+    (2, 11, 11, 64, 128, 3, 1, 3),        # one output row per M row, several anchor rows per tile
+    (2, 12, 14, 64, 128, 3, 2, 1),        # fused pool over anchor-row pairs (16-aligned pitch)
+    (2, 9, 9, 64, 256, 3, 1, 3),          # two channel tiles
+    (1, 16, 16, 64, 64, 3, 1, 3),         # the single PR1 layer shape
+    (2, 8, 30, 32, 128, 5, 1, 3),         # 5 x 5, 7 anchor rows of 34 slots
+    (2, 6, 9, 96, 64, 3, 1, 3),           # 6 planes
+    (2, 7, 12, 128, 128, 1, 1, 3),        # 1 x 1
+    (1, 6, 40, 16, 32, 7, 1, 1),          # 7 x 7
+    (2, 26, 26, 16, 32, 3, 2, 1),         # H % 4 != 0 with the pool: the last band's rows past h
+    (1, 3, 208, 16, 32, 3, 1, 1),         # a full Tiny-YOLO row (N = 208)
+]
+
+
+@pytest.mark.parametrize("case", WIN_CASES, ids=[str(c) for c in WIN_CASES])
+def test_window_path_matches_oracle(case):
+    """The window kernel (input band in shared memory, one descriptor per tap, Toeplitz filter
+    block resident) against the oracle, bit-exact: accumulators and codes, or the codes of the
+    window maximum with the fused pool, with channels of negative BN scale in every case."""
+    B, H, W, C, cout, k, pool, mode = case
+    rng = np.random.default_rng(abs(hash(case)) % (2 ** 32))
+    x = rng.integers(0, 4, (B, H, W, C), dtype=np.uint8)
+    w = np.where(rng.integers(0, 2, (cout, k, k, C)) == 1, 1, -1).astype(np.int8)
+    K = k * k * C
+    prm = _params(rng, cout, K)
+    prm.gamma[1::3] = -np.abs(prm.gamma[1::3])
+    T, sg = _fold_gpu(prm, K)
+    pad = (k - 1) // 2
+    d = ifq.conv_desc(B, H, W, C, cout, k, 1, pad, mode, ifq.IFQ_PATH_WIN, pool=pool if pool > 1 else 0)
+    assert ifq.ifq_conv_plan(d) == ifq.IFQ_PATH_WIN
+    codes, acc = _run_conv(x, w, T, sg, 1, pad, mode, ifq.IFQ_PATH_WIN, pool=pool if pool > 1 else 0)
+    A = O.conv_acc(x, w, 1, pad)
+    if acc is not None:
+        assert (acc == A).all(), f"accumulators differ at {np.argwhere(acc != A)[:5].tolist()}"
+    To, so = O.fold(prm, K)
+    ref = O.int_chain(O.maxpool_acc(A, pool, pool, 0) if pool > 1 else A, To, so)
+    assert codes.shape == ref.shape
+    assert (codes == ref).all(), f"codes differ at {np.argwhere(codes != ref)[:5].tolist()}"
