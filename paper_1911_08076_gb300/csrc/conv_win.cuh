@@ -6,23 +6,32 @@
 //   D[m][j] = sum_K A[m][K] * B[j][K],   m = (sy, n): output row offset sy and
 //   output channel n of the tile; j = an anchor pixel of the tile's band.
 //
-// B is the input itself.  A tile's band of input rows is expanded once into
-// shared memory as e4m3 bytes (a 2-bit code c is the e4m3 byte c, c * 2^-9),
-// one 16-byte slot per pixel and 16-channel plane, rows `pitch` slots apart
-// with zero slots for the padding.  The MMA's B operand for one tap (dy, dx)
-// is that band read at an offset of dy * pitch + dx slots: in the
-// non-swizzled K-major layout a core matrix is 8 rows of 16 bytes, 16 bytes
-// apart, so consecutive anchors are consecutive slots and every tap is just
-// another descriptor over the same bytes.  No im2col copy is ever made.
+// B is the input itself.  A tile's input rows are copied to shared memory by
+// the copy engine (cp.async.bulk: an image row of packed codes is contiguous)
+// and expanded once into a band of e4m3 bytes (a 2-bit code c is the e4m3
+// byte c, c * 2^-9): one 16-byte slot per pixel and 16-channel plane, zero
+// slots for the padding.  The MMA's B operand for one tap (dy, dx) is that band
+// read at an offset of dy rows and dx slots: in the non-swizzled K-major layout
+// a core matrix is 8 rows of 16 bytes, 16 bytes apart, so consecutive anchors
+// are consecutive slots and every tap is just another descriptor over the same
+// bytes.  No im2col copy is ever made.
 //
 // A is the filter bank, made resident in shared memory once per CTA as a
 // block-Toeplitz matrix: row (sy, n) holds w[n][iy - sy][ix][c] at K position
-// (iy, ix, c) for 0 <= iy - sy < k, zero elsewhere.  So one accumulator row
-// computes output row y0 + sy of channel n, and with 128 / cout output rows
-// stacked along M a layer with few channels still fills the 128 lanes of the
-// MMA.  The prepared filter rows (ifq_pack_weights: e4m3 +-1, natural
-// (dy, dx, c) order with the intra-word order of the code expansion) are its
-// source, 16 bytes at a time.
+// (iy, ix, c) for 0 <= iy - sy < k, zero elsewhere.  So accumulator row
+// (sy, n) computes output row sy of the anchor's row band for channel n, and
+// with 128 / cout output rows stacked along M a layer with few channels still
+// fills the 128 lanes of the MMA.  The prepared filter rows (ifq_pack_weights:
+// e4m3 +-1, natural (dy, dx, c) order with the intra-word order of the code
+// expansion) are its source, 16 bytes at a time.
+//
+// Anchors.  With one output row per M row (cout >= 128) the tile's R anchor
+// rows are consecutive output rows and share the band's input rows (R + k - 1
+// of them, `seg_pitch` = pitch slots apart).  With rows stacked along M, a
+// tile is R row bands of `ry` output rows side by side along N: band row iy
+// holds input row iy of each of the R bands, `pitch` slots each, so a tap's
+// offset is the same for every anchor.  Either way anchor j is (r, x) =
+// (j / pitch, j % pitch), and columns with x >= w are computed and dropped.
 //
 // Exactness is that of the main path: every product is +-c * 2^-9 and every
 // partial sum an integer multiple of 2^-9 far inside the fp32 significand
@@ -37,15 +46,16 @@
 // channels occupy in the NHWC output.  The fused 2 x 2 pool (Sec. 2.1: on
 // Y^conv, before BN and the quantizer) takes the max of A over the
 // horizontal pair in registers; the vertical pair is either two anchor rows
-// of the same thread (one output row per tile row) or two warps (stacked
-// output rows), combined as codes: code(max A) is the max of the codes for a
+// of the same thread (one output row per M row) or two warps (stacked output
+// rows), combined as codes: code(max A) is the max of the codes for a
 // positive BN scale and the min for a negative one.
 //
 // Warps: 0-3 epilogue (lane quadrant = warp), 4 TMEM allocation and MMA
-// issue, 5-8 band producers.  Two band buffers and two accumulators, so the
-// expansion of tile i+1, the MMAs of tile i and the epilogue of tile i-1 run
-// at once.  Every wait is bounded (IFQ_ETIMEOUT, then every role leaves its
-// loop; epilogue pairs keep their named barriers).
+// issue, 5-8 producers (one lane of warp 5 issues the bulk copies).  Two
+// staging buffers, two bands and two accumulators, so the copy of tile i+2,
+// the expansion of tile i+1, the MMAs of tile i and the epilogue of tile i-1
+// overlap.  Every wait is bounded (IFQ_ETIMEOUT, then the roles leave their
+// loops; warps sharing a named barrier keep reaching it).
 #pragma once
 #include "conv_common.cuh"
 
@@ -57,6 +67,8 @@ constexpr int kWinProd0 = 5;
 constexpr int kWinProdWarps = 4;
 constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 288
 constexpr int kWinXchgBytes = 4096;    // pooled codes passed between the two warps of a row pair
+constexpr int kWinMaxMma = 64;         // MMAs per tile (K' / 32)
+constexpr int kWinTabBytes = 8 * kWinMaxMma;
 constexpr int kWinMaxSmem = 232448;    // dynamic shared memory per CTA
 
 struct WinArgs {
@@ -71,20 +83,23 @@ struct WinArgs {
   int ct;           // output channels of a tile; M = ry * ct = 128
   int ry;           // output rows stacked along M
   int nct;          // channel tiles, cout / ct
-  int R;            // anchor rows of a tile (1 when ry > 1)
+  int R;            // anchor rows of a tile
   int rows;         // output rows a tile covers: ry * R
-  int pitch;        // slots per band row
+  int pitch;        // slots of one anchor row
+  int seg_pitch;    // slots between band rows: pitch (ry = 1) or R * pitch (ry > 1)
+  int nseg;         // row bands staged per tile: 1 (ry = 1) or R
   int N;            // MMA N: anchors per tile, a multiple of 16, <= 256
-  int rb;           // band rows: rows + k - 1
+  int rb;           // band rows: R + k - 1 (ry = 1) or ry + k - 1
   int kc;           // 16-byte core columns of the Toeplitz K (even)
   int kc_real;      // of which carry filter bytes: (ry + k - 1) * k * planes
   int bands;        // tiles per image and channel tile
   int ntiles;       // n * bands (per channel tile)
-  int lpool;        // 1: fused 2 x 2 / stride 2 max pool
+  int row_bytes;    // packed bytes of one input row (a multiple of 16)
   uint32_t plane_stride;   // bytes between the planes of a band buffer
   uint32_t band_bytes;     // bytes of one band buffer
+  uint32_t stage_bytes;    // bytes of one staging buffer (nseg * rb * row_bytes, rounded)
   uint32_t a_bytes;        // bytes of the resident A operand (kc * 2048)
-  FastDiv div_planes, div_pitch, div_bands;
+  FastDiv div_planes, div_pitch, div_seg, div_bands;
 };
 
 // Shared-memory descriptor of a K-major operand in the non-swizzled layout: core matrices of
@@ -92,6 +107,14 @@ struct WinArgs {
 __device__ __forceinline__ uint64_t sdesc_none(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
   return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
+}
+
+// 1-D bulk copy global -> shared on the copy engine, completing on an mbarrier (both addresses
+// 16-byte aligned, `bytes` a multiple of 16).
+__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
 }
 
 // 32 bits -> 64 bits with bit i at bit 2i.
@@ -117,35 +140,44 @@ __device__ __forceinline__ uint64_t pool_codes2(uint64_t a, uint64_t b, uint64_t
   return (ha | hb | lo) ^ flip;
 }
 
-// Byte address in a band buffer of 16-byte core column c = (iy, ix, p) of the Toeplitz K, for
+// Byte offset in a band buffer of 16-byte core column c = (iy, ix, p) of the Toeplitz K, for
 // anchor 0.
-__device__ __forceinline__ uint32_t win_col_addr(const WinArgs& a, int c) {
+__device__ __forceinline__ uint32_t win_col_offset(const WinArgs& a, int c) {
   const int p = c % a.planes, t = c / a.planes;
   const int iy = t / a.k, ix = t - iy * a.k;
-  return (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.pitch + ix);
+  return (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.seg_pitch + ix);
 }
 
-template <int POOL>
+// First output row of tile t's anchor row r (rows of a tile: R anchor rows of ry output rows).
+__device__ __forceinline__ int win_row(const WinArgs& a, int y0, int r) { return y0 + r * a.ry; }
+
+template <int POOL, int ACC>
 __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs a) {
   extern __shared__ uint8_t smem_raw_[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
   const uint32_t sA = sbase;
   const uint32_t sBand = sbase + a.a_bytes;
-  uint64_t* xchg = (uint64_t*)(smem + a.a_bytes + 2 * a.band_bytes);
-  const uint32_t barBase = sbase + a.a_bytes + 2 * a.band_bytes + kWinXchgBytes;
+  const uint32_t oStage = a.a_bytes + 2 * a.band_bytes;
+  const uint32_t sStage = sbase + oStage;
+  const uint32_t oXchg = oStage + 2 * a.stage_bytes;
+  uint64_t* xchg = (uint64_t*)(smem + oXchg);
+  uint64_t* mtab = (uint64_t*)(smem + oXchg + kWinXchgBytes);   // B descriptors of band 0, per MMA
+  const uint32_t barBase = sbase + oXchg + kWinXchgBytes + kWinTabBytes;
   auto band_full = [&](int b) { return barBase + 8u * b; };
   auto band_empty = [&](int b) { return barBase + 16u + 8u * b; };
   auto acc_full = [&](int b) { return barBase + 32u + 8u * b; };
   auto acc_empty = [&](int b) { return barBase + 48u + 8u * b; };
-  const uint32_t done_bar = barBase + 64u;
-  uint32_t* tmem_slot = (uint32_t*)(smem + a.a_bytes + 2 * a.band_bytes + kWinXchgBytes + 80);
+  auto stage_full = [&](int b) { return barBase + 64u + 8u * b; };
+  const uint32_t done_bar = barBase + 80u;
+  uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + kWinXchgBytes + kWinTabBytes + 96);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // CTA c takes channel tile c % nct and the band tiles c / nct, c / nct + G / nct, ... of it
   const int ctile = (int)blockIdx.x % a.nct;
   const int first = (int)blockIdx.x / a.nct, step = (int)gridDim.x / a.nct;
   const int n_local = first < a.ntiles ? (a.ntiles - first + step - 1) / step : 0;
+  const int nmma = a.kc >> 1;
 
   if (warp == kWinMmaWarp) {
     tmem_alloc(smem_u32(tmem_slot), 512);
@@ -157,9 +189,18 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
       mbar_init(band_empty(b), 1);
       mbar_init(acc_full(b), 1);
       mbar_init(acc_empty(b), kWinEpiWarps);
+      mbar_init(stage_full(b), 1);
     }
     mbar_init(done_bar, 1);
     fence_mbar_init();
+  }
+  // B descriptors of band buffer 0, one per MMA: the pair of core columns (2q, 2q + 1); past the
+  // filter bytes (where A is zero) the second one is the slot after the first
+  if (tid < nmma) {
+    const int c0 = 2 * tid;
+    const uint32_t b0 = win_col_offset(a, c0);
+    const uint32_t b1 = c0 + 1 < a.kc_real ? win_col_offset(a, c0 + 1) : b0 + 16u;
+    mtab[tid] = sdesc_none(sBand + b0, b1 - b0, 128u);
   }
   grid_dep_wait();
   // The resident A operand: row m = (sy, nl) at 16-byte core column c = (iy, ix, p) holds bytes
@@ -194,61 +235,92 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
   grid_dep_launch();
 
   if (warp >= kWinProd0) {
-    // =================== producers: packed input rows -> e4m3 band in shared memory ===================
+    // =================== producers: bulk copy of packed rows, expansion into the band ===================
     const int pt = tid - kWinProd0 * 32;   // 0..127
     const int cinb = a.cin >> 2;           // packed bytes per pixel
-    const int items = a.rb * a.pitch * a.planes;
-    bool ok = true;
-#pragma unroll 1
-    for (int i = 0; i < n_local && ok; ++i) {
-      const int bb = i & 1;
-      if (!__all_sync(0xffffffffu, mbar_wait_backoff(band_empty(bb), ((uint32_t)(i >> 1) & 1u) ^ 1u, 64))) {
-        ok = false;
-        break;
-      }
+    const bool issuer = pt == 0;
+    const int items = a.rb * a.seg_pitch * a.planes;
+    // rows of tile i staged in buffer i & 1: segment s (row band of ry * s output rows below y0)
+    // holds input rows y0 + s ry - pad + iy, iy < rb, at (s rb + iy) row_bytes; rows outside the
+    // image are not copied (their slots expand to zeros)
+    auto issue = [&](int i) {
       const int t = first + i * step;
       const int b = (int)fdiv((uint32_t)t, a.div_bands);
       const int y0 = (t - b * a.bands) * a.rows;
-      const uint8_t* img = a.x + (size_t)b * a.h * a.w * cinb;
-      const uint32_t dst0 = sBand + (uint32_t)bb * a.band_bytes;
-#pragma unroll 1
-      for (int base = pt; base < items; base += 4 * 128) {
-        uint32_t v[4];
-        uint32_t dst[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int it = base + u * 128;
-          v[u] = 0u;
-          dst[u] = 0xFFFFFFFFu;
-          if (it < items) {
-            const int rest = (int)fdiv((uint32_t)it, a.div_planes);
-            const int p = it - rest * a.planes;
-            const int iy = (int)fdiv((uint32_t)rest, a.div_pitch);
-            const int slot = rest - iy * a.pitch;
-            const int xx = slot - a.pad, yy = y0 - a.pad + iy;
-            if (xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
-              v[u] = ld_codes4<false>(img + ((size_t)yy * a.w + xx) * cinb + 4 * p);
-            dst[u] = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.pitch + slot);
-          }
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          if (dst[u] != 0xFFFFFFFFu) {
-            const uint32_t w = v[u];
-            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst[u]), "r"(w & 0x03030303u),
-                         "r"((w >> 2) & 0x03030303u), "r"((w >> 4) & 0x03030303u), "r"((w >> 6) & 0x03030303u)
-                         : "memory");
-          }
-        }
+      const uint8_t* img = a.x + (size_t)b * a.h * a.row_bytes;
+      const uint32_t dst = sStage + (uint32_t)(i & 1) * a.stage_bytes;
+      uint32_t total = 0;
+      for (int s = 0; s < a.nseg; ++s) {
+        const int top = win_row(a, y0, s) - a.pad;
+        const int r0 = max(0, top), r1 = min(a.h, top + a.rb);
+        if (r1 > r0) total += (uint32_t)((r1 - r0) * a.row_bytes);
       }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(band_full(bb));
+      mbar_arrive_expect_tx(stage_full(i & 1), total);
+      for (int s = 0; s < a.nseg; ++s) {
+        const int top = win_row(a, y0, s) - a.pad;
+        const int r0 = max(0, top), r1 = min(a.h, top + a.rb);
+        if (r1 > r0)
+          bulk_copy_g2s(dst + (uint32_t)((s * a.rb + (r0 - top)) * a.row_bytes), img + (size_t)r0 * a.row_bytes,
+                        (uint32_t)((r1 - r0) * a.row_bytes), stage_full(i & 1));
+      }
+    };
+    int issued = 0, waited = 0;   // tiles whose copies were issued / were waited for
+    if (issuer && n_local > 0) {
+      issue(0);
+      issued = 1;
+    }
+    bool ok = true;
+#pragma unroll 1
+    for (int i = 0; i < n_local; ++i) {
+      const int bb = i & 1;
+      if (ok) {
+        if (issuer && i + 1 < n_local) {   // stage (i + 1) & 1 was read in iteration i - 1, fenced by the barrier
+          issue(i + 1);
+          issued = i + 2;
+        }
+        bool got = mbar_wait(stage_full(bb), (uint32_t)(i >> 1) & 1u);
+        if (got) waited = i + 1;
+        got = got && mbar_wait_backoff(band_empty(bb), ((uint32_t)(i >> 1) & 1u) ^ 1u, 64);
+        ok = __all_sync(0xffffffffu, got);
+      }
+      if (ok) {
+        const int t = first + i * step;
+        const int b = (int)fdiv((uint32_t)t, a.div_bands);
+        const int y0 = (t - b * a.bands) * a.rows;
+        const uint8_t* stg = smem + oStage + (size_t)bb * a.stage_bytes;
+        const uint32_t dst0 = sBand + (uint32_t)bb * a.band_bytes;
+#pragma unroll 4
+        for (int it = pt; it < items; it += 128) {
+          const int rest = (int)fdiv((uint32_t)it, a.div_planes);
+          const int p = it - rest * a.planes;
+          const int iy = (int)fdiv((uint32_t)rest, a.div_seg);
+          const int u = rest - iy * a.seg_pitch;
+          const int s = (int)fdiv((uint32_t)u, a.div_pitch);
+          const int slot = u - s * a.pitch;
+          const int xx = slot - a.pad, yy = win_row(a, y0, s) - a.pad + iy;
+          uint32_t v = 0u;
+          if (s < a.nseg && xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
+            v = *(const uint32_t*)(stg + (size_t)(s * a.rb + iy) * a.row_bytes + xx * cinb + 4 * p);
+          const uint32_t dst = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.seg_pitch + u);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(v & 0x03030303u),
+                       "r"((v >> 2) & 0x03030303u), "r"((v >> 4) & 0x03030303u), "r"((v >> 6) & 0x03030303u)
+                       : "memory");
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(band_full(bb));
+      }
+      // every producer warp is done with staging buffer bb before a copy into it is issued
+      named_bar(3, kWinProdWarps * 32);
+    }
+    // copies issued but never waited for (after a timed-out wait) land before the CTA may exit
+    if (issuer) {
+      for (int i = waited; i < issued; ++i) mbar_wait(stage_full(i & 1), (uint32_t)(i >> 1) & 1u);
     }
   } else if (warp == kWinMmaWarp) {
     // =================== MMA issue (one elected lane; the warp runs the loop) ===================
     const uint32_t idesc = idesc_e4m3_f32(128, a.N);
-    const int nmma = a.kc >> 1;
+    const uint64_t adesc0 = sdesc_none(sA, 2048u, 128u);
     bool ok = true;
 #pragma unroll 1
     for (int i = 0; i < n_local && ok; ++i) {
@@ -262,19 +334,11 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
       }
       tc_fence_after();
       if (elect_one()) {
-        const uint32_t band = sBand + (uint32_t)bb * a.band_bytes;
         const uint32_t dacc = tmem + (uint32_t)(bb * 256);
+        const uint64_t boff = (uint64_t)(((uint32_t)bb * a.band_bytes) >> 4);
 #pragma unroll 1
-        for (int q = 0; q < nmma; ++q) {
-          const int c0 = 2 * q;
-          const uint32_t b0 = win_col_addr(a, c0);
-          // the second core column: the next K column, or (past the filter bytes, where A is zero)
-          // the slot after the first
-          const uint32_t b1 = c0 + 1 < a.kc_real ? win_col_addr(a, c0 + 1) : b0 + 16u;
-          const uint64_t ad = sdesc_none(sA + (uint32_t)c0 * 2048u, 2048u, 128u);
-          const uint64_t bd = sdesc_none(band + b0, b1 - b0, 128u);
-          mma_e4m3(dacc, ad, bd, idesc, q > 0 ? 1u : 0u);
-        }
+        for (int q = 0; q < nmma; ++q)
+          mma_e4m3(dacc, adesc0 + (uint64_t)(q * 256), mtab[q] + boff, idesc, q > 0 ? 1u : 0u);
         mma_commit(band_empty(bb));
         mma_commit(acc_full(bb));
       }
@@ -310,7 +374,6 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     const int chb = (ctile * a.ct + cg * 32) >> 2;                 // this warp's byte within a pixel
     const uint32_t lane_off = (uint32_t)(32 * q) << 16;
     // row pairs of stacked output rows (ry > 1, pooled): the odd row's warp hands its codes over
-    const int partner_off = a.ct / 32;                             // quadrant distance of sy and sy + 1
     const int pair = a.ct == 32 ? (q >> 1) : (q & 1);
     const bool odd_row = (sy & 1) != 0;
     bool ok = true;
@@ -342,19 +405,19 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
                   k0 = m0;
                   k1 = m1;
                 }
-                if (a.y_acc) {
+                if constexpr (ACC != 0) {
                   const int j = 32 * g + 16 * h + c;
                   const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
-                  const int yy = y0 + r + sy;
-                  if (j < a.N && r < a.R && xx < a.w && yy < a.h)
+                  const int yy = win_row(a, y0, r) + sy;
+                  if (r < a.R && xx < a.w && yy < a.h)
                     a.y_acc[(((size_t)b * a.h + yy) * a.w + xx) * a.cout + n] = __float2int_rn(f * 512.0f);
                 }
               }
             }
             const int j = 32 * g + lane;
             const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
-            const int yy = y0 + r + sy;
-            if (a.y_codes && j < a.N && r < a.R && xx < a.w && yy < a.h) {
+            const int yy = win_row(a, y0, r) + sy;
+            if (a.y_codes && r < a.R && xx < a.w && yy < a.h) {
               const uint64_t codes = (spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1));
               *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = codes;
             }
@@ -373,7 +436,7 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
 #pragma unroll
               for (int h = 0; h < 4; ++h) {
                 // 8 pooled columns from 16 accumulator columns of a row (and of the next row when
-                // one output row per tile row: pitch % 16 == 0)
+                // one output row per M row: pitch % 16 == 0)
                 uint32_t v[16];
                 float mx[8];
                 const int pi0 = 32 * g + 8 * h;   // first pooled index of this chunk
@@ -420,25 +483,26 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
               if (32 * g < npool) xc[32 * g + lane] = own[g];
           }
           named_bar(1 + pair, 64);
-          if (!odd_row && ok) {
-            const int py = (y0 + sy) >> 1;
+          if (!odd_row && ok && a.y_codes) {
 #pragma unroll
             for (int g = 0; g < 4; ++g) {
-              const int px = 32 * g + lane;
-              if (32 * g < npool && px < pw && py < ph && a.y_codes) {
-                const uint64_t c = pool_codes2(own[g], xc[px], flip);
+              const int pi = 32 * g + lane;
+              const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
+              const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
+              if (pi < npool && r < a.R && px < pw && py < ph) {
+                const uint64_t c = pool_codes2(own[g], xc[pi], flip);
                 *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = c;
               }
             }
           }
-        } else if (ok) {
+        } else if (ok && a.y_codes) {
           const int half = a.pitch >> 1;
 #pragma unroll
           for (int g = 0; g < 4; ++g) {
             const int pi = 32 * g + lane;
             const int pr = pi / half, px = pi - pr * half;
             const int py = (y0 >> 1) + pr;
-            if (pi < npool && px < pw && py < ph && a.y_codes)
+            if (pi < npool && px < pw && py < ph)
               *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = own[g];
           }
         }

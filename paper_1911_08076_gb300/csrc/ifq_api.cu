@@ -200,9 +200,11 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
         set_attrs_gb<4, 4, 4>() != cudaSuccess || set_attrs_gb<16, 4, 2>() != cudaSuccess ||
         set_attrs_gb<8, 4, 2>() != cudaSuccess || set_attrs_gb<4, 4, 2>() != cudaSuccess)
       return IFQ_ECUDA;
-    if (cudaFuncSetAttribute(conv_win_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
+    if (cudaFuncSetAttribute(conv_win_kernel<0, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
             cudaSuccess ||
-        cudaFuncSetAttribute(conv_win_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
+        cudaFuncSetAttribute(conv_win_kernel<0, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(conv_win_kernel<1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
             cudaSuccess)
       return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
@@ -350,8 +352,9 @@ cudaError_t launch_narrow(int cin, int pool, int cout, dim3 grid, dim3 block, co
 // Geometry of the window kernel (conv_win.cuh) for a layer, or false where it does not apply:
 // 2-bit codes in and out, stride 1, k x k with "same" padding (k odd, <= 7), cin 16 or a multiple of
 // 32, cout 32, 64 or a multiple of 128 (at most one channel tile per SM), a fused pool of 2 on even
-// sizes or none, an output row of at most 256 anchors, and the resident filters plus two band
-// buffers within the shared memory of one CTA.  Fills every field but the pointers.
+// sizes or none, input rows of whole 16-byte units (the copy engine stages them), an output row of
+// at most 256 anchors, and the resident filters plus two staging and two band buffers within the
+// shared memory of one CTA.  Fills every field but the pointers.
 bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, size_t* smem) {
   if (env_int("IFQ_WIN", 1) == 0) return false;
   if (g.in8 || g.kb != 2) return false;
@@ -368,49 +371,61 @@ bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, s
   const bool pool = g.pool == 2;
   const int H = g.ho, W = g.wo;
   if (pool && ((H & 1) || (W & 1))) return false;
+  const int cinb = d->cin / 4;
+  const long long row_bytes = (long long)W * cinb;   // one input row, copied whole
+  if (row_bytes % 16 != 0) return false;
   const int ry = 128 / ct, planes = d->cin / 16;
-  int pitch, R, N;
-  if (ry > 1) {
-    pitch = W + k - 1;
-    R = 1;
-    N = (int)round_up((size_t)W, 16);
-    if (N > 256) return false;
-  } else {
-    pitch = W + k - 1;
-    if (pool) pitch = (int)round_up((size_t)pitch, 16);   // row pairs of the pool at aligned columns
-    if (pitch > 256) return false;
-    R = std::min(H, 256 / pitch);
-    if (pool) R &= ~1;
-    if (R < 1) return false;
-    N = (int)round_up((size_t)(R * pitch), 16);
-  }
-  const int rows = ry > 1 ? ry : R;
-  const int rb = rows + k - 1;
+  // anchor rows per tile: as many as fit N <= 256, fewer while the buffers exceed shared memory
+  const int pitch = ry == 1 && pool ? (int)round_up((size_t)(W + k - 1), 16) : W + k - 1;
+  if (pitch > 256) return false;
+  const int r_max = ry > 1 ? std::max(1, std::min(256 / pitch, ceil_div(H, ry))) : std::min(H, 256 / pitch);
   const int kc_real = (ry + k - 1) * k * planes;
   const int kc = (int)round_up((size_t)kc_real, 2);
-  // slots a plane needs: the band rows, and what the MMAs read past them (N anchors from the
-  // farthest tap, and the slot after the last core column), with slack
-  const int iy_max = ry + k - 2;
-  const int slots = std::max(rb * pitch, iy_max * pitch + (k - 1) + N + 2) + 4;
-  const uint32_t ps = (uint32_t)round_up((size_t)slots * 16, 128) + (planes > 1 ? 16u : 0u);
-  const uint32_t band_bytes = (uint32_t)round_up((size_t)planes * ps, 1024);
+  if (kc / 2 > kWinMaxMma) return false;
   const uint32_t a_bytes = (uint32_t)kc * 2048u;
-  const size_t need = 1024 + (size_t)a_bytes + 2 * (size_t)band_bytes + kWinXchgBytes + 128;
-  if (need > (size_t)kWinMaxSmem) return false;
+  int R = 0, seg_pitch = 0, rb = 0, N = 0, nseg = 0;
+  uint32_t ps = 0, band_bytes = 0, stage_bytes = 0;
+  size_t need = 0;
+  for (int r = r_max; r >= 1; --r) {
+    if (ry == 1 && pool && (r & 1)) continue;   // pooled row pairs
+    // ry > 1: r row bands of ry output rows side by side along N;
+    // ry = 1: r consecutive output rows sharing the band's input rows
+    const int sp = ry > 1 ? r * pitch : pitch;
+    const int rbr = ry > 1 ? ry + k - 1 : r + k - 1;
+    const int n_ = (int)round_up((size_t)((r - 1) * pitch + W), 16);   // the last row's padding is not an anchor
+    if (n_ > 256) continue;
+    const int ns = ry > 1 ? r : 1;
+    // slots a plane needs: the band rows, and what the MMAs read past them (N anchors from the
+    // farthest tap, and the slot after the last core column), with slack
+    const int iy_max = ry + k - 2;
+    const int slots = std::max(rbr * sp, iy_max * sp + (k - 1) + n_ + 2) + 4;
+    const uint32_t ps_ = (uint32_t)round_up((size_t)slots * 16, 128) + (planes > 1 ? 16u : 0u);
+    const uint32_t bb = (uint32_t)round_up((size_t)planes * ps_, 1024);
+    const uint32_t sb = (uint32_t)round_up((size_t)ns * rbr * row_bytes, 128);
+    const size_t nd = 1024 + (size_t)a_bytes + 2 * (size_t)bb + 2 * (size_t)sb + kWinXchgBytes + kWinTabBytes + 128;
+    if (nd <= (size_t)kWinMaxSmem) {
+      R = r; seg_pitch = sp; rb = rbr; N = n_; nseg = ns; ps = ps_; band_bytes = bb; stage_bytes = sb; need = nd;
+      break;
+    }
+  }
+  if (R == 0) return false;
   if (wa) {
     memset(wa, 0, sizeof(*wa));
     wa->n = d->n; wa->h = H; wa->w = W; wa->cin = d->cin; wa->cout = d->cout; wa->k = k; wa->pad = d->pad;
     wa->Kpad = g.Kpad;
-    wa->planes = planes; wa->ct = ct; wa->ry = ry; wa->nct = nct; wa->R = R; wa->rows = rows; wa->pitch = pitch;
+    wa->planes = planes; wa->ct = ct; wa->ry = ry; wa->nct = nct; wa->R = R; wa->rows = ry * R;
+    wa->pitch = pitch; wa->seg_pitch = seg_pitch; wa->nseg = nseg;
     wa->N = N; wa->rb = rb; wa->kc = kc; wa->kc_real = kc_real;
-    wa->bands = ceil_div(H, rows);
+    wa->bands = ceil_div(H, wa->rows);
     wa->ntiles = d->n * wa->bands;
-    wa->lpool = pool ? 1 : 0;
+    wa->row_bytes = (int)row_bytes;
     wa->plane_stride = ps;
     wa->band_bytes = band_bytes;
+    wa->stage_bytes = stage_bytes;
     wa->a_bytes = a_bytes;
     wa->div_planes = make_fastdiv((uint32_t)planes);
     wa->div_pitch = make_fastdiv((uint32_t)pitch);
+    wa->div_seg = make_fastdiv((uint32_t)seg_pitch);
     wa->div_bands = make_fastdiv((uint32_t)wa->bands);
   }
   if (smem) *smem = need;
@@ -638,8 +653,9 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     // CTAs come in groups of nct, one per channel tile, each group sharing the band tiles
     const int per = std::max(1, std::min(wa.ntiles, nsm / wa.nct));
     const dim3 grid((unsigned)(per * wa.nct)), block(kWinThreads);
-    e = wa.lpool ? launch_k(conv_win_kernel<1>, grid, block, smem, st, wa)
-                 : launch_k(conv_win_kernel<0>, grid, block, smem, st, wa);
+    if (g.pool == 2) e = launch_k(conv_win_kernel<1, 0>, grid, block, smem, st, wa);
+    else if (ya) e = launch_k(conv_win_kernel<0, 1>, grid, block, smem, st, wa);
+    else e = launch_k(conv_win_kernel<0, 0>, grid, block, smem, st, wa);
   } else if (path == IFQ_PATH_TC) {
     int bn = choose_bn(g, d->cout, nsm), ks = 1;
     const int gb = granule_bytes(d, g);

@@ -295,6 +295,7 @@ def test_window_path_plan():
     assert plan(64, 13, 13, 1024, 30, 1, 1, 0, out_mode=ifq.IFQ_OUT_ACC) == TC   # cout 30
     assert plan(4, 20, 20, 48, 64, 3, 1, 1) == TC                    # cin 48
     assert plan(4, 20, 20, 64, 96, 3, 1, 1) == TC                    # cout 96
+    assert plan(2, 10, 10, 16, 32, 3, 1, 1) == TC                    # a row of 40 bytes: no bulk copy
     assert plan(4, 20, 20, 64, 64, 3, 1, 1, path=WIN) == WIN
     assert plan(4, 20, 20, 64, 64, 3, 2, 1, path=WIN) == TC          # not applicable: tensor cores
     import os

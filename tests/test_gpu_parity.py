@@ -612,20 +612,22 @@ def test_graph_with_copies_rejects_bad_io():
 WIN_CASES = [
     # B, H, W, C, cout, k, pool, out_mode
     (1, 4, 16, 16, 32, 3, 1, 3),          # smallest: one tile of 4 rows x 16 anchors, 4 rows stacked on M
-    (2, 10, 10, 16, 32, 3, 1, 3),         # ragged band (10 rows in tiles of 4), N = 16 > w
+    (2, 10, 12, 16, 32, 3, 1, 3),         # ragged band (10 rows in tiles of 4), N = 16 > w
     (2, 12, 20, 16, 32, 3, 2, 1),         # fused pool, row pairs across warps
-    (2, 9, 13, 32, 64, 3, 1, 3),          # 2 planes, 2 rows stacked on M, odd sizes
+    (2, 9, 14, 32, 64, 3, 1, 3),          # 2 planes, 2 rows stacked on M, odd height
     (3, 14, 18, 32, 64, 3, 2, 1),         # fused pool over warp pairs (sy, sy + 1)
     (2, 11, 11, 64, 128, 3, 1, 3),        # one output row per M row, several anchor rows per tile
     (2, 12, 14, 64, 128, 3, 2, 1),        # fused pool over anchor-row pairs (16-aligned pitch)
     (2, 9, 9, 64, 256, 3, 1, 3),          # two channel tiles
     (1, 16, 16, 64, 64, 3, 1, 3),         # the single PR1 layer shape
     (2, 8, 30, 32, 128, 5, 1, 3),         # 5 x 5, 7 anchor rows of 34 slots
-    (2, 6, 9, 96, 64, 3, 1, 3),           # 6 planes
+    (2, 6, 10, 96, 64, 3, 1, 3),          # 6 planes
     (2, 7, 12, 128, 128, 1, 1, 3),        # 1 x 1
     (1, 6, 40, 16, 32, 7, 1, 1),          # 7 x 7
-    (2, 26, 26, 16, 32, 3, 2, 1),         # H % 4 != 0 with the pool: the last band's rows past h
+    (2, 26, 28, 16, 32, 3, 2, 1),         # H % 4 != 0 with the pool: the last band's rows past h
     (1, 3, 208, 16, 32, 3, 1, 1),         # a full Tiny-YOLO row (N = 208)
+    (3, 20, 52, 32, 64, 3, 2, 1),         # 4 row bands side by side along N, fused pool
+    (2, 13, 56, 64, 64, 3, 1, 3),         # 4 row bands of 2 rows along N (ResNet stage-1 width), ragged
 ]
 
 
