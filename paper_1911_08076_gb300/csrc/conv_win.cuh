@@ -50,8 +50,9 @@
 // rows), combined as codes: code(max A) is the max of the codes for a
 // positive BN scale and the min for a negative one.
 //
-// Warps: 0-3 epilogue (lane quadrant = warp), 4 TMEM allocation and MMA
-// issue, 5-8 producers (one lane of warp 5 issues the bulk copies).  Two
+// Warps: 0-7 epilogue (lane quadrant = warp % 4, two warps a quadrant on
+// alternate column groups), 8 TMEM allocation and MMA issue, 9-12 producers
+// (one lane of warp 9 issues the bulk copies).  Two
 // staging buffers, two bands and two accumulators, so the copy of tile i+2,
 // the expansion of tile i+1, the MMAs of tile i and the epilogue of tile i-1
 // overlap.  Every wait is bounded (IFQ_ETIMEOUT, then the roles leave their
@@ -61,11 +62,12 @@
 
 namespace ifq {
 
-constexpr int kWinEpiWarps = 4;
-constexpr int kWinMmaWarp = 4;
-constexpr int kWinProd0 = 5;
+constexpr int kWinEpiWarps = 8;        // two per tensor-memory lane quadrant, alternate column groups
+constexpr int kWinMmaWarp = 8;
+constexpr int kWinProd0 = 9;
 constexpr int kWinProdWarps = 4;
-constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 288
+constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 416
+constexpr int kWinProdBar = 5;         // named barrier of the producer warps (1-4: epilogue row pairs)
 constexpr int kWinXchgBytes = 4096;    // pooled codes passed between the two warps of a row pair
 constexpr int kWinMaxMma = 64;         // MMAs per tile (K' / 32)
 constexpr int kWinTabBytes = 8 * kWinMaxMma;
@@ -115,6 +117,41 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uin
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
                "l"(src), "r"(bytes), "r"(bar)
                : "memory");
+}
+
+// 32 lanes x 32 consecutive columns of tensor memory -> 32 registers, with the wait in the same
+// asm statement (the destination registers are written asynchronously until the wait).
+__device__ __forceinline__ void tmem_ld32_sync(uint32_t t0, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(t0)
+      : "memory");
+}
+
+// Two loads of 32 columns (at t0 and t1) in flight together, one wait: 64 registers.
+__device__ __forceinline__ void tmem_ld2x32_sync(uint32_t t0, uint32_t t1, uint32_t (&v)[64]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31]), "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]), "=r"(v[37]), "=r"(v[38]), "=r"(v[39]), "=r"(v[40]), "=r"(v[41]), "=r"(v[42]), "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]), "=r"(v[48]), "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]), "=r"(v[55]), "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]), "=r"(v[61]), "=r"(v[62]), "=r"(v[63])
+      : "r"(t0), "r"(t1)
+      : "memory");
+}
+
+// Four loads of 16 columns (at t0..t3) in flight together, one wait: 64 registers.
+__device__ __forceinline__ void tmem_ld4x16_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, uint32_t (&v)[64]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%65];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [%66];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%67];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31]), "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]), "=r"(v[37]), "=r"(v[38]), "=r"(v[39]), "=r"(v[40]), "=r"(v[41]), "=r"(v[42]), "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]), "=r"(v[48]), "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]), "=r"(v[55]), "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]), "=r"(v[61]), "=r"(v[62]), "=r"(v[63])
+      : "r"(t0), "r"(t1), "r"(t2), "r"(t3)
+      : "memory");
 }
 
 // 32 bits -> 64 bits with bit i at bit 2i.
@@ -206,21 +243,27 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
   // The resident A operand: row m = (sy, nl) at 16-byte core column c = (iy, ix, p) holds bytes
   // [16p, 16p + 16) of tap (iy - sy, ix) of filter n, or zeros.  Layout: core column c, row group
   // m / 8, row m % 8 -> c * 2048 + (m / 8) * 128 + (m % 8) * 16.
-  for (int it = tid; it < 128 * a.kc; it += kWinThreads) {
-    const int c = it >> 7, m = it & 127;
-    const int sy = m / a.ct, nl = m - sy * a.ct;
-    const int n = ctile * a.ct + nl;
-    const uint8_t* src = a.w_prep;
-    uint32_t bytes = 0;
-    if (c < a.kc_real) {
-      const int p = c % a.planes, t = c / a.planes;
-      const int iy = t / a.k, ix = t - iy * a.k, dy = iy - sy;
-      if (dy >= 0 && dy < a.k) {
-        src = a.w_prep + (size_t)n * a.Kpad + (size_t)((dy * a.k + ix) * a.cin + 16 * p);
-        bytes = 16;
+  // Copies of 16 bytes, a warp taking 8 rows x 4 consecutive core columns: 8 runs of 64 contiguous
+  // bytes of the prepared rows, and 4 x 128 contiguous bytes of shared memory.
+  {
+    const int kcq = (a.kc + 3) >> 2;
+    for (int wi = warp; wi < 16 * kcq; wi += kWinThreads / 32) {
+      const int m = (wi & 15) * 8 + (lane & 7), c = (wi >> 4) * 4 + (lane >> 3);
+      if (c >= a.kc) continue;
+      const int sy = m / a.ct, nl = m - sy * a.ct;
+      const int n = ctile * a.ct + nl;
+      const uint8_t* src = a.w_prep;
+      uint32_t bytes = 0;
+      if (c < a.kc_real) {
+        const int p = c % a.planes, t = c / a.planes;
+        const int iy = t / a.k, ix = t - iy * a.k, dy = iy - sy;
+        if (dy >= 0 && dy < a.k) {
+          src = a.w_prep + (size_t)n * a.Kpad + (size_t)((dy * a.k + ix) * a.cin + 16 * p);
+          bytes = 16;
+        }
       }
+      cp_async_16(sA + (uint32_t)c * 2048u + (uint32_t)(m >> 3) * 128u + (uint32_t)(m & 7) * 16u, src, bytes);
     }
-    cp_async_16(sA + (uint32_t)c * 2048u + (uint32_t)(m >> 3) * 128u + (uint32_t)(m & 7) * 16u, src, bytes);
   }
   cp_async_commit();
   // both band buffers start as zeros: padding slots and the tail past the band stay zero
@@ -288,30 +331,42 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
         const int b = (int)fdiv((uint32_t)t, a.div_bands);
         const int y0 = (t - b * a.bands) * a.rows;
         const uint8_t* stg = smem + oStage + (size_t)bb * a.stage_bytes;
-        const uint32_t dst0 = sBand + (uint32_t)bb * a.band_bytes;
-#pragma unroll 4
-        for (int it = pt; it < items; it += 128) {
-          const int rest = (int)fdiv((uint32_t)it, a.div_planes);
-          const int p = it - rest * a.planes;
-          const int iy = (int)fdiv((uint32_t)rest, a.div_seg);
-          const int u = rest - iy * a.seg_pitch;
-          const int s = (int)fdiv((uint32_t)u, a.div_pitch);
-          const int slot = u - s * a.pitch;
-          const int xx = slot - a.pad, yy = win_row(a, y0, s) - a.pad + iy;
-          uint32_t v = 0u;
-          if (s < a.nseg && xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
-            v = *(const uint32_t*)(stg + (size_t)(s * a.rb + iy) * a.row_bytes + xx * cinb + 4 * p);
-          const uint32_t dst = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.seg_pitch + u);
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(v & 0x03030303u),
-                       "r"((v >> 2) & 0x03030303u), "r"((v >> 4) & 0x03030303u), "r"((v >> 6) & 0x03030303u)
-                       : "memory");
+        const uint32_t dst0 = a.a_bytes + (uint32_t)bb * a.band_bytes;   // byte offset from smem
+        // batches of 8 items a thread: all staging loads first, then the 16-byte band stores
+#pragma unroll 1
+        for (int base = pt; base < items; base += 8 * 128) {
+          uint32_t v[8];
+          uint32_t dst[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int it = base + e * 128;
+            v[e] = 0u;
+            dst[e] = 0xFFFFFFFFu;
+            if (it < items) {
+              const int rest = (int)fdiv((uint32_t)it, a.div_planes);
+              const int p = it - rest * a.planes;
+              const int iy = (int)fdiv((uint32_t)rest, a.div_seg);
+              const int u = rest - iy * a.seg_pitch;
+              const int s = (int)fdiv((uint32_t)u, a.div_pitch);
+              const int slot = u - s * a.pitch;
+              const int xx = slot - a.pad, yy = win_row(a, y0, s) - a.pad + iy;
+              if (s < a.nseg && xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
+                v[e] = *(const uint32_t*)(stg + (size_t)(s * a.rb + iy) * a.row_bytes + xx * cinb + 4 * p);
+              dst[e] = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.seg_pitch + u);
+            }
+          }
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            if (dst[e] != 0xFFFFFFFFu)
+              *(uint4*)(smem + dst[e]) = make_uint4(v[e] & 0x03030303u, (v[e] >> 2) & 0x03030303u,
+                                                    (v[e] >> 4) & 0x03030303u, (v[e] >> 6) & 0x03030303u);
         }
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(band_full(bb));
       }
       // every producer warp is done with staging buffer bb before a copy into it is issued
-      named_bar(3, kWinProdWarps * 32);
+      named_bar(kWinProdBar, kWinProdWarps * 32);
     }
     // copies issued but never waited for (after a timed-out wait) land before the CTA may exit
     if (issuer) {
@@ -348,7 +403,10 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     __syncwarp();
   } else {
     // =================== epilogue: thresholds, code packing, fused pool, stores ===================
-    const int q = warp;                          // lane quadrant
+    // Warps q and q + 4 share lane quadrant q (warp % 4) and take alternate 32-column (pooled: 32
+    // pooled-column) groups, so each quadrant has two warps hiding each other's latencies.
+    const int q = warp & 3;                      // lane quadrant
+    const int half = warp >> 2;                  // which of the alternate column groups
     const int sy = (32 * q) / a.ct;              // output row offset of this quadrant
     const int cg = ((32 * q) % a.ct) >> 5;       // 32-channel group within the channel tile
     const int n = ctile * a.ct + cg * 32 + lane;
@@ -376,6 +434,20 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     // row pairs of stacked output rows (ry > 1, pooled): the odd row's warp hands its codes over
     const int pair = a.ct == 32 ? (q >> 1) : (q & 1);
     const bool odd_row = (sy & 1) != 0;
+    // the codes of one value against the three thresholds: ballots of bit 1 and of the parity of
+    // the three compares, collected by the lane whose index is the column's within its group
+    auto code_ballot = [&](float f, int col, uint32_t& k0, uint32_t& k1) {
+      const bool p1 = f > t1, p2 = f > t2, p3 = f > t3;
+      const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
+      const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
+      if (lane == col) {
+        k0 = m0;
+        k1 = m1;
+      }
+    };
+    auto packed = [&](uint32_t k0, uint32_t k1) {
+      return spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1);
+    };
     bool ok = true;
 #pragma unroll 1
     for (int i = 0; i < n_local; ++i) {
@@ -389,88 +461,75 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
       if constexpr (POOL == 0) {
         if (ok) {
 #pragma unroll 1
-          for (int g = 0; g * 32 < a.N; ++g) {
+          for (int g = half; g * 32 < a.N; g += 2) {
+            uint32_t v[32];
+            tmem_ld32_sync(tacc + (uint32_t)(32 * g), v);
             uint32_t k0 = 0, k1 = 0;
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              uint32_t v[16];
-              tmem_ld16_sync(tacc + (uint32_t)(32 * g + 16 * h), v);
-#pragma unroll
-              for (int c = 0; c < 16; ++c) {
-                const float f = __uint_as_float(v[c]);
-                const bool p1 = f > t1, p2 = f > t2, p3 = f > t3;
-                const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
-                const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
-                if (lane == 16 * h + c) {
-                  k0 = m0;
-                  k1 = m1;
-                }
-                if constexpr (ACC != 0) {
-                  const int j = 32 * g + 16 * h + c;
-                  const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
-                  const int yy = win_row(a, y0, r) + sy;
-                  if (r < a.R && xx < a.w && yy < a.h)
-                    a.y_acc[(((size_t)b * a.h + yy) * a.w + xx) * a.cout + n] = __float2int_rn(f * 512.0f);
-                }
+            for (int c = 0; c < 32; ++c) {
+              const float f = __uint_as_float(v[c]);
+              code_ballot(f, c, k0, k1);
+              if constexpr (ACC != 0) {
+                const int j = 32 * g + c;
+                const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
+                const int yy = win_row(a, y0, r) + sy;
+                if (r < a.R && xx < a.w && yy < a.h)
+                  a.y_acc[(((size_t)b * a.h + yy) * a.w + xx) * a.cout + n] = __float2int_rn(f * 512.0f);
               }
             }
             const int j = 32 * g + lane;
             const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
             const int yy = win_row(a, y0, r) + sy;
-            if (a.y_codes && r < a.R && xx < a.w && yy < a.h) {
-              const uint64_t codes = (spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1));
-              *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = codes;
-            }
+            if (a.y_codes && r < a.R && xx < a.w && yy < a.h)
+              *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = packed(k0, k1);
           }
         }
       } else {
-        // pooled output map: (h / 2) x (w / 2)
+        // pooled output map: (h / 2) x (w / 2); groups of 32 pooled columns, alternate ones per warp
         const int pw = a.w >> 1, ph = a.h >> 1;
-        uint64_t own[4] = {0ull, 0ull, 0ull, 0ull};
-        const int npool = a.ry > 1 ? (a.N >> 1) : (a.R >> 1) * (a.pitch >> 1);
+        const int halfw = a.pitch >> 1;
+        const int npool = a.ry > 1 ? (a.N >> 1) : (a.R >> 1) * halfw;
+        uint64_t own[2] = {0ull, 0ull};
         if (ok) {
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
+          for (int gi = 0; gi < 2; ++gi) {
+            const int g = 2 * gi + half;
             if (32 * g < npool) {
               uint32_t k0 = 0, k1 = 0;
+              if (a.ry > 1) {
+                // pooled column pi <- columns 2 pi, 2 pi + 1 of this row
+                uint32_t v[64];
+                tmem_ld2x32_sync(tacc + (uint32_t)(64 * g), tacc + (uint32_t)(64 * g + 32), v);
 #pragma unroll
-              for (int h = 0; h < 4; ++h) {
-                // 8 pooled columns from 16 accumulator columns of a row (and of the next row when
-                // one output row per M row: pitch % 16 == 0)
-                uint32_t v[16];
-                float mx[8];
-                const int pi0 = 32 * g + 8 * h;   // first pooled index of this chunk
-                if (pi0 >= npool) {
+                for (int e = 0; e < 32; ++e)
+                  code_ballot(fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1])), e, k0, k1);
+              } else {
+                // pooled column (pr, px) <- columns 2 px, 2 px + 1 of anchor rows 2 pr and 2 pr + 1
+                // (pitch % 16 == 0, so 8 pooled columns are 16 aligned columns of each row)
 #pragma unroll
-                  for (int e = 0; e < 8; ++e) mx[e] = 0.f;
-                } else if (a.ry > 1) {
-                  tmem_ld16_sync(tacc + (uint32_t)(2 * pi0), v);
+                for (int hh = 0; hh < 2; ++hh) {
+                  uint32_t col[2];
 #pragma unroll
-                  for (int e = 0; e < 8; ++e) mx[e] = fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-                } else {
-                  const int half = a.pitch >> 1;
-                  const int pr = pi0 / half, px0 = pi0 - pr * half;
-                  const uint32_t col = (uint32_t)(2 * pr * a.pitch + 2 * px0);
-                  tmem_ld16_sync(tacc + col, v);
-#pragma unroll
-                  for (int e = 0; e < 8; ++e) mx[e] = fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
-                  tmem_ld16_sync(tacc + col + (uint32_t)a.pitch, v);
-#pragma unroll
-                  for (int e = 0; e < 8; ++e)
-                    mx[e] = fmaxf(mx[e], fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1])));
-                }
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                  const bool p1 = mx[e] > t1, p2 = mx[e] > t2, p3 = mx[e] > t3;
-                  const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
-                  const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
-                  if (lane == 8 * h + e) {
-                    k0 = m0;
-                    k1 = m1;
+                  for (int u = 0; u < 2; ++u) {
+                    const int pi0 = 32 * g + 16 * hh + 8 * u;
+                    const int pr = pi0 / halfw, px0 = pi0 - pr * halfw;
+                    col[u] = pi0 < npool ? (uint32_t)(2 * pr * a.pitch + 2 * px0) : 0u;
                   }
+                  uint32_t v[64];
+                  tmem_ld4x16_sync(tacc + col[0], tacc + col[0] + (uint32_t)a.pitch, tacc + col[1],
+                                   tacc + col[1] + (uint32_t)a.pitch, v);
+#pragma unroll
+                  for (int u = 0; u < 2; ++u)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                      const float top = fmaxf(__uint_as_float(v[32 * u + 2 * e]), __uint_as_float(v[32 * u + 2 * e + 1]));
+                      const float bot =
+                          fmaxf(__uint_as_float(v[32 * u + 16 + 2 * e]), __uint_as_float(v[32 * u + 16 + 2 * e + 1]));
+                      code_ballot(fmaxf(top, bot), 16 * hh + 8 * u + e, k0, k1);
+                    }
                 }
               }
-              own[g] = spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1);
+              own[gi] = packed(k0, k1);
             }
           }
         }
@@ -479,31 +538,31 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
           uint64_t* xc = xchg + (size_t)((i & 1) * 2 + pair) * 128;
           if (odd_row) {
 #pragma unroll
-            for (int g = 0; g < 4; ++g)
-              if (32 * g < npool) xc[32 * g + lane] = own[g];
+            for (int gi = 0; gi < 2; ++gi) {
+              const int g = 2 * gi + half;
+              if (32 * g < npool) xc[32 * g + lane] = own[gi];
+            }
           }
-          named_bar(1 + pair, 64);
+          named_bar(1 + pair + 2 * half, 64);
           if (!odd_row && ok && a.y_codes) {
 #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-              const int pi = 32 * g + lane;
+            for (int gi = 0; gi < 2; ++gi) {
+              const int pi = 32 * (2 * gi + half) + lane;
               const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
               const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
-              if (pi < npool && r < a.R && px < pw && py < ph) {
-                const uint64_t c = pool_codes2(own[g], xc[pi], flip);
-                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = c;
-              }
+              if (pi < npool && r < a.R && px < pw && py < ph)
+                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) =
+                    pool_codes2(own[gi], xc[pi], flip);
             }
           }
         } else if (ok && a.y_codes) {
-          const int half = a.pitch >> 1;
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            const int pi = 32 * g + lane;
-            const int pr = pi / half, px = pi - pr * half;
+          for (int gi = 0; gi < 2; ++gi) {
+            const int pi = 32 * (2 * gi + half) + lane;
+            const int pr = pi / halfw, px = pi - pr * halfw;
             const int py = (y0 >> 1) + pr;
             if (pi < npool && px < pw && py < ph)
-              *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = own[g];
+              *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = own[gi];
           }
         }
       }
