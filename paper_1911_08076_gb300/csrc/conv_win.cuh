@@ -50,9 +50,9 @@
 // rows), combined as codes: code(max A) is the max of the codes for a
 // positive BN scale and the min for a negative one.
 //
-// Warps: 0-7 epilogue (lane quadrant = warp % 4, two warps a quadrant on
-// alternate column groups), 8 TMEM allocation and MMA issue, 9-12 producers
-// (one lane of warp 9 issues the bulk copies).  Two
+// Warps: 0-15 epilogue (lane quadrant = warp % 4, four warps a quadrant on
+// interleaved column groups), 16 TMEM allocation and MMA issue, 17-20
+// producers (one lane of warp 17 issues the bulk copies).  Two
 // staging buffers, two bands and two accumulators, so the copy of tile i+2,
 // the expansion of tile i+1, the MMAs of tile i and the epilogue of tile i-1
 // overlap.  Every wait is bounded (IFQ_ETIMEOUT, then the roles leave their
@@ -62,12 +62,15 @@
 
 namespace ifq {
 
-constexpr int kWinEpiWarps = 8;        // two per tensor-memory lane quadrant, alternate column groups
-constexpr int kWinMmaWarp = 8;
-constexpr int kWinProd0 = 9;
+constexpr int kWinEpiPerQ = 4;         // epilogue warps per tensor-memory lane quadrant
+constexpr int kWinEpiWarps = 4 * kWinEpiPerQ;
+constexpr int kWinMmaWarp = kWinEpiWarps;
+constexpr int kWinProd0 = kWinEpiWarps + 1;
 constexpr int kWinProdWarps = 4;
-constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 416
-constexpr int kWinProdBar = 5;         // named barrier of the producer warps (1-4: epilogue row pairs)
+constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 672
+constexpr int kWinPoolGroups = 4;      // groups of 32 pooled columns a tile can have (N <= 256)
+constexpr int kWinGpw = (kWinPoolGroups + kWinEpiPerQ - 1) / kWinEpiPerQ;   // of them per epilogue warp
+constexpr int kWinProdBar = 1 + 2 * kWinEpiPerQ;   // producers' named barrier (1..2 kWinEpiPerQ: row pairs)
 constexpr int kWinXchgBytes = 4096;    // pooled codes passed between the two warps of a row pair
 constexpr int kWinMaxMma = 64;         // MMAs per tile (K' / 32)
 constexpr int kWinTabBytes = 8 * kWinMaxMma;
@@ -101,7 +104,7 @@ struct WinArgs {
   uint32_t band_bytes;     // bytes of one band buffer
   uint32_t stage_bytes;    // bytes of one staging buffer (nseg * rb * row_bytes, rounded)
   uint32_t a_bytes;        // bytes of the resident A operand (kc * 2048)
-  FastDiv div_planes, div_pitch, div_seg, div_bands;
+  FastDiv div_planes, div_pitch, div_seg, div_bands, div_chunks, div_rb;
 };
 
 // Shared-memory descriptor of a K-major operand in the non-swizzled layout: core matrices of
@@ -282,7 +285,6 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     const int pt = tid - kWinProd0 * 32;   // 0..127
     const int cinb = a.cin >> 2;           // packed bytes per pixel
     const bool issuer = pt == 0;
-    const int items = a.rb * a.seg_pitch * a.planes;
     // rows of tile i staged in buffer i & 1: segment s (row band of ry * s output rows below y0)
     // holds input rows y0 + s ry - pad + iy, iy < rb, at (s rb + iy) row_bytes; rows outside the
     // image are not copied (their slots expand to zeros)
@@ -332,34 +334,32 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
         const int y0 = (t - b * a.bands) * a.rows;
         const uint8_t* stg = smem + oStage + (size_t)bb * a.stage_bytes;
         const uint32_t dst0 = a.a_bytes + (uint32_t)bb * a.band_bytes;   // byte offset from smem
-        // batches of 8 items a thread: all staging loads first, then the 16-byte band stores
-#pragma unroll 1
-        for (int base = pt; base < items; base += 8 * 128) {
-          uint32_t v[8];
-          uint32_t dst[8];
+        // Row items: band row iy of row band s, 16 staged bytes (4 words) a thread.  A row inside
+        // the image expands its words into their slots; a row outside it writes zeros into the
+        // slots of its w pixels (the padding slots beside the rows are never written and stay
+        // zero from the start).
+        const int chunks = a.row_bytes >> 4;
+        const int total = a.nseg * a.rb * chunks;
+#pragma unroll 2
+        for (int it = pt; it < total; it += 128) {
+          const int row = (int)fdiv((uint32_t)it, a.div_chunks);   // staged row s rb + iy
+          const int ch = it - row * chunks;
+          const int s = (int)fdiv((uint32_t)row, a.div_rb);
+          const int iy = row - s * a.rb;
+          const int yy = win_row(a, y0, s) - a.pad + iy;
+          uint4 w4 = make_uint4(0u, 0u, 0u, 0u);
+          if (yy >= 0 && yy < a.h) w4 = *(const uint4*)(stg + (size_t)row * a.row_bytes + 16 * ch);
+          const uint32_t ws[4] = {w4.x, w4.y, w4.z, w4.w};
+          const uint32_t rowo = dst0 + 16u * (uint32_t)(iy * a.seg_pitch + s * a.pitch + a.pad);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int it = base + e * 128;
-            v[e] = 0u;
-            dst[e] = 0xFFFFFFFFu;
-            if (it < items) {
-              const int rest = (int)fdiv((uint32_t)it, a.div_planes);
-              const int p = it - rest * a.planes;
-              const int iy = (int)fdiv((uint32_t)rest, a.div_seg);
-              const int u = rest - iy * a.seg_pitch;
-              const int s = (int)fdiv((uint32_t)u, a.div_pitch);
-              const int slot = u - s * a.pitch;
-              const int xx = slot - a.pad, yy = win_row(a, y0, s) - a.pad + iy;
-              if (s < a.nseg && xx >= 0 && xx < a.w && yy >= 0 && yy < a.h)
-                v[e] = *(const uint32_t*)(stg + (size_t)(s * a.rb + iy) * a.row_bytes + xx * cinb + 4 * p);
-              dst[e] = dst0 + (uint32_t)p * a.plane_stride + 16u * (uint32_t)(iy * a.seg_pitch + u);
-            }
+          for (int e = 0; e < 4; ++e) {
+            const int qw = 4 * ch + e;                               // word of the row
+            const int xx = (int)fdiv((uint32_t)qw, a.div_planes);   // its pixel
+            const int pl = qw - xx * a.planes;                      // and plane
+            const uint32_t v = ws[e];
+            *(uint4*)(smem + rowo + (uint32_t)pl * a.plane_stride + 16u * (uint32_t)xx) =
+                make_uint4(v & 0x03030303u, (v >> 2) & 0x03030303u, (v >> 4) & 0x03030303u, (v >> 6) & 0x03030303u);
           }
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (dst[e] != 0xFFFFFFFFu)
-              *(uint4*)(smem + dst[e]) = make_uint4(v[e] & 0x03030303u, (v[e] >> 2) & 0x03030303u,
-                                                    (v[e] >> 4) & 0x03030303u, (v[e] >> 6) & 0x03030303u);
         }
         fence_proxy_async_smem();
         __syncwarp();
@@ -403,10 +403,11 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     __syncwarp();
   } else {
     // =================== epilogue: thresholds, code packing, fused pool, stores ===================
-    // Warps q and q + 4 share lane quadrant q (warp % 4) and take alternate 32-column (pooled: 32
-    // pooled-column) groups, so each quadrant has two warps hiding each other's latencies.
+    // Warps q, q + 4, q + 8, ... share lane quadrant q (warp % 4) and take every kWinEpiPerQ-th
+    // 32-column (pooled: 32 pooled-column) group, so each quadrant has several warps hiding each
+    // other's latencies.
     const int q = warp & 3;                      // lane quadrant
-    const int half = warp >> 2;                  // which of the alternate column groups
+    const int sub = warp >> 2;                   // which of the quadrant's column groups
     const int sy = (32 * q) / a.ct;              // output row offset of this quadrant
     const int cg = ((32 * q) % a.ct) >> 5;       // 32-channel group within the channel tile
     const int n = ctile * a.ct + cg * 32 + lane;
@@ -461,7 +462,7 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
       if constexpr (POOL == 0) {
         if (ok) {
 #pragma unroll 1
-          for (int g = half; g * 32 < a.N; g += 2) {
+          for (int g = sub; g * 32 < a.N; g += kWinEpiPerQ) {
             uint32_t v[32];
             tmem_ld32_sync(tacc + (uint32_t)(32 * g), v);
             uint32_t k0 = 0, k1 = 0;
@@ -489,11 +490,13 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
         const int pw = a.w >> 1, ph = a.h >> 1;
         const int halfw = a.pitch >> 1;
         const int npool = a.ry > 1 ? (a.N >> 1) : (a.R >> 1) * halfw;
-        uint64_t own[2] = {0ull, 0ull};
+        uint64_t own[kWinGpw];
+#pragma unroll
+        for (int gi = 0; gi < kWinGpw; ++gi) own[gi] = 0ull;
         if (ok) {
 #pragma unroll
-          for (int gi = 0; gi < 2; ++gi) {
-            const int g = 2 * gi + half;
+          for (int gi = 0; gi < kWinGpw; ++gi) {
+            const int g = kWinEpiPerQ * gi + sub;
             if (32 * g < npool) {
               uint32_t k0 = 0, k1 = 0;
               if (a.ry > 1) {
@@ -538,16 +541,16 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
           uint64_t* xc = xchg + (size_t)((i & 1) * 2 + pair) * 128;
           if (odd_row) {
 #pragma unroll
-            for (int gi = 0; gi < 2; ++gi) {
-              const int g = 2 * gi + half;
+            for (int gi = 0; gi < kWinGpw; ++gi) {
+              const int g = kWinEpiPerQ * gi + sub;
               if (32 * g < npool) xc[32 * g + lane] = own[gi];
             }
           }
-          named_bar(1 + pair + 2 * half, 64);
+          named_bar(1 + pair + 2 * sub, 64);
           if (!odd_row && ok && a.y_codes) {
 #pragma unroll
-            for (int gi = 0; gi < 2; ++gi) {
-              const int pi = 32 * (2 * gi + half) + lane;
+            for (int gi = 0; gi < kWinGpw; ++gi) {
+              const int pi = 32 * (kWinEpiPerQ * gi + sub) + lane;
               const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
               const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
               if (pi < npool && r < a.R && px < pw && py < ph)
@@ -557,8 +560,8 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
           }
         } else if (ok && a.y_codes) {
 #pragma unroll
-          for (int gi = 0; gi < 2; ++gi) {
-            const int pi = 32 * (2 * gi + half) + lane;
+          for (int gi = 0; gi < kWinGpw; ++gi) {
+            const int pi = 32 * (kWinEpiPerQ * gi + sub) + lane;
             const int pr = pi / halfw, px = pi - pr * halfw;
             const int py = (y0 >> 1) + pr;
             if (pi < npool && px < pw && py < ph)

@@ -427,6 +427,8 @@ bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, s
     wa->div_pitch = make_fastdiv((uint32_t)pitch);
     wa->div_seg = make_fastdiv((uint32_t)seg_pitch);
     wa->div_bands = make_fastdiv((uint32_t)wa->bands);
+    wa->div_chunks = make_fastdiv((uint32_t)(row_bytes / 16));
+    wa->div_rb = make_fastdiv((uint32_t)rb);
   }
   if (smem) *smem = need;
   return true;
