@@ -216,12 +216,14 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
 /*
  * The kernel path ifq_conv2bit takes for `d` (host; reads IFQ_FORCE_PATH as
  * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT or
- * IFQ_PATH_WIN.  The window path (the default where it applies) serves
- * stride-1 k x k layers with "same" padding (k odd, <= 7) on 2-bit codes with
- * cin 16 or a multiple of 32, cout 32, 64 or a multiple of 128, no pool or a
- * 2 x 2 pool on even sizes, output rows of at most 256 pixels, and a filter
- * bank that stays resident in one CTA's shared memory; a request for it
- * elsewhere takes the tensor-core path.  The
+ * IFQ_PATH_WIN.  The window path serves stride-1 k x k layers with "same"
+ * padding (k odd, <= 7) on 2-bit codes with cin 16 or a multiple of 32, cout
+ * 32, 64 or a multiple of 128, no pool or a 2 x 2 pool on even sizes, input
+ * rows of whole 16-byte units, output rows of at most 256 pixels, and a
+ * filter bank that stays resident in one CTA's shared memory; it is the
+ * default for such layers with a fused 2 x 2 pool and cin <= 64 (where it was
+ * measured faster), and a request for it elsewhere takes the tensor-core
+ * path.  The
  * tensor-core path needs (2^k - 1)*K <= 196608 (the accumulator range checked
  * exact on the fp8 tensor cores; 255*K for 8-bit inputs), kh, kw <= 32, and
  * for k = 3, 4 cin % 8 == 0; a request for it outside that range takes the

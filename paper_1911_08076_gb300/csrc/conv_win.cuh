@@ -23,7 +23,8 @@
 // with 128 / cout output rows stacked along M a layer with few channels still
 // fills the 128 lanes of the MMA.  The prepared filter rows (ifq_pack_weights:
 // e4m3 +-1, natural (dy, dx, c) order with the intra-word order of the code
-// expansion) are its source, 16 bytes at a time.
+// expansion) are its source: the rows of one sy are the filters shifted along K
+// by sy k cin bytes, so the copy engine loads them as 128-byte-swizzled boxes.
 //
 // Anchors.  With one output row per M row (cout >= 128) the tile's R anchor
 // rows are consecutive output rows and share the band's input rows (R + k - 1
@@ -103,7 +104,8 @@ struct WinArgs {
   uint32_t plane_stride;   // bytes between the planes of a band buffer
   uint32_t band_bytes;     // bytes of one band buffer
   uint32_t stage_bytes;    // bytes of one staging buffer (nseg * rb * row_bytes, rounded)
-  uint32_t a_bytes;        // bytes of the resident A operand (kc * 2048)
+  uint32_t a_bytes;        // bytes of the resident A operand: 16 KB per 128-byte K stage of the Toeplitz K
+  int early;               // 1: no kernel before this one in the stream writes the filters
   FastDiv div_planes, div_pitch, div_seg, div_bands, div_chunks, div_rb;
 };
 
@@ -192,7 +194,8 @@ __device__ __forceinline__ uint32_t win_col_offset(const WinArgs& a, int c) {
 __device__ __forceinline__ int win_row(const WinArgs& a, int y0, int r) { return y0 + r * a.ry; }
 
 template <int POOL, int ACC>
-__global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs a) {
+__global__ void __launch_bounds__(kWinThreads, 1)
+    conv_win_kernel(const __grid_constant__ CUtensorMap tmap_a, const WinArgs a) {
   extern __shared__ uint8_t smem_raw_[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw_ + 1023) & ~(uintptr_t)1023);
   const uint32_t sbase = smem_u32(smem);
@@ -210,7 +213,8 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
   auto acc_empty = [&](int b) { return barBase + 48u + 8u * b; };
   auto stage_full = [&](int b) { return barBase + 64u + 8u * b; };
   const uint32_t done_bar = barBase + 80u;
-  uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + kWinXchgBytes + kWinTabBytes + 96);
+  const uint32_t a_full = barBase + 88u;   // the resident A operand has landed
+  uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + kWinXchgBytes + kWinTabBytes + 104);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // CTA c takes channel tile c % nct and the band tiles c / nct, c / nct + G / nct, ... of it
@@ -232,6 +236,7 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
       mbar_init(stage_full(b), 1);
     }
     mbar_init(done_bar, 1);
+    mbar_init(a_full, 1);
     fence_mbar_init();
   }
   // B descriptors of band buffer 0, one per MMA: the pair of core columns (2q, 2q + 1); past the
@@ -243,36 +248,9 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     mtab[tid] = sdesc_none(sBand + b0, b1 - b0, 128u);
   }
   grid_dep_wait();
-  // The resident A operand: row m = (sy, nl) at 16-byte core column c = (iy, ix, p) holds bytes
-  // [16p, 16p + 16) of tap (iy - sy, ix) of filter n, or zeros.  Layout: core column c, row group
-  // m / 8, row m % 8 -> c * 2048 + (m / 8) * 128 + (m % 8) * 16.
-  // Copies of 16 bytes, a warp taking 8 rows x 4 consecutive core columns: 8 runs of 64 contiguous
-  // bytes of the prepared rows, and 4 x 128 contiguous bytes of shared memory.
-  {
-    const int kcq = (a.kc + 3) >> 2;
-    for (int wi = warp; wi < 16 * kcq; wi += kWinThreads / 32) {
-      const int m = (wi & 15) * 8 + (lane & 7), c = (wi >> 4) * 4 + (lane >> 3);
-      if (c >= a.kc) continue;
-      const int sy = m / a.ct, nl = m - sy * a.ct;
-      const int n = ctile * a.ct + nl;
-      const uint8_t* src = a.w_prep;
-      uint32_t bytes = 0;
-      if (c < a.kc_real) {
-        const int p = c % a.planes, t = c / a.planes;
-        const int iy = t / a.k, ix = t - iy * a.k, dy = iy - sy;
-        if (dy >= 0 && dy < a.k) {
-          src = a.w_prep + (size_t)n * a.Kpad + (size_t)((dy * a.k + ix) * a.cin + 16 * p);
-          bytes = 16;
-        }
-      }
-      cp_async_16(sA + (uint32_t)c * 2048u + (uint32_t)(m >> 3) * 128u + (uint32_t)(m & 7) * 16u, src, bytes);
-    }
-  }
-  cp_async_commit();
   // both band buffers start as zeros: padding slots and the tail past the band stay zero
   for (uint32_t o = (uint32_t)tid * 16u; o < 2u * a.band_bytes; o += kWinThreads * 16u)
     *(uint4*)(smem + a.a_bytes + o) = make_uint4(0u, 0u, 0u, 0u);
-  cp_async_wait<0>();
   fence_proxy_async_smem();
   tc_fence_before();
   __syncthreads();
@@ -375,8 +353,21 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
   } else if (warp == kWinMmaWarp) {
     // =================== MMA issue (one elected lane; the warp runs the loop) ===================
     const uint32_t idesc = idesc_e4m3_f32(128, a.N);
-    const uint64_t adesc0 = sdesc_none(sA, 2048u, 128u);
-    bool ok = true;
+    // The resident A operand, loaded by the copy engine in 128-byte-swizzled K stages of 128 rows
+    // x 128 bytes (the layout of a TMA box with 128B swizzle).  Row (sy, n) of the Toeplitz block
+    // is filter n shifted by sy k cin bytes along K (tap row iy = dy + sy), so the rows of one sy
+    // in K stage j are one box of the prepared filters at K = 128 j - sy k cin; the zeros before
+    // and after the filter come from the box reading outside the rows (zero fill).
+    if (!a.early) grid_dep_wait();
+    if (lane == 0) mbar_arrive_expect_tx(a_full, a.a_bytes);
+    __syncwarp();
+    const int nst = (int)(a.a_bytes >> 14);
+    for (int bx = lane; bx < nst * a.ry; bx += 32) {
+      const int j = bx / a.ry, sy = bx - j * a.ry;
+      tma_load_2d(sA + (uint32_t)j * 16384u + (uint32_t)(sy * a.ct) * 128u, &tmap_a, a_full,
+                  128 * j - sy * a.k * a.cin, ctile * a.ct);
+    }
+    bool ok = __all_sync(0xffffffffu, mbar_wait(a_full, 0));
 #pragma unroll 1
     for (int i = 0; i < n_local && ok; ++i) {
       const int bb = i & 1;
@@ -393,7 +384,8 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
         const uint64_t boff = (uint64_t)(((uint32_t)bb * a.band_bytes) >> 4);
 #pragma unroll 1
         for (int q = 0; q < nmma; ++q)
-          mma_e4m3(dacc, adesc0 + (uint64_t)(q * 256), mtab[q] + boff, idesc, q > 0 ? 1u : 0u);
+          mma_e4m3(dacc, sdesc_sw128(sA + (uint32_t)(q >> 2) * 16384u + (uint32_t)(q & 3) * 32u), mtab[q] + boff,
+                   idesc, q > 0 ? 1u : 0u);
         mma_commit(band_empty(bb));
         mma_commit(acc_full(bb));
       }
@@ -436,15 +428,15 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
     const int pair = a.ct == 32 ? (q >> 1) : (q & 1);
     const bool odd_row = (sy & 1) != 0;
     // the codes of one value against the three thresholds: ballots of bit 1 and of the parity of
-    // the three compares, collected by the lane whose index is the column's within its group
+    // the three compares, kept by the lane whose index is the column's within its group (a masked
+    // select, not a branch: a divergent branch per column would reconverge the warp 32 times)
     auto code_ballot = [&](float f, int col, uint32_t& k0, uint32_t& k1) {
       const bool p1 = f > t1, p2 = f > t2, p3 = f > t3;
       const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
       const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
-      if (lane == col) {
-        k0 = m0;
-        k1 = m1;
-      }
+      const uint32_t pick = 0u - (uint32_t)(lane == col);
+      k0 = (m0 & pick) | (k0 & ~pick);
+      k1 = (m1 & pick) | (k1 & ~pick);
     };
     auto packed = [&](uint32_t k0, uint32_t k1) {
       return spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1);
@@ -583,6 +575,7 @@ __global__ void __launch_bounds__(kWinThreads, 1) conv_win_kernel(const WinArgs 
   if (warp == kWinMmaWarp) {
     tc_fence_after();
     mbar_wait(done_bar, 0);
+    mbar_wait(a_full, 0);   // the A copies have landed (already true unless a wait ran out)
     tmem_dealloc(tmem, 512);
   }
 }

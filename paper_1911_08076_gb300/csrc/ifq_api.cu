@@ -382,7 +382,7 @@ bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, s
   const int kc_real = (ry + k - 1) * k * planes;
   const int kc = (int)round_up((size_t)kc_real, 2);
   if (kc / 2 > kWinMaxMma) return false;
-  const uint32_t a_bytes = (uint32_t)kc * 2048u;
+  const uint32_t a_bytes = (uint32_t)ceil_div(kc, 8) * 16384u;   // 128-byte K stages of 128 rows
   int R = 0, seg_pitch = 0, rb = 0, N = 0, nseg = 0;
   uint32_t ps = 0, band_bytes = 0, stage_bytes = 0;
   size_t need = 0;
@@ -440,13 +440,24 @@ bool win_supported(const ifq_conv_desc* d, const ConvGeom& g) {
   return win_plan(d, g, nsm, nullptr, nullptr);
 }
 
+// Where the window kernel is the default (measured on GB300 against the tensor-core kernel, layer
+// by layer in the benchmark stacks): layers with a fused 2 x 2 pool and at most 64 input
+// channels.  Tiny-YOLO conv2 (16 -> 32 at 208 x 208, b64) 65 vs 128 us, conv3 38 vs 51, conv4 21 vs
+// 28; IFQ-Tinier-YOLO conv3..conv5 27 / 19 / 14 vs 38 / 21 / 16 us.  Without a pool its epilogue
+// thresholds twice the columns, and with 128 or more input channels its resident filter block and
+// per-tile setup cost more than the other kernel's gather: there the tensor-core kernel stays ahead
+// (ResNet-18 stage 1: 21 vs 18 us; Tinier conv6: 16 vs 14 us).
+bool win_wins(const ifq_conv_desc* d, const ConvGeom& g) {
+  return g.pool == 2 && d->cin <= 64 && win_supported(d, g);
+}
+
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
     path = forced ? forced
                   : (direct_supported(d, g) ? IFQ_PATH_DIRECT
-                                            : (win_supported(d, g) ? IFQ_PATH_WIN
+                                            : (win_wins(d, g) ? IFQ_PATH_WIN
                                                                    : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL
                                                                                         : IFQ_PATH_TC)));
   }
@@ -655,9 +666,12 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     // CTAs come in groups of nct, one per channel tile, each group sharing the band tiles
     const int per = std::max(1, std::min(wa.ntiles, nsm / wa.nct));
     const dim3 grid((unsigned)(per * wa.nct)), block(kWinThreads);
-    if (g.pool == 2) e = launch_k(conv_win_kernel<1, 0>, grid, block, smem, st, wa);
-    else if (ya) e = launch_k(conv_win_kernel<0, 1>, grid, block, smem, st, wa);
-    else e = launch_k(conv_win_kernel<0, 0>, grid, block, smem, st, wa);
+    wa.early = early ? 1 : 0;
+    CUtensorMap tma;
+    if (!encode_wmap(d, g, w_prep, wa.ct, &tma)) return IFQ_ECUDA;
+    if (g.pool == 2) e = launch_k(conv_win_kernel<1, 0>, grid, block, smem, st, tma, wa);
+    else if (ya) e = launch_k(conv_win_kernel<0, 1>, grid, block, smem, st, tma, wa);
+    else e = launch_k(conv_win_kernel<0, 0>, grid, block, smem, st, tma, wa);
   } else if (path == IFQ_PATH_TC) {
     int bn = choose_bn(g, d->cout, nsm), ks = 1;
     const int gb = granule_bytes(d, g);

@@ -280,16 +280,19 @@ def test_last_forward_mode_before_any_forward_is_einval():
 
 
 def test_window_path_plan():
-    """The window path takes stride-1 k x k 'same' layers on 2-bit codes with cin 16 or a multiple of
-    32, cout 32, 64 or a multiple of 128, whose resident filter block and two input bands fit one
-    CTA's shared memory; everything else keeps its previous path, and IFQ_WIN=0 turns it off."""
+    """The window path applies to stride-1 k x k 'same' layers on 2-bit codes with cin 16 or a
+    multiple of 32, cout 32, 64 or a multiple of 128, whose resident filter block and buffers fit
+    one CTA's shared memory, and is the default for those with a fused 2 x 2 pool and cin <= 64;
+    everything else keeps its previous path, and IFQ_WIN=0 turns it off."""
     WIN, TC = ifq.IFQ_PATH_WIN, ifq.IFQ_PATH_TC
     plan = lambda *a, **k: ifq.ifq_conv_plan(ifq.conv_desc(*a, **k))
     assert plan(64, 208, 208, 16, 32, 3, 1, 1, pool=2) == WIN       # Tiny-YOLO conv2, fused pool
     assert plan(64, 104, 104, 32, 64, 3, 1, 1, pool=2) == WIN       # Tiny-YOLO conv3
     assert plan(64, 52, 52, 64, 128, 3, 1, 1, pool=2) == WIN        # Tiny-YOLO conv4
-    assert plan(32, 56, 56, 64, 64, 3, 1, 1) == WIN                  # ResNet-18 stage 1
-    assert plan(1, 16, 16, 64, 64, 3, 1, 1, out_mode=ifq.IFQ_OUT_BOTH) == WIN
+    assert plan(32, 56, 56, 64, 64, 3, 1, 1) == TC                   # no pool: the other kernel is faster
+    assert plan(32, 56, 56, 64, 64, 3, 1, 1, path=WIN) == WIN        # ... but the window path applies
+    assert plan(64, 26, 26, 128, 256, 3, 1, 1, pool=2) == TC         # 128 input channels: likewise
+    assert plan(1, 16, 16, 64, 64, 3, 1, 1, out_mode=ifq.IFQ_OUT_BOTH, path=WIN) == WIN
     assert plan(32, 56, 56, 64, 128, 3, 2, 1) == TC                  # stride 2
     assert plan(256, 56, 56, 256, 256, 3, 1, 1) == TC                # filter block too large
     assert plan(64, 13, 13, 1024, 30, 1, 1, 0, out_mode=ifq.IFQ_OUT_ACC) == TC   # cout 30
