@@ -22,6 +22,8 @@ __device__ __forceinline__ uint32_t fdiv(uint32_t n, FastDiv f) {
 
 struct ConvArgs {
   const uint8_t* x;      // packed input codes, NHWC
+  const uint8_t* wbits;  // filter sign bits in the e4m3 rows' K order, [cout][Kpad / 8] bytes (bit = +1),
+                         // read by the kernels that expand B in shared memory (BX), else unused
   const int32_t* thr;    // [cout][lvl]
   const int8_t* sign;    // [cout]
   uint8_t* y_codes;      // packed output codes or nullptr

@@ -81,7 +81,14 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
 // order does not matter.  A receive slot is reused for the next tile once its owner has read it
 // (send_ok); clusters synchronise once after setup and once before exit, so no CTA's shared memory
 // goes away while a partner may still write it.
-template <int BN, int GB, int SB, int SBO, int KS = 1>
+//
+// BX = 1: the filter tile (B) is not loaded by TMA as e4m3 bytes but expanded in shared memory from
+// the filters' sign bits (1 bit per weight instead of 8) by the gather group that fills the same K
+// stage, into the 128B-swizzled layout TMA would have written.  For layers whose filters are read
+// from DRAM about once (few row tiles, e.g. fully connected layers) that cuts the filter stream
+// eightfold.  K positions past the filter read -1 from the bits, which is harmless: the gathered
+// codes are zero there.
+template <int BN, int GB, int SB, int SBO, int KS = 1, int BX = 0>
 __global__ void __launch_bounds__(kConvThreads, 1)
     conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_w, const ConvArgs args) {
   static_assert(2 * BN <= kTmemA && kTmemA + 32 * kStages <= 512, "tensor memory budget");
@@ -130,7 +137,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   }
   if (tid == 0) {
     for (int s = 0; s < kS; ++s) {
-      mbar_init(full(s), 4 + 1);   // one gather group (4 warps) + the TMA producer
+      mbar_init(full(s), BX ? 4 : 4 + 1);   // one gather group (4 warps) [+ the TMA producer]
       mbar_init(empty(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -227,13 +234,57 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           if constexpr (SB == 2) expand2(cur[kU - 1], o);
           else expand4(cur[kU - 2], cur[kU - 1], o);
           tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
+          if constexpr (BX != 0) {
+            // this K stage's filter tile from sign bits: thread i of the group (128) takes BN / 8
+            // bytes of bits, BN / 16 chunks of 16 bits -> 16 e4m3 bytes (+1 = 0x38, -1 = 0xB8) at
+            // row r, chunk c of the 128B-swizzled slot (chunk c of row r at c ^ (r % 8))
+            const int jt = it / nk, kk = it - jt * nk;
+            const int tt = cid + jt * G;
+            const int n0 = (tt - (int)fdiv((uint32_t)tt, args.div_nt) * args.nt) * BN;
+            constexpr int kCpt = BN / 16;                   // chunks per thread
+            const int gi = quarter * 32 + lane;             // 0..127
+            const int rr = gi / (8 / kCpt), c0 = (gi % (8 / kCpt)) * kCpt;
+            const int nrow = n0 + rr;
+            uint32_t bw[kCpt / 2 > 0 ? kCpt / 2 : 1];
+            if constexpr (kCpt >= 2) {
+#pragma unroll
+              for (int q2 = 0; q2 < kCpt / 2; ++q2) bw[q2] = 0u;
+              if (nrow < args.cout) {
+                const uint32_t* src = (const uint32_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
+                                                        (size_t)(kb + kk) * (kBK / 8) + c0 * 2);
+#pragma unroll
+                for (int q2 = 0; q2 < kCpt / 2; ++q2) bw[q2] = __ldg(src + q2);
+              }
+            } else {
+              bw[0] = 0u;
+              if (nrow < args.cout)
+                bw[0] = __ldg((const uint16_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
+                                                (size_t)(kb + kk) * (kBK / 8) + c0 * 2));
+            }
+            const uint32_t rowb = sB + (uint32_t)(s * L::kB) + (uint32_t)rr * 128u;
+#pragma unroll
+            for (int cc = 0; cc < kCpt; ++cc) {
+              const uint32_t bits16 = (bw[cc >> 1] >> (16 * (cc & 1))) & 0xFFFFu;
+              uint32_t w4[4];
+#pragma unroll
+              for (int nb = 0; nb < 4; ++nb) {
+                const uint32_t x = (((bits16 >> (4 * nb)) & 0xFu) * 0x00204081u) & 0x01010101u;
+                w4[nb] = 0xB8B8B8B8u - (x << 7);
+              }
+              const uint32_t dst = rowb + (uint32_t)((((c0 + cc) ^ (rr & 7)) & 7) << 4);
+              asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w4[0]), "r"(w4[1]), "r"(w4[2]),
+                           "r"(w4[3])
+                           : "memory");
+            }
+            fence_proxy_async_smem();
+          }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(full(s));
         }
       }
     }
-  } else if (warp == kWarpTma) {
+  } else if (warp == kWarpTma && BX == 0) {
     if (!args.early) grid_dep_wait();
     // =================== TMA producer (filters) ===================
     // the whole warp runs the loop; one elected lane issues

@@ -114,11 +114,11 @@ cudaError_t launch_k_cluster(void (*kern)(Exp...), int cluster, dim3 grid, dim3 
 // One instance of the tensor-core kernel.  KS > 1 (split K over clusters of KS CTAs): the grid is
 // as many clusters as can be resident at once (cudaOccupancyMaxActiveClusters), at most one per
 // tile.
-template <int BN, int GB, int SB, int SBO, int KS = 1>
+template <int BN, int GB, int SB, int SBO, int KS = 1, int BX = 0>
 struct TcInst {
   using L = TcSmem<BN, SBO, KS>;
   static_assert(L::bytes <= 232448, "shared memory budget");
-  static constexpr auto kern = conv_tc_kernel<BN, GB, SB, SBO, KS>;
+  static constexpr auto kern = conv_tc_kernel<BN, GB, SB, SBO, KS, BX>;
   static cudaError_t set_attr() {
     return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::bytes);
   }
@@ -166,6 +166,8 @@ struct TcInst {
 // exist for 16-byte granules (every layer with 64 or more 2-bit, or 32 or more 4-bit, channels).
 #define IFQ_TC_VARIANTS(X, GB, SB, SBO) X(128, GB, SB, SBO, 1) X(64, GB, SB, SBO, 1) X(32, GB, SB, SBO, 1)
 #define IFQ_TC_SPLIT_VARIANTS(X, GB, SB, SBO) X(64, GB, SB, SBO, 2)
+// the split instance that expands its filter tiles from sign bits (2-bit codes, 16-byte granules)
+using TcSplitBits = TcInst<64, 16, 2, 2, 2, 1>;
 
 template <int GB, int SB, int SBO>
 cudaError_t set_attrs_gb() {
@@ -175,6 +177,9 @@ cudaError_t set_attrs_gb() {
   IFQ_TC_VARIANTS(IFQ_SET, GB, SB, SBO)
   if constexpr (GB == 16) {
     IFQ_TC_SPLIT_VARIANTS(IFQ_SET, GB, SB, SBO)
+    if constexpr (SB == 2 && SBO == 2) {
+      if (e == cudaSuccess) e = TcSplitBits::set_attr();
+    }
   }
 #undef IFQ_SET
   return e;
@@ -310,8 +315,12 @@ size_t prep_masks_offset(const ifq_conv_desc* d, const ConvGeom& g) {
   return prep_bits_offset(d, g) + round_up((size_t)d->cout * g.kwords * 4, 256);
 }
 
+// Layers on codes: then the sign bits in the e4m3 rows' K order, [cout][Kpad / 8] bytes, where the
+// 8-bit-input layers keep their masks.
+size_t prep_pbits_offset(const ifq_conv_desc* d, const ConvGeom& g) { return prep_masks_offset(d, g); }
+
 size_t prep_bytes(const ifq_conv_desc* d, const ConvGeom& g) {
-  return g.in8 ? prep_masks_offset(d, g) + (size_t)g.K * 4 : prep_bits_offset(d, g) + (size_t)d->cout * g.kwords * 4;
+  return g.in8 ? prep_masks_offset(d, g) + (size_t)g.K * 4 : prep_pbits_offset(d, g) + (size_t)d->cout * g.Kpad / 8;
 }
 
 bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g);
@@ -529,7 +538,11 @@ void choose_split(const ConvGeom& g, int cout, int nsm, int* bn, int* ks) {
 }
 
 template <int GB, int SB, int SBO>
-cudaError_t launch_tc_gb(int bn, int ks, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st) {
+cudaError_t launch_tc_gb(int bn, int ks, const CUtensorMap& tm, const ConvArgs& a, int nsm, cudaStream_t st,
+                         bool bx = false) {
+  if constexpr (GB == 16 && SB == 2 && SBO == 2) {
+    if (bx && bn == 64 && ks == 2) return TcSplitBits::launch(tm, a, nsm, st);
+  }
 #define IFQ_LAUNCH(BN, G, S, SO, KS) \
   if (bn == BN && ks == KS) return TcInst<BN, G, S, SO, KS>::launch(tm, a, nsm, st);
   IFQ_TC_VARIANTS(IFQ_LAUNCH, GB, SB, SBO)
@@ -579,6 +592,7 @@ bool encode_wmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, 
 void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const void* x, const int32_t* thr,
                     const int8_t* sign, uint8_t* yc, int32_t* ya, ConvArgs* a, bool stack = false) {
   a->x = (const uint8_t*)x;
+  a->wbits = nullptr;
   a->thr = thr;
   a->sign = sign;
   a->y_codes = yc;
@@ -685,8 +699,14 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
     a.early = early ? 1 : 0;
-    if (g.sbi == 2) {
-      if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st);
+    a.wbits = g.in8 ? nullptr : (const uint8_t*)w_prep + prep_pbits_offset(d, g);
+    // Filter tiles expanded from sign bits in shared memory where the filters are streamed from DRAM
+    // about once (at most two 128-row tiles, the fully connected layers): the split instance only.
+    // IFQ_TC_BX = 0 / 2 forbids / forces it where the split instance runs.
+    const int bx_env = env_int("IFQ_TC_BX", 1);
+    const bool bx = bx_env != 0 && (bx_env == 2 || ceil_div(g.M, kBM) <= 2);
+    if (g.sbi == 2 && g.sb == 2) {
+      if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st, bx);
       else if (gb == 8) e = launch_tc_gb<8, 2, 2>(bn, ks, tm, a, nsm, st);
       else if (gb == 4) e = launch_tc_gb<4, 2, 2>(bn, ks, tm, a, nsm, st);
       else e = launch_tc_gb<1, 2, 2>(bn, ks, tm, a, nsm, st);
@@ -1276,8 +1296,10 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
   if ((rc = ensure_init(&nsm))) return rc;
   uint8_t* base = (uint8_t*)w_prep;
   const int blocks = launch_1d_blocks((size_t)d->cout * (g.Kpad / 4), 256, nsm);
-  prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
-                                                     d->cout, g.Kk, g.Kpad, g.kwords, 32 / g.sbi, g.in8 ? 1 : 0);
+  prep_weights_kernel<<<blocks, 256, 0, S(stream)>>>(
+      w_bits, base, (uint32_t*)(base + prep_bits_offset(d, g)),
+      g.in8 ? nullptr : (uint32_t*)(base + prep_pbits_offset(d, g)), d->cout, g.Kk, g.Kpad, g.kwords, 32 / g.sbi,
+      g.in8 ? 1 : 0);
   if (g.in8)
     prep_direct_masks_kernel<<<launch_1d_blocks((size_t)g.K, 256, nsm), 256, 0, S(stream)>>>(
         (const uint32_t*)(base + prep_bits_offset(d, g)), (uint32_t*)(base + prep_masks_offset(d, g)), d->cout, g.K,

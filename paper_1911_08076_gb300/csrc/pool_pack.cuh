@@ -313,8 +313,8 @@ __global__ void pack_signs_kernel(const int8_t* w, uint32_t* bits, int rows, int
 // in8: the input is 8-bit values read as two 4-bit fields, so kernel position k
 // is filter position k/2 times 1 (low nibble, k even) or 16 (high nibble):
 // +-16 are the e4m3 bytes 0x58 / 0xD8.  K is the kernel's K (twice the filter's).
-__global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_t* bits_copy, int cout, int K,
-                                    int Kpad, int kwords, int cpw, int in8) {
+__global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_t* bits_copy, uint32_t* pbits, int cout,
+                                    int K, int Kpad, int kwords, int cpw, int in8) {
   const long total = (long)cout * (Kpad / 4);
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
     const int n = (int)(i / (Kpad / 4));
@@ -339,6 +339,24 @@ __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_
   const long tw = (long)cout * kwords;
   for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < tw; i += (long)gridDim.x * blockDim.x)
     bits_copy[i] = bits[i];
+  // the same signs in the e4m3 rows' K order, one bit per byte position (set: +1): what the kernels
+  // that expand the filter tile in shared memory read; positions past K are 0 (-1 there is harmless:
+  // the gathered codes are zero)
+  if (pbits && !in8) {
+    const long tp = (long)cout * (Kpad / 32);
+    for (long i = (long)blockIdx.x * blockDim.x + threadIdx.x; i < tp; i += (long)gridDim.x * blockDim.x) {
+      const int n = (int)(i / (Kpad / 32));
+      const int p0 = (int)(i % (Kpad / 32)) * 32;
+      uint32_t w = 0;
+      for (int b = 0; b < 32; ++b) {
+        const int pos = p0 + b;
+        const int j = pos / cpw, p = pos - j * cpw;
+        const int k = cpw * j + (cpw >> 2) * (p & 3) + (p >> 2);
+        if (k < K && ((bits[(size_t)n * kwords + (k >> 5)] >> (k & 31)) & 1u)) w |= 1u << b;
+      }
+      pbits[i] = w;
+    }
+  }
 }
 
 }  // namespace ifq

@@ -135,3 +135,50 @@ def test_split_k_resnet18_stack_equals_unsplit(monkeypatch):
     last = len(wl.layers) - 1
     got = synth.unpack_codes(st.y_codes[last][:1].cpu().numpy(), wl.layers[last].cout)
     assert (got == one[last]).all()
+
+
+BITS_CASES = [c for c in SPLIT_CASES if c[8] == 2]
+
+
+@pytest.mark.parametrize("case", BITS_CASES, ids=[str(c) for c in BITS_CASES])
+def test_split_k_with_filter_tiles_from_sign_bits(case, monkeypatch):
+    """The split kernel whose filter tiles are expanded in shared memory from the sign bits (one
+    bit per weight streamed instead of an e4m3 byte; IFQ_TC_BX = 2 forces it), bit-exact against the
+    oracle, including K padded past the filter (C = 320: 2880 of 2944 positions) and partial channel
+    tiles."""
+    monkeypatch.setenv("IFQ_TC_BX", "2")
+    test_split_k_matches_oracle(case, monkeypatch)
+
+
+def test_fc_layers_take_the_sign_bit_filters_by_default(monkeypatch):
+    """AlexNet's FC6 and FC7 shapes (one 128-row tile): the default run (filter tiles from sign bits)
+    equals the run that loads e4m3 filter tiles, codes and accumulators."""
+    rng = np.random.default_rng(6)
+    for (B, H, C, cout, k, mode) in ((128, 6, 256, 4096, 6, ifq.IFQ_OUT_CODES), (128, 1, 4096, 4096, 1, ifq.IFQ_OUT_ACC)):
+        x = rng.integers(0, 4, (B, H, H, C), dtype=np.uint8)
+        w = np.where(rng.integers(0, 2, (cout, k, k, C)) == 1, 1, -1).astype(np.int8)
+        prm = _params(rng, cout, k * k * C, 2)
+        T, sg = _fold(prm, k * k * C)
+        outs = []
+        for bx in ("1", "0"):
+            monkeypatch.setenv("IFQ_TC_BX", bx)
+            monkeypatch.delenv("IFQ_TC_KS", raising=False)
+            d = ifq.conv_desc(B, H, H, C, cout, k, 1, 0, mode, TC)
+            xp = torch.from_numpy(synth.pack_codes(x)).to(DEV)
+            bits = torch.from_numpy(synth.pack_signs(w).view(np.int32)).to(DEV)
+            prep = torch.empty(ifq.ifq_weights_prep_bytes(d), dtype=torch.uint8, device=DEV)
+            ifq.ifq_pack_weights(d, bits, prep)
+            yc = torch.zeros((B, 1, 1, cout // 4), dtype=torch.uint8, device=DEV) if mode & 1 else None
+            ya = torch.zeros((B, 1, 1, cout), dtype=torch.int32, device=DEV) if mode & 2 else None
+            ifq.ifq_conv2bit(d, xp, prep, torch.from_numpy(T).to(DEV), torch.from_numpy(sg).to(DEV), yc, ya)
+            torch.cuda.synchronize()
+            assert ifq.ifq_device_status() == ifq.IFQ_OK
+            outs.append((None if yc is None else yc.cpu(), None if ya is None else ya.cpu()))
+        for a, b in zip(outs[0], outs[1]):
+            if a is not None:
+                assert torch.equal(a, b)
+        A = O.conv_acc(x, w, 1, 0)
+        if mode & 2:
+            assert (outs[0][1].numpy() == A).all()
+        else:
+            assert (synth.unpack_codes(outs[0][0].numpy(), cout) == O.int_chain(A, *O.fold(prm, k * k * C))).all()
