@@ -284,7 +284,9 @@ __global__ void __launch_bounds__(kConvThreads, 1)
         }
       }
     }
-  } else if (warp == kWarpTma && BX == 0) {
+  } else if (warp == kWarpTma) {
+    // (with BX the gather groups write the filter tiles: this warp has no work)
+    if constexpr (BX == 0) {
     if (!args.early) grid_dep_wait();
     // =================== TMA producer (filters) ===================
     // the whole warp runs the loop; one elected lane issues
@@ -313,6 +315,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
         mbar_wait(full(i % kS), (uint32_t)(i / kS) & 1u);
     }
     __syncwarp();
+    }
   } else if (warp == kWarpMma || warp == kWarpMma2) {
     // =================== MMA issue ===================
     // Two MMA warps take alternate pairs of K stages of every tile into the same accumulator:
