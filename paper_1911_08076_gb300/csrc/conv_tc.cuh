@@ -194,8 +194,34 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)(cid + l_tile * G), args.div_nt) * kBM + r
                                                 : args.M);
     // packed codes of kAh of this group's stages in registers (16 registers either way)
-    constexpr int kAh = SB == 2 ? kAhead : 1;
-    auto next_load = [&](uint4 (&u)[kU]) {
+    // (the bits-expanding instance keeps one own stage ahead, four in the CTA's sequence, to stay
+    // within 72 registers)
+    constexpr int kAh = SB == 2 && BX == 0 ? kAhead : 1;
+    // BX: this thread's share of the stage's filter sign bits travels with its codes (row bx_r of
+    // the channel tile, 16-bit chunks bx_c0 .. bx_c0 + BN / 16 - 1 of the stage's 128 positions)
+    constexpr int kCpt = BN / 16;
+    constexpr int kBw = BX ? (kCpt + 1) / 2 : 1;
+    const int bx_gi = quarter * 32 + lane;
+    const int bx_r = bx_gi / (8 / kCpt), bx_c0 = (bx_gi % (8 / kCpt)) * kCpt;
+    uint32_t bring[kAh][kBw];
+    auto next_bits = [&](uint32_t (&b)[kBw]) {
+#pragma unroll
+      for (int q2 = 0; q2 < kBw; ++q2) b[q2] = 0u;
+      if constexpr (BX != 0) {
+        if (l_tile < n_local) {
+          const int tt = cid + l_tile * G;
+          const int nrow = (tt - (int)fdiv((uint32_t)tt, args.div_nt) * args.nt) * BN + bx_r;
+          if (nrow < args.cout) {
+            const uint32_t* src = (const uint32_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
+                                                    (size_t)(kb + l_k) * (kBK / 8) + bx_c0 * 2);
+#pragma unroll
+            for (int q2 = 0; q2 < kBw; ++q2) b[q2] = __ldg(src + q2);
+          }
+        }
+      }
+    };
+    auto next_load = [&](uint4 (&u)[kU], uint32_t (&bu)[kBw]) {
+      next_bits(bu);
 #pragma unroll
       for (int q = 0; q < kU; ++q) u[q] = load_unit<GB>(sTab, g, (kb + l_k) * kU + q);
       l_k += kGatherGroups;
@@ -209,7 +235,9 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     for (int d = 0; d < kAh; ++d) {
 #pragma unroll
       for (int q = 0; q < kU; ++q) ring[d][q] = make_uint4(0u, 0u, 0u, 0u);
-      if (d < own) next_load(ring[d]);
+#pragma unroll
+      for (int q2 = 0; q2 < kBw; ++q2) bring[d][q2] = 0u;
+      if (d < own) next_load(ring[d], bring[d]);
     }
     bool ok = true;
 #pragma unroll 1
@@ -221,7 +249,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           uint4 cur[kU];
 #pragma unroll
           for (int q = 0; q < kU; ++q) cur[q] = ring[d][q];
-          if (j + kAh < own) next_load(ring[d]);
+          uint32_t bw[kBw];
+#pragma unroll
+          for (int q2 = 0; q2 < kBw; ++q2) bw[q2] = bring[d][q2];
+          if (j + kAh < own) next_load(ring[d], bring[d]);
           const int it = group + kGatherGroups * j;
           const int s = it % kS;
           const uint32_t ph = (uint32_t)(it / kS) & 1u;
@@ -235,32 +266,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           else expand4(cur[kU - 2], cur[kU - 1], o);
           tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
           if constexpr (BX != 0) {
-            // this K stage's filter tile from sign bits: thread i of the group (128) takes BN / 8
-            // bytes of bits, BN / 16 chunks of 16 bits -> 16 e4m3 bytes (+1 = 0x38, -1 = 0xB8) at
-            // row r, chunk c of the 128B-swizzled slot (chunk c of row r at c ^ (r % 8))
-            const int jt = it / nk, kk = it - jt * nk;
-            const int tt = cid + jt * G;
-            const int n0 = (tt - (int)fdiv((uint32_t)tt, args.div_nt) * args.nt) * BN;
-            constexpr int kCpt = BN / 16;                   // chunks per thread
-            const int gi = quarter * 32 + lane;             // 0..127
-            const int rr = gi / (8 / kCpt), c0 = (gi % (8 / kCpt)) * kCpt;
-            const int nrow = n0 + rr;
-            uint32_t bw[kCpt / 2 > 0 ? kCpt / 2 : 1];
-            if constexpr (kCpt >= 2) {
-#pragma unroll
-              for (int q2 = 0; q2 < kCpt / 2; ++q2) bw[q2] = 0u;
-              if (nrow < args.cout) {
-                const uint32_t* src = (const uint32_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
-                                                        (size_t)(kb + kk) * (kBK / 8) + c0 * 2);
-#pragma unroll
-                for (int q2 = 0; q2 < kCpt / 2; ++q2) bw[q2] = __ldg(src + q2);
-              }
-            } else {
-              bw[0] = 0u;
-              if (nrow < args.cout)
-                bw[0] = __ldg((const uint16_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
-                                                (size_t)(kb + kk) * (kBK / 8) + c0 * 2));
-            }
+            // this K stage's filter tile from sign bits (loaded with the codes, kAh stages ahead):
+            // 16-bit chunks -> 16 e4m3 bytes (+1 = 0x38, -1 = 0xB8) at row bx_r, chunk c of the
+            // 128B-swizzled slot (chunk c of row r at c ^ (r % 8))
+            const int rr = bx_r, c0 = bx_c0;
             const uint32_t rowb = sB + (uint32_t)(s * L::kB) + (uint32_t)rr * 128u;
 #pragma unroll
             for (int cc = 0; cc < kCpt; ++cc) {
