@@ -66,19 +66,24 @@ constexpr int kAhead = 2;        // own K stages of packed codes a gather thread
 // order of the 4-ary search, and the sign) for SB = 4.
 // KS > 1 (split K over a cluster of KS CTAs): KS - 1 receive slots of fp32 partial sums, one per
 // partner, each 128 rows x BN / KS columns (rows padded by 16 bytes), and two more barriers.
-template <int BN, int SB = 2, int KS = 1>
+// BX = 1 (filter tiles expanded from sign bits): a ring of kBitStages slots of BN rows x 16 bytes
+// (one K stage's 128 sign bits a row), filled by TMA ahead of the gather, and its two barriers a slot.
+template <int BN, int SB = 2, int KS = 1, int BX = 0>
 struct TcSmem {
   static constexpr int kB = BN * kBK;
   static constexpr int kThrCol = SB == 2 ? 16 : 80;       // bytes of thresholds per column
   static constexpr int kRecvRow = BN / KS + 4;             // floats per row of a receive slot
   static constexpr int kRecvSlot = kBM * kRecvRow * 4;     // bytes of a receive slot
+  static constexpr int kBitStages = BX ? 32 : 0;
+  static constexpr int kBitSlot = BN * 16;
   static constexpr int offB = 0;
   static constexpr int offThr = offB + kStages * kB;       // 2 buffers of BN columns
   static constexpr int offTab = offThr + 2 * BN * kThrCol; // kMaxTab x int2
   static constexpr int offRecv = offTab + kMaxTab * 8;
-  static constexpr int offBar = offRecv + (KS - 1) * kRecvSlot;
-  // full, empty, acc_full[2], acc_empty[2], done (+ recv_full, send_ok)
-  static constexpr int nBar = 2 * kStages + 5 + (KS > 1 ? 2 : 0);
+  static constexpr int offBits = offRecv + (KS - 1) * kRecvSlot;
+  static constexpr int offBar = offBits + kBitStages * kBitSlot;
+  // full, empty, acc_full[2], acc_empty[2], done (+ recv_full, send_ok) (+ bits_full, bits_empty)
+  static constexpr int nBar = 2 * kStages + 5 + (KS > 1 ? 2 : 0) + 2 * kBitStages;
   static constexpr int offTmem = offBar + nBar * 8;
   static constexpr int bytes = offTmem + 16 + 1024;        // + alignment slack
 };

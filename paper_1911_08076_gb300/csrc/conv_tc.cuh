@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   static_assert((SB == 2 || SB == 4) && (SBO == 2 || SBO == 4), "stored code width");
   static_assert(KS == 1 || KS == 2 || KS == 4, "K split");
   static_assert(BN / KS / 2 >= 16, "an epilogue thread takes at least 16 columns of a block");
-  using L = TcSmem<BN, SBO, KS>;
+  using L = TcSmem<BN, SBO, KS, BX>;
   constexpr int kU = kBK * SB / 8 / 16;       // 16-byte units of packed codes per K stage
   constexpr int kCpb = 8 / SB;                // codes per byte
   constexpr int kS = kStages;
@@ -117,6 +117,12 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   // block; send_ok when every partner has read the partial this CTA stored in its slot
   const uint32_t recv_full = barBase + 8u * (2 * kS + 5);
   const uint32_t send_ok = barBase + 8u * (2 * kS + 6);
+  // BX: bits_full[i] completes when slot i of the sign-bit ring has landed; bits_empty[i] when the
+  // gather group that read it is done with it
+  constexpr int kBitBar0 = 2 * kS + 5 + (KS > 1 ? 2 : 0);
+  auto bits_full = [&](int i) { return barBase + 8u * (kBitBar0 + i); };
+  auto bits_empty = [&](int i) { return barBase + 8u * (kBitBar0 + L::kBitStages + i); };
+  const uint32_t sBits = sbase + L::offBits;
   uint32_t* tmem_slot = (uint32_t*)(smem + L::offTmem);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -145,6 +151,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       mbar_init(acc_empty(b), kEpiWarps);  // drained and zeroed by every epilogue warp
     }
     mbar_init(done_bar, 2);
+    for (int i = 0; i < L::kBitStages; ++i) {
+      mbar_init(bits_full(i), 1);
+      mbar_init(bits_empty(i), 4);   // the 4 warps of the gather group that expands the stage
+    }
     if constexpr (KS > 1) {
       mbar_init(recv_full, (KS - 1) * kEpiWarps * 32);   // every epilogue thread of every partner
       mbar_init(send_ok, (KS - 1) * kEpiWarps * 32);
@@ -194,34 +204,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)(cid + l_tile * G), args.div_nt) * kBM + r
                                                 : args.M);
     // packed codes of kAh of this group's stages in registers (16 registers either way)
-    // (the bits-expanding instance keeps one own stage ahead, four in the CTA's sequence, to stay
-    // within 72 registers)
-    constexpr int kAh = SB == 2 && BX == 0 ? kAhead : 1;
-    // BX: this thread's share of the stage's filter sign bits travels with its codes (row bx_r of
-    // the channel tile, 16-bit chunks bx_c0 .. bx_c0 + BN / 16 - 1 of the stage's 128 positions)
+    constexpr int kAh = SB == 2 ? kAhead : 1;
+    // BX: this thread's share of a stage's filter tile: row bx_r of the channel tile, 16-bit chunks
+    // bx_c0 .. bx_c0 + BN / 16 - 1 of the stage's 128 sign bits
     constexpr int kCpt = BN / 16;
-    constexpr int kBw = BX ? (kCpt + 1) / 2 : 1;
     const int bx_gi = quarter * 32 + lane;
     const int bx_r = bx_gi / (8 / kCpt), bx_c0 = (bx_gi % (8 / kCpt)) * kCpt;
-    uint32_t bring[kAh][kBw];
-    auto next_bits = [&](uint32_t (&b)[kBw]) {
-#pragma unroll
-      for (int q2 = 0; q2 < kBw; ++q2) b[q2] = 0u;
-      if constexpr (BX != 0) {
-        if (l_tile < n_local) {
-          const int tt = cid + l_tile * G;
-          const int nrow = (tt - (int)fdiv((uint32_t)tt, args.div_nt) * args.nt) * BN + bx_r;
-          if (nrow < args.cout) {
-            const uint32_t* src = (const uint32_t*)(args.wbits + (size_t)nrow * (args.nk * (kBK / 8)) +
-                                                    (size_t)(kb + l_k) * (kBK / 8) + bx_c0 * 2);
-#pragma unroll
-            for (int q2 = 0; q2 < kBw; ++q2) b[q2] = __ldg(src + q2);
-          }
-        }
-      }
-    };
-    auto next_load = [&](uint4 (&u)[kU], uint32_t (&bu)[kBw]) {
-      next_bits(bu);
+    auto next_load = [&](uint4 (&u)[kU]) {
 #pragma unroll
       for (int q = 0; q < kU; ++q) u[q] = load_unit<GB>(sTab, g, (kb + l_k) * kU + q);
       l_k += kGatherGroups;
@@ -235,9 +224,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     for (int d = 0; d < kAh; ++d) {
 #pragma unroll
       for (int q = 0; q < kU; ++q) ring[d][q] = make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-      for (int q2 = 0; q2 < kBw; ++q2) bring[d][q2] = 0u;
-      if (d < own) next_load(ring[d], bring[d]);
+      if (d < own) next_load(ring[d]);
     }
     bool ok = true;
 #pragma unroll 1
@@ -249,10 +236,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           uint4 cur[kU];
 #pragma unroll
           for (int q = 0; q < kU; ++q) cur[q] = ring[d][q];
-          uint32_t bw[kBw];
-#pragma unroll
-          for (int q2 = 0; q2 < kBw; ++q2) bw[q2] = bring[d][q2];
-          if (j + kAh < own) next_load(ring[d], bring[d]);
+          if (j + kAh < own) next_load(ring[d]);
           const int it = group + kGatherGroups * j;
           const int s = it % kS;
           const uint32_t ph = (uint32_t)(it / kS) & 1u;
@@ -270,6 +254,22 @@ __global__ void __launch_bounds__(kConvThreads, 1)
             // 16-bit chunks -> 16 e4m3 bytes (+1 = 0x38, -1 = 0xB8) at row bx_r, chunk c of the
             // 128B-swizzled slot (chunk c of row r at c ^ (r % 8))
             const int rr = bx_r, c0 = bx_c0;
+            const int bs = it % L::kBitStages;
+            if (!__all_sync(0xffffffffu, mbar_wait(bits_full(bs), (uint32_t)(it / L::kBitStages) & 1u))) {
+              ok = false;
+              break;
+            }
+            uint32_t bw[(kCpt + 1) / 2];
+#pragma unroll
+            for (int q2 = 0; q2 < (kCpt + 1) / 2; ++q2) {
+              uint32_t v;
+              asm volatile("ld.shared.b32 %0, [%1];"
+                           : "=r"(v)
+                           : "r"(sBits + (uint32_t)(bs * L::kBitSlot + rr * 16 + c0 * 2 + 4 * q2)));
+              bw[q2] = v;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bits_empty(bs));
             const uint32_t rowb = sB + (uint32_t)(s * L::kB) + (uint32_t)rr * 128u;
 #pragma unroll
             for (int cc = 0; cc < kCpt; ++cc) {
@@ -294,7 +294,35 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       }
     }
   } else if (warp == kWarpTma) {
-    // (with BX the gather groups write the filter tiles: this warp has no work)
+    if constexpr (BX != 0) {
+      // =================== TMA producer (filter sign bits, kBitStages stages ahead) ===================
+      // tmap_w maps the sign bits: [cout][Kpad / 8] bytes, boxes of BN rows x 16 bytes
+      if (!args.early) grid_dep_wait();
+      int it = 0;
+      bool ok = true;
+#pragma unroll 1
+      for (int jt = 0; jt < n_local && ok; ++jt) {
+        const int t = cid + jt * G;
+        const int n0 = (t - (int)fdiv((uint32_t)t, args.div_nt) * args.nt) * BN;
+#pragma unroll 1
+        for (int k = 0; k < nk; ++k, ++it) {
+          const int bs = it % L::kBitStages;
+          const uint32_t ph = (uint32_t)(it / L::kBitStages) & 1u;
+          if (!__all_sync(0xffffffffu, mbar_wait_backoff(bits_empty(bs), ph ^ 1u, 64))) { ok = false; break; }
+          if (elect_one()) {
+            mbar_arrive_expect_tx(bits_full(bs), (uint32_t)L::kBitSlot);
+            tma_load_2d(sBits + (uint32_t)(bs * L::kBitSlot), &tmap_w, bits_full(bs), (kb + k) * (kBK / 8), n0);
+          }
+          __syncwarp();
+        }
+      }
+      // drain: every bits load issued has landed before the CTA may exit
+      if (!ok) {
+        for (int i = it - L::kBitStages < 0 ? 0 : it - L::kBitStages; i < it; ++i)
+          mbar_wait(bits_full(i % L::kBitStages), (uint32_t)(i / L::kBitStages) & 1u);
+      }
+      __syncwarp();
+    }
     if constexpr (BX == 0) {
     if (!args.early) grid_dep_wait();
     // =================== TMA producer (filters) ===================

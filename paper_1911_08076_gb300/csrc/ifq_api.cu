@@ -116,7 +116,7 @@ cudaError_t launch_k_cluster(void (*kern)(Exp...), int cluster, dim3 grid, dim3 
 // tile.
 template <int BN, int GB, int SB, int SBO, int KS = 1, int BX = 0>
 struct TcInst {
-  using L = TcSmem<BN, SBO, KS>;
+  using L = TcSmem<BN, SBO, KS, BX>;
   static_assert(L::bytes <= 232448, "shared memory budget");
   static constexpr auto kern = conv_tc_kernel<BN, GB, SB, SBO, KS, BX>;
   static cudaError_t set_attr() {
@@ -589,6 +589,19 @@ bool encode_wmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, 
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// TMA descriptor of the filter sign bits in the e4m3 rows' K order ([cout][Kpad / 8] bytes after the
+// sign words): boxes of bn rows x 16 bytes (one K stage), no swizzle.
+bool encode_bitmap(const ifq_conv_desc* d, const ConvGeom& g, const void* w_prep, int bn, CUtensorMap* tm) {
+  if (!get_encode()) return false;
+  cuuint64_t gdim[2] = {(cuuint64_t)(g.Kpad / 8), (cuuint64_t)d->cout};
+  cuuint64_t gstride[1] = {(cuuint64_t)(g.Kpad / 8)};
+  cuuint32_t box[2] = {16u, (cuuint32_t)bn};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, (uint8_t*)const_cast<void*>(w_prep) + prep_pbits_offset(d, g),
+                  gdim, gstride, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 void fill_conv_args(const ifq_conv_desc* d, const ConvGeom& g, int bn, const void* x, const int32_t* thr,
                     const int8_t* sign, uint8_t* yc, int32_t* ya, ConvArgs* a, bool stack = false) {
   a->x = (const uint8_t*)x;
@@ -694,17 +707,19 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
       else if (g.sb == 4) choose_split<16, 4, 4>(g, d->cout, nsm, &bn, &ks);
       else choose_split<16, 4, 2>(g, d->cout, nsm, &bn, &ks);
     }
-    CUtensorMap tm;
-    if (!encode_wmap(d, g, w_prep, bn, &tm)) return IFQ_ECUDA;
     ConvArgs a;
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
     a.early = early ? 1 : 0;
     a.wbits = g.in8 ? nullptr : (const uint8_t*)w_prep + prep_pbits_offset(d, g);
     // Filter tiles expanded from sign bits in shared memory where the filters are streamed from DRAM
-    // about once (at most two 128-row tiles, the fully connected layers): the split instance only.
-    // IFQ_TC_BX = 0 / 2 forbids / forces it where the split instance runs.
+    // about once (at most two 128-row tiles, the fully connected layers): the split instance only,
+    // its TMA warp streaming the bits.  IFQ_TC_BX = 0 / 2 forbids / forces it where the split
+    // instance runs.
     const int bx_env = env_int("IFQ_TC_BX", 1);
-    const bool bx = bx_env != 0 && (bx_env == 2 || ceil_div(g.M, kBM) <= 2);
+    const bool bx = bx_env != 0 && (bx_env == 2 || ceil_div(g.M, kBM) <= 2) && bn == 64 && ks == 2 && gb == 16 &&
+                    g.sbi == 2 && g.sb == 2;
+    CUtensorMap tm;
+    if (!(bx ? encode_bitmap(d, g, w_prep, bn, &tm) : encode_wmap(d, g, w_prep, bn, &tm))) return IFQ_ECUDA;
     if (g.sbi == 2 && g.sb == 2) {
       if (gb == 16) e = launch_tc_gb<16, 2, 2>(bn, ks, tm, a, nsm, st, bx);
       else if (gb == 8) e = launch_tc_gb<8, 2, 2>(bn, ks, tm, a, nsm, st);
