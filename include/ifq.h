@@ -93,6 +93,9 @@ int ifq_version(void);
  *   IFQ_TC_BN        = 32 / 64 / 128: the tensor-core kernel's output-channel tile width.
  *   IFQ_TC_KS        = 1 / 2: forbid / force splitting K over clusters of two CTAs (by default only
  *                      layers that would leave more than half of the SMs idle are split).
+ *   IFQ_TC_BX        = 1 / 2: the split tensor-core kernel expands its filter tiles in shared memory
+ *                      from the sign bits (1 bit per weight read instead of 8) for layers with at most
+ *                      two 128-row tiles / wherever it runs (off by default: not faster where measured).
  *   IFQ_PDL          = 0: launch without programmatic dependent launch.
  *   IFQ_GRAPH_BRANCH = 0: capture stacks as one chain, without side branches.
  *   IFQ_STACK        = 1: run qualifying stacks as one persistent launch (ifq_forward).

@@ -711,11 +711,13 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     fill_conv_args(d, g, bn, x, thr, sign, yc, ya, &a);
     a.early = early ? 1 : 0;
     a.wbits = g.in8 ? nullptr : (const uint8_t*)w_prep + prep_pbits_offset(d, g);
-    // Filter tiles expanded from sign bits in shared memory where the filters are streamed from DRAM
-    // about once (at most two 128-row tiles, the fully connected layers): the split instance only,
-    // its TMA warp streaming the bits.  IFQ_TC_BX = 0 / 2 forbids / forces it where the split
-    // instance runs.
-    const int bx_env = env_int("IFQ_TC_BX", 1);
+    // Filter tiles expanded from sign bits in shared memory (the split instance only, its TMA warp
+    // streaming the bits): opt-in.  It reads 1 bit per weight from DRAM instead of an e4m3 byte, but
+    // on AlexNet's FC layers (b128) it measured 22.4 / 16.3 us against 20.6 / 16.4 us for FC6 / FC7:
+    // those single-tile launches are bound by the K-stage pipeline's latency, not by the filter
+    // stream.  IFQ_TC_BX = 1 takes it where the filters are read about once (at most two 128-row
+    // tiles), 2 wherever the split instance runs.
+    const int bx_env = env_int("IFQ_TC_BX", 0);
     const bool bx = bx_env != 0 && (bx_env == 2 || ceil_div(g.M, kBM) <= 2) && bn == 64 && ks == 2 && gb == 16 &&
                     g.sbi == 2 && g.sb == 2;
     CUtensorMap tm;

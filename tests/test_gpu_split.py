@@ -150,9 +150,9 @@ def test_split_k_with_filter_tiles_from_sign_bits(case, monkeypatch):
     test_split_k_matches_oracle(case, monkeypatch)
 
 
-def test_fc_layers_take_the_sign_bit_filters_by_default(monkeypatch):
-    """AlexNet's FC6 and FC7 shapes (one 128-row tile): the default run (filter tiles from sign bits)
-    equals the run that loads e4m3 filter tiles, codes and accumulators."""
+def test_fc_layers_with_sign_bit_filters_equal_e4m3_filter_tiles(monkeypatch):
+    """AlexNet's FC6 and FC7 shapes (one 128-row tile): the run with filter tiles from sign bits
+    (IFQ_TC_BX = 1) equals the run that loads e4m3 filter tiles, codes and accumulators."""
     rng = np.random.default_rng(6)
     for (B, H, C, cout, k, mode) in ((128, 6, 256, 4096, 6, ifq.IFQ_OUT_CODES), (128, 1, 4096, 4096, 1, ifq.IFQ_OUT_ACC)):
         x = rng.integers(0, 4, (B, H, H, C), dtype=np.uint8)
