@@ -246,7 +246,7 @@ def cpu_baseline(wl, x, params, seconds: float):
     O.build()
     threads = len(os.sched_getaffinity(0))
     per_img = sum(conv_ops(l, 1) for l in wl.layers if l.kind == "conv")
-    n_done, dt, n = 0, 0.0, 1
+    n_done, dt, n = 0, 0.0, threads   # one image per host thread to start with
     while dt < seconds and n_done < wl.batch:
         n = min(n, wl.batch - n_done)
         t0 = time.perf_counter()
