@@ -381,7 +381,8 @@ def job_throughput(ops_per_rank_step: float, world: int, step_ms_max: float) -> 
     return world * ops_per_rank_step / (step_ms_max * 1e-3) / 1e12
 
 
-PATH_NAMES = {0: "auto", 1: "conv_tc_kernel", 2: "bitserial", 3: "conv_direct_kernel", 4: "conv_win_kernel"}
+PATH_NAMES = {0: "auto", 1: "conv_tc_kernel", 2: "bitserial", 3: "conv_direct_kernel", 4: "conv_win_kernel",
+              5: "conv_warp_kernel"}
 
 
 def kernel_of(ifq, st, li):

@@ -72,7 +72,14 @@ typedef enum {
 enum { IFQ_OUT_CODES = 1, IFQ_OUT_ACC = 2, IFQ_OUT_BOTH = 3 };
 
 /* Kernel path of a convolution (ifq_conv_desc.path). */
-enum { IFQ_PATH_AUTO = 0, IFQ_PATH_TC = 1, IFQ_PATH_BITSERIAL = 2, IFQ_PATH_DIRECT = 3, IFQ_PATH_WIN = 4 };
+enum {
+  IFQ_PATH_AUTO = 0,
+  IFQ_PATH_TC = 1,
+  IFQ_PATH_BITSERIAL = 2,
+  IFQ_PATH_DIRECT = 3,
+  IFQ_PATH_WIN = 4,
+  IFQ_PATH_WARP = 5
+};
 
 /* Layer kinds of ifq_forward. */
 enum { IFQ_LAYER_CONV = 1, IFQ_LAYER_POOL = 2, IFQ_LAYER_FIXED = 3 };
@@ -86,10 +93,12 @@ int ifq_version(void);
 /*
  * Environment switches, read on every call that uses them (for experiments; the defaults are the
  * measured best):
- *   IFQ_FORCE_PATH   = 1 / 2 / 3 / 4: request IFQ_PATH_TC / IFQ_PATH_BITSERIAL / IFQ_PATH_DIRECT /
- *                      IFQ_PATH_WIN where a descriptor says IFQ_PATH_AUTO (ifq_conv_plan reports the
- *                      result).
+ *   IFQ_FORCE_PATH   = 1 / 2 / 3 / 4 / 5: request IFQ_PATH_TC / IFQ_PATH_BITSERIAL / IFQ_PATH_DIRECT /
+ *                      IFQ_PATH_WIN / IFQ_PATH_WARP where a descriptor says IFQ_PATH_AUTO
+ *                      (ifq_conv_plan reports the result).
  *   IFQ_WIN          = 0: never take the window path (IFQ_PATH_WIN requests take the tensor-core path).
+ *   IFQ_WARP         = 0: never take the warp-MMA path (IFQ_PATH_WARP requests take the tensor-core
+ *                      path).
  *   IFQ_TC_BN        = 32 / 64 / 128: the tensor-core kernel's output-channel tile width.
  *   IFQ_TC_KS        = 1 / 2: forbid / force splitting K over clusters of two CTAs (by default only
  *                      layers that would leave more than half of the SMs idle are split).
@@ -218,8 +227,15 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
 
 /*
  * The kernel path ifq_conv2bit takes for `d` (host; reads IFQ_FORCE_PATH as
- * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT or
- * IFQ_PATH_WIN.  The window path serves stride-1 k x k layers with "same"
+ * ifq_conv2bit does): IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT,
+ * IFQ_PATH_WIN or IFQ_PATH_WARP.  The warp-MMA path (mma.sync e4m3 tiles of
+ * 16 pixels x 8 channels, accumulators and the fused pool in registers)
+ * serves 3 x 3 stride-1 layers with padding 1 on 2-bit codes with cin 8 or 16
+ * or on 8-bit values with cin 4, with 2-bit codes or accumulators out,
+ * cout 8, 16 or 32, and no pool or a 2 x 2 pool on even sizes; it is the
+ * default (where it was measured faster) for such layers on codes with cin 8
+ * and for such layers on 8-bit values without a pool, and a request for it
+ * elsewhere takes the tensor-core path.  The window path serves stride-1 k x k layers with "same"
  * padding (k odd, <= 7) on 2-bit codes with cin 16 or a multiple of 32, cout
  * 32, 64 or a multiple of 128, no pool or a 2 x 2 pool on even sizes, input
  * rows of whole 16-byte units, output rows of at most 256 pixels, and a

@@ -116,14 +116,6 @@ __device__ __forceinline__ uint64_t sdesc_none(uint32_t saddr, uint32_t lbo, uin
          ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
 }
 
-// 1-D bulk copy global -> shared on the copy engine, completing on an mbarrier (both addresses
-// 16-byte aligned, `bytes` a multiple of 16).
-__device__ __forceinline__ void bulk_copy_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-               "l"(src), "r"(bytes), "r"(bar)
-               : "memory");
-}
-
 // 32 lanes x 32 consecutive columns of tensor memory -> 32 registers, with the wait in the same
 // asm statement (the destination registers are written asynchronously until the wait).
 __device__ __forceinline__ void tmem_ld32_sync(uint32_t t0, uint32_t (&v)[32]) {

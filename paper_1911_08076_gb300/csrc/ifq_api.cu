@@ -17,6 +17,7 @@
 #include "conv_bitserial.cuh"
 #include "conv_direct.cuh"
 #include "conv_tc.cuh"
+#include "conv_warp.cuh"
 #include "conv_win.cuh"
 #include "ifq.h"
 #include "pool_pack.cuh"
@@ -192,6 +193,29 @@ struct DevState {
 };
 DevState g_dev[kMaxDevices];
 
+// The warp-MMA kernel's instances (conv_warp.cuh) and their shared-memory limit.
+constexpr int kWarpMaxSmem = 200 * 1024;
+constexpr long long kWarpSmPerSm = 226 * 1024;   // shared memory of an SM available to CTAs
+template <int E, int NT, int POOL, int IN8>
+cudaError_t set_warp_attr() {
+  return cudaFuncSetAttribute(conv_warp_kernel<E, NT, POOL, IN8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kWarpMaxSmem);
+}
+cudaError_t set_warp_attrs() {
+  cudaError_t e = cudaSuccess;
+  auto set = [&](cudaError_t r) { if (e == cudaSuccess) e = r; };
+  set(set_warp_attr<8, 1, 1, 1>()); set(set_warp_attr<8, 1, 2, 1>());
+  set(set_warp_attr<8, 2, 1, 1>()); set(set_warp_attr<8, 2, 2, 1>());
+  set(set_warp_attr<8, 4, 1, 1>()); set(set_warp_attr<8, 4, 2, 1>());
+  set(set_warp_attr<8, 1, 1, 0>()); set(set_warp_attr<8, 1, 2, 0>());
+  set(set_warp_attr<8, 2, 1, 0>()); set(set_warp_attr<8, 2, 2, 0>());
+  set(set_warp_attr<8, 4, 1, 0>()); set(set_warp_attr<8, 4, 2, 0>());
+  set(set_warp_attr<16, 1, 1, 0>()); set(set_warp_attr<16, 1, 2, 0>());
+  set(set_warp_attr<16, 2, 1, 0>()); set(set_warp_attr<16, 2, 2, 0>());
+  set(set_warp_attr<16, 4, 1, 0>()); set(set_warp_attr<16, 4, 2, 0>());
+  return e;
+}
+
 // Per-device one-time setup (shared-memory limits of the kernels, SM count).
 int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
   int dev = 0;
@@ -212,6 +236,7 @@ int ensure_init(int* nsm_out, bool* stack_ok = nullptr) {
         cudaFuncSetAttribute(conv_win_kernel<1, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kWinMaxSmem) !=
             cudaSuccess)
       return IFQ_ECUDA;
+    if (set_warp_attrs() != cudaSuccess) return IFQ_ECUDA;
     if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return IFQ_ECUDA;
     if (cudaFuncSetAttribute(conv_stack_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, StackSmem::bytes) !=
         cudaSuccess)
@@ -289,7 +314,7 @@ int check_conv(const ifq_conv_desc* d, ConvGeom* g) {
   if (d->cin % 4 != 0) return IFQ_ESHAPE;
   if (d->out_mode < IFQ_OUT_CODES || d->out_mode > IFQ_OUT_BOTH) return IFQ_EINVAL;
   if ((d->out_mode & IFQ_OUT_CODES) && d->cout % 4 != 0) return IFQ_ESHAPE;
-  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_WIN) return IFQ_EINVAL;
+  if (d->path < IFQ_PATH_AUTO || d->path > IFQ_PATH_WARP) return IFQ_EINVAL;
   const long long K = (long long)d->kh * d->kw * d->cin;
   const long long M = (long long)d->n * g->ho * g->wo;
   if (K > kMaxK || d->cout > 65536 || M >= (1LL << 31)) return IFQ_ERANGE;
@@ -460,16 +485,116 @@ bool win_wins(const ifq_conv_desc* d, const ConvGeom& g) {
   return g.pool == 2 && d->cin <= 64 && win_supported(d, g);
 }
 
+// Geometry of the warp-MMA kernel (conv_warp.cuh) for a layer, or false where it does not apply:
+// 3 x 3, stride 1, padding 1; 2-bit codes in with cin 8 or 16, or 8-bit values with cin 4; 2-bit
+// codes and / or int32 accumulators out, cout 8, 16 or 32; no pool or a 2 x 2 pool on even sizes;
+// a band of at least two output rows within the shared memory of one CTA.  Fills every field but
+// the pointers; *E and *NT select the instance.
+bool warp_plan(const ifq_conv_desc* d, const ConvGeom& g, WarpConvArgs* wa, size_t* smem, int* E, int* NT) {
+  if (env_int("IFQ_WARP", 1) == 0) return false;
+  if (d->kh != 3 || d->kw != 3 || d->stride != 1 || d->pad != 1) return false;
+  if (g.in8 ? d->cin != 4 : !(g.sbi == 2 && (d->cin == 8 || d->cin == 16))) return false;
+  if (g.kb != 2 || !(d->cout == 8 || d->cout == 16 || d->cout == 32)) return false;
+  if (g.pool != 1 && g.pool != 2) return false;
+  if (g.pool == 2 && ((g.ho & 1) || (g.wo & 1))) return false;
+  const int e = g.in8 ? 8 : d->cin, nt = d->cout / 8;
+  const int pp = e / 8, ksd = (3 * pp + 3) / 4, nb = nt * 3 * ksd;
+  const int strips = ceil_div(g.wo, 16);
+  const long long row_bytes = (long long)(16 * strips + 2) * e;
+  const int cinb = g.in8 ? d->cin : d->cin / 4;
+  const long long raw_pitch = (long long)g.wo * cinb;
+  const int bulk = raw_pitch % 16 == 0 ? 1 : 0;   // whole 16-byte units: the copy engine stages the rows
+  if (row_bytes > kWarpMaxSmem) return false;
+  // output rows per band: up to 16, fewer while two CTAs' shared memory would not fit an SM
+  // (then while one would not), so that a CTA's copy and expansion overlap the other's MMAs
+  auto bytes_of = [&](int rb) {
+    return (long long)warp_smem(nb, d->cout, rb, (int)row_bytes, (int)raw_pitch, bulk).bytes;
+  };
+  int rb = std::min(16, (int)round_up((size_t)g.ho, 2));
+  while (rb > 2 && 2 * bytes_of(rb) > kWarpSmPerSm) rb -= 2;
+  while (rb > 2 && bytes_of(rb) > kWarpMaxSmem) rb -= 2;
+  if (bytes_of(rb) > kWarpMaxSmem) return false;
+  if (wa) {
+    memset(wa, 0, sizeof(*wa));
+    wa->n = d->n; wa->h = g.ho; wa->w = g.wo; wa->cin = d->cin; wa->cout = d->cout; wa->kwords = g.kwords;
+    wa->pho = g.pho; wa->pwo = g.pwo;
+    wa->strips = strips;
+    wa->rb = rb;
+    wa->bands = ceil_div(g.ho, rb);
+    wa->row_bytes = (int)row_bytes;
+    wa->units = strips * (rb / 2);
+    wa->bulk = bulk;
+    wa->raw_pitch = (int)raw_pitch;
+    wa->total = d->n * wa->bands;
+    wa->div_bands = make_fastdiv((uint32_t)wa->bands);
+    wa->div_strips = make_fastdiv((uint32_t)strips);
+    wa->div_slots = make_fastdiv((uint32_t)(16 * strips + 2));
+  }
+  if (smem) *smem = (size_t)bytes_of(rb);
+  if (E) *E = e;
+  if (NT) *NT = nt;
+  return true;
+}
+
+bool warp_supported(const ifq_conv_desc* d, const ConvGeom& g) {
+  return warp_plan(d, g, nullptr, nullptr, nullptr, nullptr);
+}
+
+// Where the warp-MMA kernel is the default (measured on GB300, full-size layers at batch 64, L2
+// flushed, against the kernel each layer took before): 2-bit layers with 8 input channels
+// (IFQ-Tinier-YOLO conv2, 8 -> 16 at 208 x 208: 46 vs 103 us on the narrow bit-serial kernel with the
+// fused pool, 62 vs 107 us without) and 8-bit-input layers without a fused pool (3 x 3 4 -> 8 at
+// 416 x 416: 144 vs 207 us on the direct kernel).  Elsewhere it loses: one e4m3 mma.sync issues about
+// four instructions on this GPU, and the tcgen05 window kernel (16-channel layers: Tiny-YOLO conv2
+// 66 vs 124 us) or the direct kernel (the pooled first layer: 91 vs 107 us) stays ahead.
+bool warp_wins(const ifq_conv_desc* d, const ConvGeom& g) {
+  return warp_supported(d, g) && (g.in8 ? g.pool == 1 : d->cin == 8);
+}
+
+// A persistent launch: as many CTAs as fit the SMs at once (at most one per band).
+template <int E, int NT, int POOL, int IN8>
+cudaError_t launch_warp_inst(int nsm, size_t smem, cudaStream_t st, const WarpConvArgs& a) {
+  const int threads = warp_conv_threads(E, NT);
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, conv_warp_kernel<E, NT, POOL, IN8>, threads,
+                                                                smem);
+  if (e != cudaSuccess) return e;
+  const int grid = std::max(1, std::min(a.total, nsm * std::max(1, per_sm)));
+  return launch_k(conv_warp_kernel<E, NT, POOL, IN8>, dim3((unsigned)grid), dim3((unsigned)threads), smem, st, a);
+}
+
+template <int E, int NT>
+cudaError_t launch_warp_en(int pool, bool in8, int nsm, size_t smem, cudaStream_t st, const WarpConvArgs& a) {
+  if constexpr (E == 8) {
+    if (in8)
+      return pool == 2 ? launch_warp_inst<E, NT, 2, 1>(nsm, smem, st, a) : launch_warp_inst<E, NT, 1, 1>(nsm, smem, st, a);
+  }
+  return pool == 2 ? launch_warp_inst<E, NT, 2, 0>(nsm, smem, st, a) : launch_warp_inst<E, NT, 1, 0>(nsm, smem, st, a);
+}
+
+cudaError_t launch_warp(int E, int NT, int pool, bool in8, int nsm, size_t smem, cudaStream_t st,
+                        const WarpConvArgs& a) {
+  if (E == 8)
+    return NT == 1 ? launch_warp_en<8, 1>(pool, in8, nsm, smem, st, a)
+                   : (NT == 2 ? launch_warp_en<8, 2>(pool, in8, nsm, smem, st, a)
+                              : launch_warp_en<8, 4>(pool, in8, nsm, smem, st, a));
+  return NT == 1 ? launch_warp_en<16, 1>(pool, false, nsm, smem, st, a)
+                 : (NT == 2 ? launch_warp_en<16, 2>(pool, false, nsm, smem, st, a)
+                            : launch_warp_en<16, 4>(pool, false, nsm, smem, st, a));
+}
+
 int choose_path(const ifq_conv_desc* d, const ConvGeom& g) {
   int path = d->path;
   if (path == IFQ_PATH_AUTO) {
     const int forced = env_int("IFQ_FORCE_PATH", 0);
     path = forced ? forced
-                  : (direct_supported(d, g) ? IFQ_PATH_DIRECT
-                                            : (win_wins(d, g) ? IFQ_PATH_WIN
-                                                                   : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL
-                                                                                        : IFQ_PATH_TC)));
+                  : (warp_wins(d, g) ? IFQ_PATH_WARP
+                                     : (direct_supported(d, g) ? IFQ_PATH_DIRECT
+                                                               : (win_wins(d, g) ? IFQ_PATH_WIN
+                                                                                 : (narrow_wins(d, g) ? IFQ_PATH_BITSERIAL
+                                                                                                      : IFQ_PATH_TC))));
   }
+  if (path == IFQ_PATH_WARP && !warp_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_WIN && !win_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_DIRECT && !direct_supported(d, g)) path = IFQ_PATH_TC;
   if (path == IFQ_PATH_TC && !tc_supported(d, g)) path = IFQ_PATH_BITSERIAL;
@@ -680,6 +805,18 @@ int run_conv(const ifq_conv_desc* d, const void* x, const void* w_prep, const in
     else if (d->cout <= 8) e = launch_k(conv_direct_kernel<4>, grid, block, 0, st, a);
     else if (d->cout <= 16) e = launch_k(conv_direct_kernel<8>, grid, block, 0, st, a);
     else e = launch_k(conv_direct_kernel<16>, grid, block, 0, st, a);
+  } else if (path == IFQ_PATH_WARP) {
+    WarpConvArgs wa;
+    size_t smem = 0;
+    int E = 0, NT = 0;
+    if (!warp_plan(d, g, &wa, &smem, &E, &NT)) return IFQ_EUNSUPPORTED;
+    wa.x = (const uint8_t*)x;
+    wa.wbits = (const uint32_t*)((const uint8_t*)w_prep + prep_bits_offset(d, g));
+    wa.thr = thr;
+    wa.sign = sign;
+    wa.y_codes = yc;
+    wa.y_acc = ya;
+    e = launch_warp(E, NT, g.pool, g.in8, nsm, smem, st, wa);
   } else if (path == IFQ_PATH_WIN) {
     WinArgs wa;
     size_t smem = 0;
@@ -963,7 +1100,8 @@ bool stack_eligible(const ifq_layer* layers, int nlayers, size_t* bytes) {
     // the persistent kernel computes every layer with the tensor-core data path: layers whose own
     // launch would take that path or the window path qualify
     const int p = choose_path(&layers[i].conv, g);
-    if (!(p == IFQ_PATH_TC || (p == IFQ_PATH_WIN && tc_supported(&layers[i].conv, g)))) return false;
+    if (!(p == IFQ_PATH_TC || ((p == IFQ_PATH_WIN || p == IFQ_PATH_WARP) && tc_supported(&layers[i].conv, g))))
+      return false;
     tab += g.Kpad / (4 * granule_bytes(&layers[i].conv, g, true));
   }
   if (tab > kMaxStackTab) return false;

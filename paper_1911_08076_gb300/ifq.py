@@ -21,7 +21,7 @@ _lib = None
 
 IFQ_OK, IFQ_EINVAL, IFQ_ESHAPE, IFQ_EALIGN, IFQ_ERANGE, IFQ_ECUDA, IFQ_ETIMEOUT, IFQ_EUNSUPPORTED, IFQ_EWORKSPACE = range(9)
 IFQ_OUT_CODES, IFQ_OUT_ACC, IFQ_OUT_BOTH = 1, 2, 3
-IFQ_PATH_AUTO, IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT, IFQ_PATH_WIN = 0, 1, 2, 3, 4
+IFQ_PATH_AUTO, IFQ_PATH_TC, IFQ_PATH_BITSERIAL, IFQ_PATH_DIRECT, IFQ_PATH_WIN, IFQ_PATH_WARP = 0, 1, 2, 3, 4, 5
 IFQ_LAYER_CONV, IFQ_LAYER_POOL, IFQ_LAYER_FIXED = 1, 2, 3
 IFQ_FORWARD_LAYERS, IFQ_FORWARD_PERSISTENT = 1, 2
 

@@ -311,3 +311,40 @@ def test_window_path_plan():
             del os.environ["IFQ_WIN"]
         else:
             os.environ["IFQ_WIN"] = old
+
+
+def test_warp_path_plan():
+    """The warp-MMA path applies to 3 x 3 stride-1 layers with padding 1 on 2-bit codes with cin 8 or
+    16 or on 8-bit values with cin 4, cout 8, 16 or 32, no pool or a 2 x 2 pool on even sizes; a
+    request for it elsewhere takes the tensor-core path, and IFQ_WARP=0 turns it off."""
+    WARP, TC = ifq.IFQ_PATH_WARP, ifq.IFQ_PATH_TC
+    plan = lambda *a, **k: ifq.ifq_conv_plan(ifq.conv_desc(*a, **k))
+    assert plan(64, 208, 208, 8, 16, 3, 1, 1, pool=2, path=WARP) == WARP
+    assert plan(64, 416, 416, 4, 8, 3, 1, 1, pool=2, in_bits=8, path=WARP) == WARP
+    assert plan(64, 208, 208, 16, 32, 3, 1, 1, pool=2, path=WARP) == WARP
+    assert plan(2, 13, 17, 8, 8, 3, 1, 1, out_mode=ifq.IFQ_OUT_BOTH, path=WARP) == WARP
+    # the default where it was measured faster: 8-channel codes, and 8-bit values without a pool
+    assert plan(64, 208, 208, 8, 16, 3, 1, 1, pool=2) == WARP
+    assert plan(64, 208, 208, 8, 16, 3, 1, 1) == WARP
+    assert plan(64, 416, 416, 4, 8, 3, 1, 1, in_bits=8) == WARP
+    assert plan(64, 416, 416, 4, 8, 3, 1, 1, pool=2, in_bits=8) == ifq.IFQ_PATH_DIRECT
+    assert plan(64, 208, 208, 16, 32, 3, 1, 1, pool=2) == ifq.IFQ_PATH_WIN
+    assert plan(2, 16, 16, 32, 64, 3, 1, 1, path=WARP) == TC          # cin 32
+    assert plan(2, 16, 16, 16, 64, 3, 1, 1, path=WARP) == TC          # cout 64
+    assert plan(2, 16, 16, 16, 24, 3, 1, 1, path=WARP) == TC          # cout 24
+    assert plan(2, 16, 16, 16, 32, 3, 2, 1, path=WARP) == TC          # stride 2
+    assert plan(2, 16, 16, 16, 32, 5, 1, 2, path=WARP) == TC          # 5 x 5
+    assert plan(2, 16, 16, 16, 32, 3, 1, 0, path=WARP) == TC          # no padding
+    assert plan(2, 16, 16, 4, 8, 3, 1, 1, path=WARP) == TC            # cin 4 on codes
+    assert plan(2, 16, 16, 8, 16, 3, 1, 1, kbits=4, path=WARP) == TC  # 4-bit codes
+    assert plan(2, 16, 16, 16, 32, 3, 1, 1, pool=4, path=WARP) == TC  # 4 x 4 pool
+    import os
+    old = os.environ.get("IFQ_WARP")
+    os.environ["IFQ_WARP"] = "0"
+    try:
+        assert plan(64, 208, 208, 8, 16, 3, 1, 1, pool=2, path=WARP) == TC
+    finally:
+        if old is None:
+            del os.environ["IFQ_WARP"]
+        else:
+            os.environ["IFQ_WARP"] = old

@@ -18,9 +18,12 @@ def _status(fn, *a, **kw):
 
 def test_8bit_input_plan_and_refusals():
     d = ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, ifq.IFQ_OUT_BOTH, in_bits=8)
-    assert ifq.ifq_conv_plan(d) == DI                          # few channels: the direct path
+    assert ifq.ifq_conv_plan(d) == ifq.IFQ_PATH_WARP           # 3 x 3, few channels, no pool: warp MMAs
     d.path = TC
     assert ifq.ifq_conv_plan(d) == TC
+    d.path = DI
+    assert ifq.ifq_conv_plan(d) == DI
+    assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 8, 5, 1, 2, in_bits=8)) == DI      # 5 x 5: direct
     assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 8, 3, 1, 1, pool=2, in_bits=8)) == DI
     assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 4, 64, 3, 1, 1, in_bits=8)) == TC      # cout > 32
     assert ifq.ifq_conv_plan(ifq.conv_desc(2, 20, 20, 32, 8, 3, 1, 1, in_bits=8)) == TC      # K = 288 > 257

@@ -103,10 +103,11 @@ def test_conv_plan_refuses_a_fused_pool_off_the_tensor_cores():
 
 
 def test_conv_plan_takes_the_narrow_bitserial_kernel_where_it_wins():
-    """2-bit 3x3 stride-1 layers with cin * cout <= 128 (IFQ-Tinier-YOLO's conv2, 8 -> 16) run on
-    the narrow bit-serial kernel; wider ones take the tensor cores (the window path where it
-    applies)."""
-    assert ifq.ifq_conv_plan(ifq.conv_desc(64, 208, 208, 8, 16, 3, 1, 1, pool=2)) == BS
+    """2-bit 3x3 stride-1 layers with cin * cout <= 128 run on the narrow bit-serial kernel unless
+    the warp-MMA kernel takes them (8 input channels: IFQ-Tinier-YOLO's conv2, 8 -> 16); wider ones
+    take the tensor cores (the window path where it applies)."""
+    assert ifq.ifq_conv_plan(ifq.conv_desc(64, 208, 208, 8, 16, 3, 1, 1, pool=2)) == ifq.IFQ_PATH_WARP
+    assert ifq.ifq_conv_plan(ifq.conv_desc(64, 208, 208, 4, 16, 3, 1, 1, pool=2)) == BS
     assert ifq.ifq_conv_plan(ifq.conv_desc(64, 208, 208, 16, 32, 3, 1, 1, pool=2)) == ifq.IFQ_PATH_WIN
     assert ifq.ifq_conv_plan(ifq.conv_desc(2, 16, 16, 8, 16, 3, 2, 1)) == TC      # stride 2
     assert ifq.ifq_conv_plan(ifq.conv_desc(2, 16, 16, 16, 32, 3, 1, 1, pool=2, path=BS)) == BS
