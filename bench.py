@@ -164,15 +164,21 @@ def measure_rates(stream):
     L.bench_tc_e4m3_tops.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.POINTER(dbl)]
     L.bench_mma_s8_tops.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.POINTER(dbl)]
     out = {}
+    L.bench_tc_e4m3_tops_a.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                       ctypes.POINTER(dbl)]
     for n in (128, 256):
         v = dbl(0.0)
         rc = L.bench_tc_e4m3_tops(n, 8192, 5, ctypes.c_void_p(stream.cuda_stream), ctypes.byref(v))
         out[f"tcgen05_e4m3_n{n}_tops"] = v.value if rc == 0 else None
     v = dbl(0.0)
+    rc = L.bench_tc_e4m3_tops_a(128, 1, 8192, 5, ctypes.c_void_p(stream.cuda_stream), ctypes.byref(v))
+    out["tcgen05_e4m3_tmem_a_n128_tops"] = v.value if rc == 0 else None
+    v = dbl(0.0)
     rc = L.bench_mma_s8_tops(4096, 3, ctypes.c_void_p(stream.cuda_stream), ctypes.byref(v))
     out["mma_sync_s8_tops"] = v.value if rc == 0 else None
     out["how"] = ("same process, before the timed regions: one CTA per SM issuing M128xNxK32 e4m3 tcgen05 MMAs "
-                  "back to back; 4 CTAs x 8 warps per SM issuing m16n8k32 s8 mma.sync; 2 ops per MAC")
+                  "back to back (A in shared memory; tmem_a: A in tensor memory, as the conv issues them); "
+                  "4 CTAs x 8 warps per SM issuing m16n8k32 s8 mma.sync; 2 ops per MAC")
     return out
 
 
@@ -610,7 +616,9 @@ def run_ours(args):
     r["vs_measured_rates"] = {
         "tcgen05_e4m3_n128": frac(rates.get("tcgen05_e4m3_n128_tops")),
         "tcgen05_e4m3_n256": frac(rates.get("tcgen05_e4m3_n256_tops")),
-        "note": "achieved / the e4m3 tcgen05 rate measured in this process (the conv's own instruction)"}
+        "tcgen05_e4m3_tmem_a_n128": frac(rates.get("tcgen05_e4m3_tmem_a_n128_tops")),
+        "note": "achieved / the e4m3 tcgen05 rate measured in this process (the conv's own instruction; "
+                "tmem_a: with A in tensor memory, the operand form the conv issues)"}
     s8 = rates.get("mma_sync_s8_tops")
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,

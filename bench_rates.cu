@@ -45,9 +45,11 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t a) {
 
 constexpr int kOperandBytes = 32768;   // A: 128 rows x 128 B; B: up to 256 rows x 128 B
 
-// One CTA per SM: one thread issues `iters` M128 x N x K32 e4m3 MMAs on operands of +1.0
-// in shared memory, alternating between two accumulators; the rest of the CTA waits.
-__global__ void __launch_bounds__(128, 1) tc_e4m3_rate_kernel(int n, int iters, float* sink) {
+// One CTA per SM: one thread issues `iters` M128 x N x K32 e4m3 MMAs on operands of +1.0,
+// alternating between two accumulators; the rest of the CTA waits.  a_tmem = 0: both operands in
+// shared memory; a_tmem = 1 (N <= 128): A in tensor memory (columns 256..287, written by every
+// warp for its lane quarter), B in shared memory, the form the tensor-core conv issues.
+__global__ void __launch_bounds__(128, 1) tc_e4m3_rate_kernel(int n, int iters, int a_tmem, float* sink) {
   extern __shared__ uint8_t raw[];
   uint8_t* sm = (uint8_t*)(((uintptr_t)raw + 1023) & ~(uintptr_t)1023);
   __shared__ __align__(8) uint64_t bar;
@@ -67,15 +69,37 @@ __global__ void __launch_bounds__(128, 1) tc_e4m3_rate_kernel(int n, int iters, 
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
   const uint32_t tmem = tslot;
+  if (a_tmem) {
+    // A: 128 lanes x 32 columns of e4m3 +1.0 (four K = 32 steps of 8 columns)
+    const uint32_t ta = tmem + 256u + ((uint32_t)(warp * 32) << 16);
+    const uint32_t one = 0x38383838u;
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2};\n\t"
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%1], {%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2,%2};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(ta), "r"(ta + 16u), "r"(one)
+        : "memory");
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+  }
   if (tid == 0) {
     const uint32_t idesc = (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
     const uint64_t ad = sw128_desc(saddr(sm)), bd = sw128_desc(saddr(sm + 128 * 128));
-    for (int i = 0; i < iters; ++i)
-      asm volatile(
-          "{.reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;}" ::"r"(
-              tmem + (uint32_t)((i & 1) * 256)),
-          "l"(ad + 2 * (i & 3)), "l"(bd + 2 * (i & 3)), "r"(idesc), "r"(i > 1 ? 1 : 0)
-          : "memory");
+    if (a_tmem) {
+      for (int i = 0; i < iters; ++i)
+        asm volatile(
+            "{.reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;}" ::"r"(
+                tmem + (uint32_t)((i & 1) * 128)),
+            "r"(tmem + 256u + (uint32_t)(8 * (i & 3))), "l"(bd + 2 * (i & 3)), "r"(idesc), "r"(i > 1 ? 1 : 0)
+            : "memory");
+    } else {
+      for (int i = 0; i < iters; ++i)
+        asm volatile(
+            "{.reg .pred p; setp.ne.b32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;}" ::"r"(
+                tmem + (uint32_t)((i & 1) * 256)),
+            "l"(ad + 2 * (i & 3)), "l"(bd + 2 * (i & 3)), "r"(idesc), "r"(i > 1 ? 1 : 0)
+            : "memory");
+    }
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(saddr(&bar))
                  : "memory");
   }
@@ -125,11 +149,12 @@ int sm_count() {
 extern "C" {
 
 // Dense ops per second (2 per MAC), in TOPS, of the e4m3 tcgen05 MMA at M = 128, K = 32 and
-// the given N (a multiple of 16, 16..256), measured over `reps` launches of `iters` MMAs per
-// SM on `stream` (after one warm-up launch).  Returns 0 on success, 1 on a bad argument, 2 on a
-// CUDA error, 3 if a wait ran out.
-int bench_tc_e4m3_tops(int n, int iters, int reps, void* stream, double* tops) {
-  if (!tops || n < 16 || n > 256 || n % 16 || iters < 1 || reps < 1) return 1;
+// the given N (a multiple of 16, 16..256; at most 128 with a_tmem), A in shared memory (a_tmem = 0)
+// or in tensor memory (a_tmem = 1), measured over `reps` launches of `iters` MMAs per SM on
+// `stream` (after one warm-up launch).  Returns 0 on success, 1 on a bad argument, 2 on a CUDA
+// error, 3 if a wait ran out.
+int bench_tc_e4m3_tops_a(int n, int a_tmem, int iters, int reps, void* stream, double* tops) {
+  if (!tops || n < 16 || n > (a_tmem ? 128 : 256) || n % 16 || iters < 1 || reps < 1) return 1;
   const int sms = sm_count();
   if (sms < 1) return 2;
   cudaStream_t st = (cudaStream_t)stream;
@@ -141,9 +166,9 @@ int bench_tc_e4m3_tops(int n, int iters, int reps, void* stream, double* tops) {
   if (cudaFuncSetAttribute(tc_e4m3_rate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) == cudaSuccess &&
       cudaMalloc(&sink, sizeof(float) * sms) == cudaSuccess && cudaEventCreate(&e0) == cudaSuccess &&
       cudaEventCreate(&e1) == cudaSuccess) {
-    tc_e4m3_rate_kernel<<<sms, 128, smem, st>>>(n, 64, sink);
+    tc_e4m3_rate_kernel<<<sms, 128, smem, st>>>(n, 64, a_tmem, sink);
     cudaEventRecord(e0, st);
-    for (int r = 0; r < reps; ++r) tc_e4m3_rate_kernel<<<sms, 128, smem, st>>>(n, iters, sink);
+    for (int r = 0; r < reps; ++r) tc_e4m3_rate_kernel<<<sms, 128, smem, st>>>(n, iters, a_tmem, sink);
     cudaEventRecord(e1, st);
     float ms = 0.f;
     if (cudaEventSynchronize(e1) == cudaSuccess && cudaEventElapsedTime(&ms, e0, e1) == cudaSuccess && ms > 0.f) {
@@ -157,6 +182,11 @@ int bench_tc_e4m3_tops(int n, int iters, int reps, void* stream, double* tops) {
   if (e1) cudaEventDestroy(e1);
   if (sink) cudaFree(sink);
   return rc;
+}
+
+// bench_tc_e4m3_tops_a with A in shared memory.
+int bench_tc_e4m3_tops(int n, int iters, int reps, void* stream, double* tops) {
+  return bench_tc_e4m3_tops_a(n, 0, iters, reps, stream, tops);
 }
 
 // Dense ops per second (2 per MAC), in TOPS, of warp mma.sync.m16n8k32 s8 x s8 -> s32 with 4

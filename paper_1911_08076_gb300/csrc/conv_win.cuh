@@ -48,8 +48,8 @@
 // Y^conv, before BN and the quantizer) takes the max of A over the
 // horizontal pair in registers; the vertical pair is either two anchor rows
 // of the same thread (one output row per M row) or two warps (stacked output
-// rows), combined as codes: code(max A) is the max of the codes for a
-// positive BN scale and the min for a negative one.
+// rows), which swap halves of their horizontal maxima through shared memory,
+// so each thresholds the window maximum of half the pooled columns.
 //
 // Warps: 0-15 epilogue (lane quadrant = warp % 4, four warps a quadrant on
 // interleaved column groups), 16 TMEM allocation and MMA issue, 17-20
@@ -72,7 +72,7 @@ constexpr int kWinThreads = 32 * (kWinEpiWarps + 1 + kWinProdWarps);   // 672
 constexpr int kWinPoolGroups = 4;      // groups of 32 pooled columns a tile can have (N <= 256)
 constexpr int kWinGpw = (kWinPoolGroups + kWinEpiPerQ - 1) / kWinEpiPerQ;   // of them per epilogue warp
 constexpr int kWinProdBar = 1 + 2 * kWinEpiPerQ;   // producers' named barrier (1..2 kWinEpiPerQ: row pairs)
-constexpr int kWinXchgBytes = 4096;    // pooled codes passed between the two warps of a row pair
+constexpr int kWinXchgBytes = 3 * kWinEpiWarps * 2048;   // horizontal maxima of the row pairs (stacked rows, pooled)
 constexpr int kWinMaxMma = 64;         // MMAs per tile (K' / 32)
 constexpr int kWinTabBytes = 8 * kWinMaxMma;
 constexpr int kWinMaxSmem = 232448;    // dynamic shared memory per CTA
@@ -105,6 +105,7 @@ struct WinArgs {
   uint32_t band_bytes;     // bytes of one band buffer
   uint32_t stage_bytes;    // bytes of one staging buffer (nseg * rb * row_bytes, rounded)
   uint32_t a_bytes;        // bytes of the resident A operand: 16 KB per 128-byte K stage of the Toeplitz K
+  uint32_t xchg_bytes;     // row-pair exchange buffers: kWinXchgBytes with stacked rows and a pool, else 0
   int early;               // 1: no kernel before this one in the stream writes the filters
   FastDiv div_planes, div_pitch, div_seg, div_bands, div_chunks, div_rb;
 };
@@ -162,18 +163,6 @@ __device__ __forceinline__ uint64_t spread_bits(uint32_t x) {
   return v;
 }
 
-// Field-wise max of two words of 32 two-bit codes, after flipping (c ^ 3) the fields set in `flip`
-// and flipping the result back: the max for plain fields, the min for flipped ones.
-__device__ __forceinline__ uint64_t pool_codes2(uint64_t a, uint64_t b, uint64_t flip) {
-  constexpr uint64_t H = 0xAAAAAAAAAAAAAAAAull, L = 0x5555555555555555ull;
-  a ^= flip;
-  b ^= flip;
-  const uint64_t ha = a & H, hb = b & H;
-  const uint64_t only_a = (ha & ~hb) >> 1, only_b = (hb & ~ha) >> 1;
-  const uint64_t lo = ((a & L) & ~only_b) | ((b & L) & ~only_a);
-  return (ha | hb | lo) ^ flip;
-}
-
 // Byte offset in a band buffer of 16-byte core column c = (iy, ix, p) of the Toeplitz K, for
 // anchor 0.
 __device__ __forceinline__ uint32_t win_col_offset(const WinArgs& a, int c) {
@@ -196,9 +185,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
   const uint32_t oStage = a.a_bytes + 2 * a.band_bytes;
   const uint32_t sStage = sbase + oStage;
   const uint32_t oXchg = oStage + 2 * a.stage_bytes;
-  uint64_t* xchg = (uint64_t*)(smem + oXchg);
-  uint64_t* mtab = (uint64_t*)(smem + oXchg + kWinXchgBytes);   // B descriptors of band 0, per MMA
-  const uint32_t barBase = sbase + oXchg + kWinXchgBytes + kWinTabBytes;
+  float4* xchg4 = (float4*)(smem + oXchg);
+  uint64_t* mtab = (uint64_t*)(smem + oXchg + a.xchg_bytes);   // B descriptors of band 0, per MMA
+  const uint32_t barBase = sbase + oXchg + a.xchg_bytes + kWinTabBytes;
   auto band_full = [&](int b) { return barBase + 8u * b; };
   auto band_empty = [&](int b) { return barBase + 16u + 8u * b; };
   auto acc_full = [&](int b) { return barBase + 32u + 8u * b; };
@@ -206,7 +195,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
   auto stage_full = [&](int b) { return barBase + 64u + 8u * b; };
   const uint32_t done_bar = barBase + 80u;
   const uint32_t a_full = barBase + 88u;   // the resident A operand has landed
-  uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + kWinXchgBytes + kWinTabBytes + 104);
+  uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + a.xchg_bytes + kWinTabBytes + 104);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // CTA c takes channel tile c % nct and the band tiles c / nct, c / nct + G / nct, ... of it
@@ -412,7 +401,6 @@ __global__ void __launch_bounds__(kWinThreads, 1)
       }
     }
     const uint32_t negmask = __ballot_sync(0xffffffffu, neg);
-    const uint64_t flip = spread_bits(negmask) * 3ull;
     const int rowb = a.cout >> 2;                                  // output bytes per pixel
     const int chb = (ctile * a.ct + cg * 32) >> 2;                 // this warp's byte within a pixel
     const uint32_t lane_off = (uint32_t)(32 * q) << 16;
@@ -474,6 +462,64 @@ __global__ void __launch_bounds__(kWinThreads, 1)
         const int pw = a.w >> 1, ph = a.h >> 1;
         const int halfw = a.pitch >> 1;
         const int npool = a.ry > 1 ? (a.N >> 1) : (a.R >> 1) * halfw;
+        if (a.ry > 1) {
+          // Rows sy (even) and sy + 1 of each pooled window live in the two warps of a row pair.
+          // Each warp takes the horizontal maxima of its 32 pooled columns, hands the half the
+          // partner thresholds to it through shared memory (four 16-byte stores a lane), takes the
+          // vertical max of the half it keeps (the even row keeps pooled columns 0..15 of the group,
+          // the odd row 16..31) and thresholds only that: the quantizer sees max A over the whole
+          // 2 x 2 window, as Sec. 2.1 places the pool.  Buffers alternate with the tile parity, so a
+          // warp never overwrites a half its partner has not read yet.
+          const int g = sub;   // kWinGpw == 1: one group of 32 pooled columns per warp
+          const bool act = ok && 32 * g < npool;
+          // slots of 128 float4 ([e4][lane]): one per epilogue warp for the half it keeps (read back
+          // by the same lane), then one per tile parity and warp for the half it hands over; the
+          // partner is the warp of the other row of the pair: quadrant q ^ (ct / 32), same sub
+          float4* mine = xchg4 + (size_t)warp * 128;
+          float4* give = xchg4 + (size_t)(kWinEpiWarps + (i & 1) * kWinEpiWarps + warp) * 128;
+          const float4* take = xchg4 + (size_t)(kWinEpiWarps + (i & 1) * kWinEpiWarps + (warp ^ (a.ct >> 5))) * 128;
+          auto half = [&](auto kept_c) {
+            constexpr int kKept = decltype(kept_c)::value, kGive = 16 - kKept;
+            // pooled columns [c, c + 16) come from accumulator columns [2 c, 2 c + 32); both halves
+            // of this row's horizontal maxima go to shared memory (the kept one to this warp's own
+            // slot), so nothing stays in registers across the barrier
+            if (act) {
+#pragma unroll
+              for (int hh = 0; hh < 2; ++hh) {
+                uint32_t v[32];
+                tmem_ld32_sync(tacc + (uint32_t)(64 * g + 32 * hh), v);
+                float4* dst = (hh == 0) == (kKept == 0) ? mine : give;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                  float m4[4];
+#pragma unroll
+                  for (int j = 0; j < 4; ++j)
+                    m4[j] = fmaxf(__uint_as_float(v[8 * q4 + 2 * j]), __uint_as_float(v[8 * q4 + 2 * j + 1]));
+                  dst[q4 * 32 + lane] = make_float4(m4[0], m4[1], m4[2], m4[3]);
+                }
+              }
+            }
+            named_bar(1 + pair + 2 * sub, 64);
+            if (act) {
+              uint32_t k0 = 0, k1 = 0;
+#pragma unroll
+              for (int q4 = 0; q4 < 4; ++q4) {
+                const float4 o = take[q4 * 32 + lane], m = mine[q4 * 32 + lane];
+                code_ballot(fmaxf(m.x, o.x), 4 * q4, k0, k1);
+                code_ballot(fmaxf(m.y, o.y), 4 * q4 + 1, k0, k1);
+                code_ballot(fmaxf(m.z, o.z), 4 * q4 + 2, k0, k1);
+                code_ballot(fmaxf(m.w, o.w), 4 * q4 + 3, k0, k1);
+              }
+              const int pi = 32 * g + kKept + lane;
+              const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
+              const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
+              if (a.y_codes && lane < 16 && pi < npool && r < a.R && px < pw && py < ph)
+                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = packed(k0, k1);
+            }
+          };
+          if (odd_row) half(std::integral_constant<int, 16>{});
+          else half(std::integral_constant<int, 0>{});
+        } else {
         uint64_t own[kWinGpw];
 #pragma unroll
         for (int gi = 0; gi < kWinGpw; ++gi) own[gi] = 0ull;
@@ -483,14 +529,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int g = kWinEpiPerQ * gi + sub;
             if (32 * g < npool) {
               uint32_t k0 = 0, k1 = 0;
-              if (a.ry > 1) {
-                // pooled column pi <- columns 2 pi, 2 pi + 1 of this row
-                uint32_t v[64];
-                tmem_ld2x32_sync(tacc + (uint32_t)(64 * g), tacc + (uint32_t)(64 * g + 32), v);
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                  code_ballot(fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1])), e, k0, k1);
-              } else {
+              {
                 // pooled column (pr, px) <- columns 2 px, 2 px + 1 of anchor rows 2 pr and 2 pr + 1
                 // (pitch % 16 == 0, so 8 pooled columns are 16 aligned columns of each row)
 #pragma unroll
@@ -520,29 +559,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             }
           }
         }
-        if (a.ry > 1) {
-          // rows sy (even) and sy + 1 of the window live in two warps: the odd one hands over
-          uint64_t* xc = xchg + (size_t)((i & 1) * 2 + pair) * 128;
-          if (odd_row) {
-#pragma unroll
-            for (int gi = 0; gi < kWinGpw; ++gi) {
-              const int g = kWinEpiPerQ * gi + sub;
-              if (32 * g < npool) xc[32 * g + lane] = own[gi];
-            }
-          }
-          named_bar(1 + pair + 2 * sub, 64);
-          if (!odd_row && ok && a.y_codes) {
-#pragma unroll
-            for (int gi = 0; gi < kWinGpw; ++gi) {
-              const int pi = 32 * (kWinEpiPerQ * gi + sub) + lane;
-              const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
-              const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
-              if (pi < npool && r < a.R && px < pw && py < ph)
-                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) =
-                    pool_codes2(own[gi], xc[pi], flip);
-            }
-          }
-        } else if (ok && a.y_codes) {
+        if (ok && a.y_codes) {
 #pragma unroll
           for (int gi = 0; gi < kWinGpw; ++gi) {
             const int pi = 32 * (kWinEpiPerQ * gi + sub) + lane;
@@ -551,6 +568,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             if (pi < npool && px < pw && py < ph)
               *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = own[gi];
           }
+        }
         }
       }
       if (ok) {
