@@ -15,8 +15,9 @@
 //     multiple of 2^-9 of magnitude <= (2^k - 1) K * 2^-9, far inside the
 //     24-bit fp32 significand for the magnitudes the host admits, so the fp32
 //     accumulator in tensor memory holds it exactly: D = A / 512.
-//   * Thresholds: sign*A > T  <=>  sign*D > T/512, and T/512 is exact in fp32
-//     (|T| < 2^24), so the epilogue compares the accumulator in fp32 directly.
+//   * Thresholds: for 2-bit codes [sign*A > T] = sat(D * 512 sign - T), an exact integer
+//     saturated to {0, 1} by one fma.sat on the FMA pipe; for 3- and 4-bit codes
+//     sign*A > T  <=>  sign*D > T/512 (T/512 is exact in fp32, |T| < 2^24).
 //
 // K ordering inside each chunk of one 32-bit word of packed codes (16 two-bit
 // or 8 four-bit codes): the expansion produces byte p = 4q + t from code
@@ -67,6 +68,21 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
   const float4 g = t5[1 + q];
   return 4u * q + (uint32_t)(sv > g.x) + (uint32_t)(sv > g.y) + (uint32_t)(sv > g.z);
 }
+
+// The 2-bit code of one accumulator D = A / 512 against its column's thresholds
+// t = (-T1, -T2, -T3, 512 s), as a float 0..3, on the FMA pipe: s A - T_i = fma(D, 512 s, -T_i) is
+// an exact integer (|s A - T_i| < 2^24), and saturating it to [0, 1] gives exactly [s A > T_i].
+__device__ __forceinline__ float sat_fma(float a, float b, float c) {
+  float r;
+  asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+__device__ __forceinline__ float code3f(float d, const float4& t) {
+  return sat_fma(d, t.w, t.x) + sat_fma(d, t.w, t.y) + sat_fma(d, t.w, t.z);
+}
+// Codes are packed by accumulating code * 4^j into a float that starts at 2^23: its low mantissa
+// bits are then the packed field (exact while the sum stays below 2^23, i.e. up to 8 codes).
+constexpr float kPackBase = 8388608.0f;
 
 // GB: bytes per gathered granule: 16, 8, 4 or 1 (the largest that divides the packed bytes of a
 // pixel); SB: bits per stored input code (2 for k = 2, 4 for k = 3 and 4 and for the two nibbles of
@@ -446,14 +462,15 @@ __global__ void __launch_bounds__(kConvThreads, 1)
         for (int c = et; c < BN; c += 256) {
           const int nn = n0 + c;
           const bool has = nn < args.cout && args.thr;
-          // sign*A > T  <=>  sign*D > T/512 with D = A/512 (exact in fp32)
           if constexpr (SBO == 2) {
-            float4 v = make_float4(0.f, 0.f, 0.f, 1.f);
+            // (-T1, -T2, -T3, 512 s): code3f evaluates [s A > T_i] as sat(D * 512 s - T_i)
+            float4 v = make_float4(0.f, 0.f, 0.f, 512.f);
             if (has)
-              v = make_float4((float)args.thr[3 * nn] * (1.0f / 512.0f), (float)args.thr[3 * nn + 1] * (1.0f / 512.0f),
-                              (float)args.thr[3 * nn + 2] * (1.0f / 512.0f), (float)args.sign[nn]);
+              v = make_float4(-(float)args.thr[3 * nn], -(float)args.thr[3 * nn + 1], -(float)args.thr[3 * nn + 2],
+                              512.f * (float)args.sign[nn]);
             sThr[tb * BN + c] = v;
           } else {
+            // sign*A > T  <=>  sign*D > T/512 with D = A/512 (exact in fp32)
             float4* t5 = sThr + (size_t)(tb * BN + c) * 5;
             auto T = [&](int i) {
               return has && i < args.lvl ? (float)args.thr[(size_t)args.lvl * nn + i] * (1.0f / 512.0f) : INFINITY;
@@ -537,15 +554,14 @@ __global__ void __launch_bounds__(kConvThreads, 1)
             a4[j] = fmaxf(h1 ? a8[j + 4] : a8[j], __shfl_xor_sync(0xffffffffu, h1 ? a8[j] : a8[j + 4], 1));
           const int sub = (h2 ? 8 : 0) + (h1 ? 4 : 0);
           uint32_t bits = 0;
+          if constexpr (SBO == 2) {
+            float pk = kPackBase;
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            if constexpr (SBO == 2) {
-              const float4 tq = th[c0 + sub + j];
-              const float sv = a4[j] * tq.w;
-              bits |= ((uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z)) << (2 * j);
-            } else {
-              bits |= code15(a4[j], th + (c0 + sub + j) * 5) << (4 * j);
-            }
+            for (int j = 0; j < 4; ++j) pk = fmaf(code3f(a4[j], th[c0 + sub + j]), (float)(1 << (2 * j)), pk);
+            bits = __float_as_uint(pk) & 0xFFu;
+          } else {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) bits |= code15(a4[j], th + (c0 + sub + j) * 5) << (4 * j);
           }
           const int cabs = n0 + c_lo + c0 + sub;
           if (args.y_codes && m < args.M && cabs < args.cout) {
@@ -565,15 +581,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           }
         }
         if constexpr (SBO == 2) {
-          uint32_t wd = 0;
+          float lo = kPackBase, hi = kPackBase;
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float4 tq = th[c0 + j];
-            const float sv = __uint_as_float(v[j]) * tq.w;
-            const uint32_t code = (uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z);
-            wd |= code << (2 * j);
+          for (int j = 0; j < 8; ++j) {
+            lo = fmaf(code3f(__uint_as_float(v[j]), th[c0 + j]), (float)(1 << (2 * j)), lo);
+            hi = fmaf(code3f(__uint_as_float(v[j + 8]), th[c0 + j + 8]), (float)(1 << (2 * j)), hi);
           }
-          packed[c0 / 16] = wd;
+          packed[c0 / 16] = __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x5410);
         } else {
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
