@@ -234,6 +234,15 @@ __device__ __forceinline__ void tmem_st16_sync(uint32_t taddr, const uint32_t* o
       : "memory");
 }
 
+// fma(a, b, c) saturated to [0, 1] (one fma.sat on the FMA pipe).  The threshold epilogues use it
+// as an exact step function: for integers x, sat(x) = [x > 0], and a * 512 s - T with a = A / 512
+// is the integer s A - T (|s A - T| < 2^24 for every layer the tensor-core paths admit).
+__device__ __forceinline__ float sat_fma(float a, float b, float c) {
+  float r;
+  asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // 64 packed two-bit codes -> 16 registers of e4m3 bytes (register 4j+q holds byte t = code 4t + q
 // of the 16 codes in word j).
 __device__ __forceinline__ void expand2(uint4 v, uint32_t* o) {

@@ -71,12 +71,8 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
 
 // The 2-bit code of one accumulator D = A / 512 against its column's thresholds
 // t = (-T1, -T2, -T3, 512 s), as a float 0..3, on the FMA pipe: s A - T_i = fma(D, 512 s, -T_i) is
-// an exact integer (|s A - T_i| < 2^24), and saturating it to [0, 1] gives exactly [s A > T_i].
-__device__ __forceinline__ float sat_fma(float a, float b, float c) {
-  float r;
-  asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
-  return r;
-}
+// an exact integer (|s A - T_i| < 2^24), and saturating it to [0, 1] gives exactly [s A > T_i]
+// (sat_fma, conv_common.cuh).
 __device__ __forceinline__ float code3f(float d, const float4& t) {
   return sat_fma(d, t.w, t.x) + sat_fma(d, t.w, t.y) + sat_fma(d, t.w, t.z);
 }

@@ -39,12 +39,11 @@
 // (the planner admits 3 K <= 196608), so D = A_int / 512 exactly.
 //
 // Epilogue: tensor-memory lane m is one output channel of one output row, so
-// its three thresholds are per-thread constants.  A channel with a negative
-// BN scale compares against a' = (-T - 1) / 512 in ascending order and flips
-// its code (c ^ 3): sign * A > T  <=>  A < -T  <=>  not (A > -T - 1).  The
-// codes of 32 channels of one pixel are gathered with two warp ballots (bit 1
-// and the parity of the three compares) and packed into the 8 bytes those
-// channels occupy in the NHWC output.  The fused 2 x 2 pool (Sec. 2.1: on
+// its three thresholds and its sign are per-thread constants.  Each step
+// [sign * A > T_i] is an exact saturated fma of D (see sat_fma), the sign
+// folded into the multiplier.  The codes of 32 channels of one pixel are
+// gathered with two warp ballots (bit 1 and bit 0 of the code) and packed into
+// the 8 bytes those channels occupy in the NHWC output.  The fused 2 x 2 pool (Sec. 2.1: on
 // Y^conv, before BN and the quantizer) takes the max of A over the
 // horizontal pair in registers; the vertical pair is either two anchor rows
 // of the same thread (one output row per M row) or two warps (stacked output
@@ -75,6 +74,7 @@ constexpr int kWinProdBar = 1 + 2 * kWinEpiPerQ;   // producers' named barrier (
 constexpr int kWinXchgBytes = 3 * kWinEpiWarps * 2048;   // horizontal maxima of the row pairs (stacked rows, pooled)
 constexpr int kWinMaxMma = 64;         // MMAs per tile (K' / 32)
 constexpr int kWinTabBytes = 8 * kWinMaxMma;
+constexpr int kWinStashBytes = kWinEpiWarps * 32 * 8;   // per epilogue warp, 32 pairs of ballots
 constexpr int kWinMaxSmem = 232448;    // dynamic shared memory per CTA
 
 struct WinArgs {
@@ -139,16 +139,17 @@ __device__ __forceinline__ void tmem_ld2x32_sync(uint32_t t0, uint32_t t1, uint3
       : "memory");
 }
 
-// Four loads of 16 columns (at t0..t3) in flight together, one wait: 64 registers.
-__device__ __forceinline__ void tmem_ld4x16_sync(uint32_t t0, uint32_t t1, uint32_t t2, uint32_t t3, uint32_t (&v)[64]) {
+// Two loads of 16 columns (at t0 and t1) in flight together, one wait: 32 registers.
+__device__ __forceinline__ void tmem_ld2x16_sync(uint32_t t0, uint32_t t1, uint32_t (&v)[32]) {
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%64];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%65];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [%66];\n\t"
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%67];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%32];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%33];\n\t"
       "tcgen05.wait::ld.sync.aligned;"
-      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31]), "=r"(v[32]), "=r"(v[33]), "=r"(v[34]), "=r"(v[35]), "=r"(v[36]), "=r"(v[37]), "=r"(v[38]), "=r"(v[39]), "=r"(v[40]), "=r"(v[41]), "=r"(v[42]), "=r"(v[43]), "=r"(v[44]), "=r"(v[45]), "=r"(v[46]), "=r"(v[47]), "=r"(v[48]), "=r"(v[49]), "=r"(v[50]), "=r"(v[51]), "=r"(v[52]), "=r"(v[53]), "=r"(v[54]), "=r"(v[55]), "=r"(v[56]), "=r"(v[57]), "=r"(v[58]), "=r"(v[59]), "=r"(v[60]), "=r"(v[61]), "=r"(v[62]), "=r"(v[63])
-      : "r"(t0), "r"(t1), "r"(t2), "r"(t3)
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(t0), "r"(t1)
       : "memory");
 }
 
@@ -196,6 +197,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
   const uint32_t done_bar = barBase + 80u;
   const uint32_t a_full = barBase + 88u;   // the resident A operand has landed
   uint32_t* tmem_slot = (uint32_t*)(smem + oXchg + a.xchg_bytes + kWinTabBytes + 104);
+  uint2* win_stash = (uint2*)(smem + oXchg + a.xchg_bytes + kWinTabBytes + 128);   // 32 ballot pairs a warp
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // CTA c takes channel tile c % nct and the band tiles c / nct, c / nct + G / nct, ... of it
@@ -384,42 +386,41 @@ __global__ void __launch_bounds__(kWinThreads, 1)
     const int sy = (32 * q) / a.ct;              // output row offset of this quadrant
     const int cg = ((32 * q) % a.ct) >> 5;       // 32-channel group within the channel tile
     const int n = ctile * a.ct + cg * 32 + lane;
-    // thresholds in the fp32 domain of D = A / 512; negative scale: ascending (-T - 1) / 512
-    float t1 = 0.f, t2 = 0.f, t3 = 0.f;
-    bool neg = false;
+    // this lane's channel: -T1, -T2, -T3 and 512 s, so that sat_fma(D, 512 s, -T_i) = [s A > T_i]
+    // exactly (D = A / 512; the FMA pipe, not the ALU pipe the compares would take)
+    float nt1 = 0.f, nt2 = 0.f, nt3 = 0.f, s512 = 512.f;
     if (a.thr) {
-      const int32_t T0 = a.thr[3 * n], T1 = a.thr[3 * n + 1], T2 = a.thr[3 * n + 2];
-      neg = a.sign[n] < 0;
-      if (!neg) {
-        t1 = (float)T0 * (1.0f / 512.0f);
-        t2 = (float)T1 * (1.0f / 512.0f);
-        t3 = (float)T2 * (1.0f / 512.0f);
-      } else {
-        t1 = (float)(-T2 - 1) * (1.0f / 512.0f);
-        t2 = (float)(-T1 - 1) * (1.0f / 512.0f);
-        t3 = (float)(-T0 - 1) * (1.0f / 512.0f);
-      }
+      nt1 = -(float)a.thr[3 * n];
+      nt2 = -(float)a.thr[3 * n + 1];
+      nt3 = -(float)a.thr[3 * n + 2];
+      s512 = 512.f * (float)a.sign[n];
     }
-    const uint32_t negmask = __ballot_sync(0xffffffffu, neg);
+    // ballots of a column group, kept by lane 0 at [column] and read back by the column's lane
+    const uint32_t stash = smem_u32(win_stash) + (uint32_t)warp * 256u;
     const int rowb = a.cout >> 2;                                  // output bytes per pixel
     const int chb = (ctile * a.ct + cg * 32) >> 2;                 // this warp's byte within a pixel
     const uint32_t lane_off = (uint32_t)(32 * q) << 16;
     // row pairs of stacked output rows (ry > 1, pooled): the odd row's warp hands its codes over
     const int pair = a.ct == 32 ? (q >> 1) : (q & 1);
     const bool odd_row = (sy & 1) != 0;
-    // the codes of one value against the three thresholds: ballots of bit 1 and of the parity of
-    // the three compares, kept by the lane whose index is the column's within its group (a masked
-    // select, not a branch: a divergent branch per column would reconverge the warp 32 times)
-    auto code_ballot = [&](float f, int col, uint32_t& k0, uint32_t& k1) {
-      const bool p1 = f > t1, p2 = f > t2, p3 = f > t3;
-      const uint32_t m1 = __ballot_sync(0xffffffffu, p2);
-      const uint32_t m0 = __ballot_sync(0xffffffffu, p1 ^ p2 ^ p3);
-      const uint32_t pick = 0u - (uint32_t)(lane == col);
-      k0 = (m0 & pick) | (k0 & ~pick);
-      k1 = (m1 & pick) | (k1 & ~pick);
+    // The code of one value is x1 + x2 + x3 with x_i = [s A > T_i] in {0, 1}, x1 >= x2 >= x3 (the
+    // thresholds ascend): bit 1 is x2 and bit 0 is x1 - x2 + x3.  Their two warp ballots (the codes of
+    // this warp's 32 channels for one pixel) go to the stash at the column's index (lane 0 stores,
+    // one shared-memory store instead of a per-lane select), and packed() hands the column's lane its
+    // pair: the 8 bytes those channels occupy in the NHWC output.  Warp-uniform calls only.
+    auto code_ballot = [&](float f, int col, uint32_t&, uint32_t&) {
+      const float x1 = sat_fma(f, s512, nt1), x2 = sat_fma(f, s512, nt2), x3 = sat_fma(f, s512, nt3);
+      const uint32_t m1 = __ballot_sync(0xffffffffu, x2 > 0.5f);
+      const uint32_t m0 = __ballot_sync(0xffffffffu, x1 - x2 + x3 > 0.5f);
+      if (lane == 0)
+        asm volatile("st.shared.v2.u32 [%0], {%1, %2};" ::"r"(stash + 8u * (uint32_t)col), "r"(m0), "r"(m1) : "memory");
     };
-    auto packed = [&](uint32_t k0, uint32_t k1) {
-      return spread_bits(k0 ^ negmask) | (spread_bits(k1 ^ negmask) << 1);
+    auto packed = [&](uint32_t, uint32_t) {
+      __syncwarp();
+      uint32_t m0, m1;
+      asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(m0), "=r"(m1) : "r"(stash + 8u * (uint32_t)lane) : "memory");
+      __syncwarp();
+      return spread_bits(m0) | (spread_bits(m1) << 1);
     };
     bool ok = true;
 #pragma unroll 1
@@ -453,8 +454,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int j = 32 * g + lane;
             const int r = (int)fdiv((uint32_t)j, a.div_pitch), xx = j - r * a.pitch;
             const int yy = win_row(a, y0, r) + sy;
+            const uint64_t pk = packed(k0, k1);
             if (a.y_codes && r < a.R && xx < a.w && yy < a.h)
-              *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = packed(k0, k1);
+              *(uint64_t*)(a.y_codes + (((size_t)b * a.h + yy) * a.w + xx) * rowb + chb) = pk;
           }
         }
       } else {
@@ -513,8 +515,9 @@ __global__ void __launch_bounds__(kWinThreads, 1)
               const int pi = 32 * g + kKept + lane;
               const int r = (int)fdiv((uint32_t)(2 * pi), a.div_pitch), xx = 2 * pi - r * a.pitch;
               const int py = (win_row(a, y0, r) + sy) >> 1, px = xx >> 1;
+              const uint64_t pk = packed(k0, k1);
               if (a.y_codes && lane < 16 && pi < npool && r < a.R && px < pw && py < ph)
-                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = packed(k0, k1);
+                *(uint64_t*)(a.y_codes + (((size_t)b * ph + py) * pw + px) * rowb + chb) = pk;
             }
           };
           if (odd_row) half(std::integral_constant<int, 16>{});
@@ -541,18 +544,17 @@ __global__ void __launch_bounds__(kWinThreads, 1)
                     const int pr = pi0 / halfw, px0 = pi0 - pr * halfw;
                     col[u] = pi0 < npool ? (uint32_t)(2 * pr * a.pitch + 2 * px0) : 0u;
                   }
-                  uint32_t v[64];
-                  tmem_ld4x16_sync(tacc + col[0], tacc + col[0] + (uint32_t)a.pitch, tacc + col[1],
-                                   tacc + col[1] + (uint32_t)a.pitch, v);
 #pragma unroll
-                  for (int u = 0; u < 2; ++u)
+                  for (int u = 0; u < 2; ++u) {
+                    uint32_t v[32];   // 16 columns of the top row, then of the bottom row
+                    tmem_ld2x16_sync(tacc + col[u], tacc + col[u] + (uint32_t)a.pitch, v);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                      const float top = fmaxf(__uint_as_float(v[32 * u + 2 * e]), __uint_as_float(v[32 * u + 2 * e + 1]));
-                      const float bot =
-                          fmaxf(__uint_as_float(v[32 * u + 16 + 2 * e]), __uint_as_float(v[32 * u + 16 + 2 * e + 1]));
+                      const float top = fmaxf(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                      const float bot = fmaxf(__uint_as_float(v[16 + 2 * e]), __uint_as_float(v[16 + 2 * e + 1]));
                       code_ballot(fmaxf(top, bot), 16 * hh + 8 * u + e, k0, k1);
                     }
+                  }
                 }
               }
               own[gi] = packed(k0, k1);

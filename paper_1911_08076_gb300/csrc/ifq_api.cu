@@ -437,7 +437,8 @@ bool win_plan(const ifq_conv_desc* d, const ConvGeom& g, int nsm, WinArgs* wa, s
     const uint32_t ps_ = (uint32_t)round_up((size_t)slots * 16, 128) + (planes > 1 ? 16u : 0u);
     const uint32_t bb = (uint32_t)round_up((size_t)planes * ps_, 1024);
     const uint32_t sb = (uint32_t)round_up((size_t)ns * rbr * row_bytes, 128);
-    const size_t nd = 1024 + (size_t)a_bytes + 2 * (size_t)bb + 2 * (size_t)sb + xchg + kWinTabBytes + 128;
+    const size_t nd = 1024 + (size_t)a_bytes + 2 * (size_t)bb + 2 * (size_t)sb + xchg + kWinTabBytes + 128 +
+                      kWinStashBytes;
     if (nd <= (size_t)kWinMaxSmem) {
       R = r; seg_pitch = sp; rb = rbr; N = n_; nseg = ns; ps = ps_; band_bytes = bb; stage_bytes = sb; need = nd;
       break;
@@ -478,7 +479,7 @@ bool win_supported(const ifq_conv_desc* d, const ConvGeom& g) {
 
 // Where the window kernel is the default (measured on GB300 against the tensor-core kernel, layer
 // by layer in the benchmark stacks): layers with a fused 2 x 2 pool and at most 64 input
-// channels.  Tiny-YOLO conv2 (16 -> 32 at 208 x 208, b64) 58 vs 128 us, conv3 34 vs 51, conv4 21 vs
+// channels.  Tiny-YOLO conv2 (16 -> 32 at 208 x 208, b64) 54 vs 128 us, conv3 34 vs 51, conv4 21 vs
 // 28; IFQ-Tinier-YOLO conv3..conv5 24 / 17 / 14 vs 38 / 21 / 16 us.  Without a pool its epilogue
 // thresholds twice the columns, and with 128 or more input channels its resident filter block and
 // per-tile setup cost more than the other kernel's gather: there the tensor-core kernel stays ahead
@@ -548,7 +549,7 @@ bool warp_supported(const ifq_conv_desc* d, const ConvGeom& g) {
 // fused pool, 62 vs 107 us without) and 8-bit-input layers without a fused pool (3 x 3 4 -> 8 at
 // 416 x 416: 144 vs 207 us on the direct kernel).  Elsewhere it loses: one e4m3 mma.sync issues about
 // four instructions on this GPU, and the tcgen05 window kernel (16-channel layers: Tiny-YOLO conv2
-// 58 vs 124 us) or the direct kernel (the pooled first layer: 91 vs 107 us) stays ahead.
+// 54 vs 124 us) or the direct kernel (the pooled first layer: 91 vs 107 us) stays ahead.
 bool warp_wins(const ifq_conv_desc* d, const ConvGeom& g) {
   return warp_supported(d, g) && (g.in8 ? g.pool == 1 : d->cin == 8);
 }
