@@ -243,14 +243,36 @@ __device__ __forceinline__ float sat_fma(float a, float b, float c) {
   return r;
 }
 
-// 64 packed two-bit codes -> 16 registers of e4m3 bytes (register 4j+q holds byte t = code 4t + q
-// of the 16 codes in word j).
+// 16 packed two-bit codes (one word) -> 4 registers of e4m3 bytes: register q holds, in byte t,
+// code 4t + q.  Registers with q odd keep the code where it sits, in bits 2..3 of the byte: the
+// e4m3 byte 4c, the value 4c * 2^-9 (e4m3 bytes 0..15 are the values 0..15 times 2^-9).  Their
+// filter bytes are +-0.25 instead of +-1 (prep_weights_kernel), so every product is still c * 2^-9
+// exactly, and one shift by 4 serves all four registers: five ALU instructions per word instead of
+// seven.
+__device__ __forceinline__ void expand2w(uint32_t w, uint32_t* o) {
+  const uint32_t h = w >> 4;
+  o[0] = w & 0x03030303u;
+  o[1] = w & 0x0C0C0C0Cu;
+  o[2] = h & 0x03030303u;
+  o[3] = h & 0x0C0C0C0Cu;
+}
+
+// 64 packed two-bit codes -> 16 registers (register 4j+q from word j, as expand2w).
 __device__ __forceinline__ void expand2(uint4 v, uint32_t* o) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-  for (int j = 0; j < 4; ++j)
-#pragma unroll
-    for (int q = 0; q < 4; ++q) o[4 * j + q] = (w[j] >> (2 * q)) & 0x03030303u;
+  expand2w(v.x, o);
+  expand2w(v.y, o + 4);
+  expand2w(v.z, o + 8);
+  expand2w(v.w, o + 12);
+}
+
+// 8 registers -> 8 consecutive tensor-memory columns of this warp's 32 lanes, with the wait for the
+// store in the same asm statement (the store reads its source registers asynchronously).
+__device__ __forceinline__ void tmem_st8_sync(uint32_t taddr, const uint32_t* o) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};\n\t"
+      "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+      "r"(o[0]), "r"(o[1]), "r"(o[2]), "r"(o[3]), "r"(o[4]), "r"(o[5]), "r"(o[6]), "r"(o[7])
+      : "memory");
 }
 
 // 64 four-bit codes (two 16-byte units, 8 words) -> 16 registers of e4m3 bytes: word j of the 8

@@ -10,7 +10,8 @@
 // integer MMA):
 //   * A: code c in 0..15 is the e4m3 byte c, i.e. the value c * 2^-9
 //     (subnormal below 8); the k-bit -> 8-bit expansion is a mask per byte lane.
-//   * B: +1 / -1 are the e4m3 bytes 0x38 / 0xB8 (+-1.0).
+//   * B: +1 / -1 are the e4m3 bytes 0x38 / 0xB8 (+-1.0), or 0x28 / 0xA8 (+-0.25)
+//     at the K positions where the 2-bit expansion leaves a code as 4c.
 //   * Every product is c * 2^-9 exactly; every partial sum is an integer
 //     multiple of 2^-9 of magnitude <= (2^k - 1) K * 2^-9, far inside the
 //     24-bit fp32 significand for the magnitudes the host admits, so the fp32
@@ -22,7 +23,9 @@
 // K ordering inside each chunk of one 32-bit word of packed codes (16 two-bit
 // or 8 four-bit codes): the expansion produces byte p = 4q + t from code
 // (cpw/4) t + q, cpw = codes per word (a transpose).  The prepared filter rows
-// use the same order, so the dot product over K is unchanged.
+// use the same order, so the dot product over K is unchanged.  For 2-bit
+// codes the odd registers q of a word hold 4c (a mask without a shift), and
+// the filter bytes at those K positions are +-0.25: the product is c * 2^-9.
 //
 // Data path.  The expanded A operand never touches shared memory: gather
 // threads load packed codes from global memory into registers several K
@@ -254,13 +257,23 @@ __global__ void __launch_bounds__(kConvThreads, 1)
           const uint32_t ph = (uint32_t)(it / kS) & 1u;
           if (!__all_sync(0xffffffffu, mbar_wait_backoff(empty(s), ph ^ 1u, 64))) { ok = false; break; }
           tc_fence_after();
-          uint32_t o[16];
-          if constexpr (SB == 2) expand2(cur[0], o);
-          else expand4(cur[0], cur[1], o);
-          tmem_st16_sync(tA + (uint32_t)(s * 32), o);
-          if constexpr (SB == 2) expand2(cur[kU - 1], o);
-          else expand4(cur[kU - 2], cur[kU - 1], o);
-          tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
+          if constexpr (SB == 2) {
+            // 8 columns (two packed words) at a time: fewer live registers than 16
+#pragma unroll
+            for (int hq = 0; hq < 4; ++hq) {
+              const uint4 u = cur[hq >> 1];
+              uint32_t o8[8];
+              expand2w((hq & 1) ? u.z : u.x, o8);
+              expand2w((hq & 1) ? u.w : u.y, o8 + 4);
+              tmem_st8_sync(tA + (uint32_t)(s * 32 + 8 * hq), o8);
+            }
+          } else {
+            uint32_t o[16];
+            expand4(cur[0], cur[1], o);
+            tmem_st16_sync(tA + (uint32_t)(s * 32), o);
+            expand4(cur[kU - 2], cur[kU - 1], o);
+            tmem_st16_sync(tA + (uint32_t)(s * 32 + 16), o);
+          }
           if constexpr (BX != 0) {
             // this K stage's filter tile from sign bits (loaded with the codes, kAh stages ahead):
             // 16-bit chunks -> 16 e4m3 bytes (+1 = 0x38, -1 = 0xB8) at row bx_r, chunk c of the
@@ -289,8 +302,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
               uint32_t w4[4];
 #pragma unroll
               for (int nb = 0; nb < 4; ++nb) {
+                // word nb of the chunk: +-1 (0x38 / 0xB8), or +-0.25 (0x28 / 0xA8) for the odd
+                // words, whose gathered codes are 4c (expand2)
                 const uint32_t x = (((bits16 >> (4 * nb)) & 0xFu) * 0x00204081u) & 0x01010101u;
-                w4[nb] = 0xB8B8B8B8u - (x << 7);
+                w4[nb] = ((nb & 1) ? 0xA8A8A8A8u : 0xB8B8B8B8u) - (x << 7);
               }
               const uint32_t dst = rowb + (uint32_t)((((c0 + cc) ^ (rr & 7)) & 7) << 4);
               asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(w4[0]), "r"(w4[1]), "r"(w4[2]),

@@ -319,7 +319,7 @@ __global__ void __launch_bounds__(kWinThreads, 1)
             const int pl = qw - xx * a.planes;                      // and plane
             const uint32_t v = ws[e];
             *(uint4*)(smem + rowo + (uint32_t)pl * a.plane_stride + 16u * (uint32_t)xx) =
-                make_uint4(v & 0x03030303u, (v >> 2) & 0x03030303u, (v >> 4) & 0x03030303u, (v >> 6) & 0x03030303u);
+                make_uint4(v & 0x03030303u, v & 0x0C0C0C0Cu, (v >> 4) & 0x03030303u, (v >> 4) & 0x0C0C0C0Cu);
           }
         }
         fence_proxy_async_smem();

@@ -310,6 +310,9 @@ __global__ void pack_signs_kernel(const int8_t* w, uint32_t* bits, int rows, int
 // tensor-core A expansion: with cpw codes per packed word (16 for 2-bit, 8 for
 // 4-bit fields), byte p of chunk j holds k = cpw*j + (cpw/4)*(p%4) + p/4;
 // +1 -> 0x38, -1 -> 0xB8, k >= K -> 0; followed by a copy of the sign words.
+// 2-bit fields: the bytes of the odd 4-byte words of a chunk (p/4 odd) hold
+// +-0.25 (0x28 / 0xA8) instead, because the expansion leaves those codes as 4c
+// (the e4m3 value 4c * 2^-9); each product is c * 2^-9 either way.
 // in8: the input is 8-bit values read as two 4-bit fields, so kernel position k
 // is filter position k/2 times 1 (low nibble, k even) or 16 (high nibble):
 // +-16 are the e4m3 bytes 0x58 / 0xD8.  K is the kernel's K (twice the filter's).
@@ -330,7 +333,10 @@ __global__ void prep_weights_kernel(const uint32_t* bits, uint8_t* e4m3, uint32_
         const int kf = in8 ? (k >> 1) : k;                       // filter position
         const bool hi = in8 && (k & 1);
         const bool pos = (bits[(size_t)n * kwords + (kf >> 5)] >> (kf & 31)) & 1u;
-        byte = pos ? (hi ? 0x58u : 0x38u) : (hi ? 0xD8u : 0xB8u);
+        // 2-bit fields: the odd words of a chunk (p / 4 odd) carry the codes as 4c (expand2), so
+        // their weights are +-0.25 (0x28 / 0xA8)
+        const bool quarter = cpw == 16 && ((p >> 2) & 1);
+        byte = pos ? (hi ? 0x58u : (quarter ? 0x28u : 0x38u)) : (hi ? 0xD8u : (quarter ? 0xA8u : 0xB8u));
       }
       out |= byte << (8 * t);
     }
