@@ -90,11 +90,18 @@ struct TcSmem {
 
 // The input row (output pixel) that a gather thread reads in one tile: a base
 // pointer for tap (0,0) (possibly outside the image; dereferenced only when
-// valid) and bitmasks of the taps dy / dx that fall inside the image.
+// valid) and the taps that fall inside the image: bit dy of vyx for the filter
+// rows, bit 16 + dx for the filter columns (kh, kw <= 15, so bits 15 and 31
+// are never set).
 struct RowGeom {
   const uint8_t* base;
-  uint32_t vy, vx;
+  uint32_t vyx;
 };
+
+// A K-granule's tap as a mask for tap_ok: bit dy and bit 16 + dx; past K, all ones (never inside,
+// because bits 15 and 31 of a row's mask are clear).
+__host__ __device__ constexpr int tap_mask(int dy, int dx) { return (int)((1u << dy) | (1u << (16 + dx))); }
+constexpr int kTapNone = -1;
 
 // bits lo..hi-1 of a tap mask (empty when hi <= lo); hi - lo <= 32
 __device__ __forceinline__ uint32_t bit_range(int lo, int hi) {
@@ -104,7 +111,7 @@ __device__ __forceinline__ uint32_t bit_range(int lo, int hi) {
 __device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
   RowGeom g;
   g.base = a.x;
-  g.vy = g.vx = 0;
+  g.vyx = 0;
   if (m < a.M) {
     int b, oy, ox;
     if (a.lpool == 0) {
@@ -123,16 +130,14 @@ __device__ __forceinline__ RowGeom row_geom(const ConvArgs& a, int m) {
     }
     const int iy0 = oy * a.stride - a.pad, ix0 = ox * a.stride - a.pad;
     g.base = a.x + ((long long)b * a.h * a.w + (long long)iy0 * a.w + ix0) * a.cinb;
-    g.vy = bit_range(max(0, -iy0), min(a.kh, a.h - iy0));
-    g.vx = bit_range(max(0, -ix0), min(a.kw, a.w - ix0));
+    g.vyx = bit_range(max(0, -iy0), min(a.kh, a.h - iy0)) | (bit_range(max(0, -ix0), min(a.kw, a.w - ix0)) << 16);
   }
   return g;
 }
 
-__device__ __forceinline__ bool tap_ok(const RowGeom& g, int2 e) {
-  const int dy = e.y >> 8, dx = e.y & 0xFF;
-  return dy != 0xFF && ((g.vy >> dy) & (g.vx >> dx) & 1u);
-}
+// Whether a granule's tap (e.y = tap_mask(dy, dx), or kTapNone past K) lies inside the image for
+// this row: both its row bit and its column bit are set.
+__device__ __forceinline__ bool tap_ok(const RowGeom& g, int2 e) { return (g.vyx & (uint32_t)e.y) == (uint32_t)e.y; }
 
 // Loads of packed codes.  COHERENT = false: the codes were written by an earlier kernel and
 // stay read-only for this one, so they may take the non-coherent read-only path (ld.global.nc).

@@ -178,16 +178,16 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   }
   if (warp == kWarpTma && lane == 0) prefetch_tmap(&tmap_w);
   // K-granule table: byte offset of each granule from the row's tap-(0,0)
-  // pointer, and its tap (dy, dx); dy = 0xFF past K.
+  // pointer, and its tap as tap_mask(dy, dx); kTapNone past K.
   {
     const int cinb = args.cinb;
     for (int gk = tid; gk < args.ntab; gk += kConvThreads) {
       const int k0 = gk * kCpb * GB;
       const int tap = k0 / args.cin, cc = k0 - tap * args.cin;
-      int2 e = make_int2(0, 0xFF << 8);
+      int2 e = make_int2(0, kTapNone);
       if (tap < args.kh * args.kw) {
         const int dy = tap / args.kw, dx = tap - dy * args.kw;
-        e = make_int2((dy * args.w + dx) * cinb + cc / kCpb, (dy << 8) | dx);
+        e = make_int2((dy * args.w + dx) * cinb + cc / kCpb, tap_mask(dy, dx));
       }
       sTab[gk] = e;
     }
@@ -219,7 +219,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     RowGeom g = row_geom(args, l_tile < n_local ? (int)fdiv((uint32_t)(cid + l_tile * G), args.div_nt) * kBM + r
                                                 : args.M);
     // packed codes of kAh of this group's stages in registers (16 registers either way)
-    constexpr int kAh = SB == 2 ? kAhead : 1;
+    // (1-byte granules, 16 loads a unit: one stage ahead, within the register cap)
+    constexpr int kAh = SB == 2 && GB > 1 ? kAhead : 1;
     // BX: this thread's share of a stage's filter tile: row bx_r of the channel tile, 16-bit chunks
     // bx_c0 .. bx_c0 + BN / 16 - 1 of the stage's 128 sign bits
     constexpr int kCpt = BN / 16;

@@ -692,11 +692,11 @@ int granule_bytes(const ifq_conv_desc* d, const ConvGeom& g, bool stack = false)
 }
 
 // Whether the tensor-core kernel supports this shape: an accumulator magnitude inside the
-// checked exact range, taps addressable by 32-bit masks, a K-granule table that fits, and an
+// checked exact range, filter rows and columns addressable by 15-bit masks (kh, kw <= 15), a K-granule table that fits, and an
 // instantiated granule (4-bit fields need 4-byte granules, cin % 8 == 0).
 bool tc_supported(const ifq_conv_desc* d, const ConvGeom& g) {
   const long long amax = (long long)(g.in8 ? 255 : g.lvl) * g.K;   // largest |A|
-  if (amax > kTcMaxAcc || d->kh > 32 || d->kw > 32) return false;
+  if (amax > kTcMaxAcc || d->kh > 15 || d->kw > 15) return false;
   const int gb = granule_bytes(d, g, true);   // the smaller granule of the two kernels: the larger table
   if (g.sbi == 4 && gb == 1) return false;
   if ((long long)g.Kpad * g.sbi / 8 / gb > kMaxTab) return false;

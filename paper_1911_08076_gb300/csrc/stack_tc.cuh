@@ -341,10 +341,10 @@ __global__ void __launch_bounds__(kStackThreads, 1) conv_stack_kernel(const __gr
     for (int gk = tid; gk < a.ntab; gk += kStackThreads) {
       const int k0 = gk * gran;
       const int tap = k0 / a.cin, cc = k0 - tap * a.cin;
-      int2 e = make_int2(0, 0xFF << 8);
+      int2 e = make_int2(0, kTapNone);
       if (tap < a.kh * a.kw) {
         const int dy = tap / a.kw, dx = tap - dy * a.kw;
-        e = make_int2((dy * a.w + dx) * cinb + (cc >> 2), (dy << 8) | dx);
+        e = make_int2((dy * a.w + dx) * cinb + (cc >> 2), tap_mask(dy, dx));
       }
       sTab[P.L[l].tab_off + gk] = e;
     }
