@@ -239,15 +239,18 @@ __device__ __forceinline__ void stack_epi_tile(const ConvArgs& a, uint32_t tacc,
   for (int c0 = 0; c0 < CW; c0 += 16) {
     uint32_t v[16];
     tmem_ld16_sync(tacc + c0, v);
-    uint32_t wd = 0;
+    // the code of D = A / 512 against th = (-T1, -T2, -T3, 512 s): [s A > T_i] = sat(D 512 s - T_i)
+    // (exact integers, sat_fma), summed and packed by accumulating code * 4^j into a float based at
+    // 2^23 (8 codes a float), on the FMA pipe
+    float lo = 8388608.0f, hi = 8388608.0f;
 #pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const float4 tq = th[c0 + j];
-      const float sv = __uint_as_float(v[j]) * tq.w;
-      const uint32_t code = (uint32_t)(sv > tq.x) + (uint32_t)(sv > tq.y) + (uint32_t)(sv > tq.z);
-      wd |= code << (2 * j);
+    for (int j = 0; j < 8; ++j) {
+      const float4 ta = th[c0 + j], tb = th[c0 + j + 8];
+      const float da = __uint_as_float(v[j]), db = __uint_as_float(v[j + 8]);
+      lo = fmaf(sat_fma(da, ta.w, ta.x) + sat_fma(da, ta.w, ta.y) + sat_fma(da, ta.w, ta.z), (float)(1 << (2 * j)), lo);
+      hi = fmaf(sat_fma(db, tb.w, tb.x) + sat_fma(db, tb.w, tb.y) + sat_fma(db, tb.w, tb.z), (float)(1 << (2 * j)), hi);
     }
-    packed[c0 / 16] = wd;
+    packed[c0 / 16] = __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x5410);
     if (a.y_acc && m < a.M) {
       const int cbase = cb + c0;
       int32_t* dst = a.y_acc + (size_t)m * a.cout + cbase;
@@ -535,11 +538,10 @@ __global__ void __launch_bounds__(kStackThreads, 1) conv_stack_kernel(const __gr
           thr_n0 = n0;
           for (int cc = et; cc < bn; cc += 256) {
             const int nn = n0 + cc;
-            float4 v = make_float4(0.f, 0.f, 0.f, 1.f);
+            float4 v = make_float4(0.f, 0.f, 0.f, 512.f);
             if (nn < a.cout && a.thr)
-              v = make_float4((float)__ldg(a.thr + 3 * nn) * (1.0f / 512.0f),
-                              (float)__ldg(a.thr + 3 * nn + 1) * (1.0f / 512.0f),
-                              (float)__ldg(a.thr + 3 * nn + 2) * (1.0f / 512.0f), (float)__ldg(a.sign + nn));
+              v = make_float4(-(float)__ldg(a.thr + 3 * nn), -(float)__ldg(a.thr + 3 * nn + 1),
+                              -(float)__ldg(a.thr + 3 * nn + 2), 512.f * (float)__ldg(a.sign + nn));
             sThr[tb * kStackBN + cc] = v;
           }
           named_bar(1, kEpiWarps * 32);
