@@ -144,6 +144,7 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
   __shared__ __align__(16) uint32_t sW[TAPS * NC];   // [tap][n] +-1 byte words
   __shared__ int32_t sT[NC * 15];
   __shared__ int32_t sS[NC];
+  __shared__ int4 sT3[NC];                            // lvl = 3: {T1, T2, T3, sign} per channel
   grid_dep_launch();
   grid_dep_wait();
   for (int i = threadIdx.x; i < TAPS * NC; i += blockDim.x) {
@@ -157,6 +158,9 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
     for (int i = threadIdx.x; i < a.cout * a.lvl; i += blockDim.x) sT[i] = a.thr[i];
   if (a.sign)
     for (int i = threadIdx.x; i < a.cout; i += blockDim.x) sS[i] = a.sign[i];
+  if (a.thr && a.sign && a.lvl == 3)
+    for (int i = threadIdx.x; i < a.cout; i += blockDim.x)
+      sT3[i] = make_int4(a.thr[3 * i], a.thr[3 * i + 1], a.thr[3 * i + 2], a.sign[i]);
   __syncthreads();
   const uint32_t* x32 = (const uint32_t*)a.x;
   for (int it = blockIdx.x * blockDim.x + threadIdx.x; it < a.total; it += gridDim.x * blockDim.x) {
@@ -166,14 +170,23 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
     const int py = t - b * a.pho;
     const int iy0 = py * P - a.pad, ix0 = px * P - a.pad;
     uint32_t win[WIN * WIN];
+    if (iy0 >= 0 && ix0 >= 0 && iy0 + WIN <= a.h && ix0 + WIN <= a.w) {
+      // the whole window inside the image (all but the border pixels): one address, no checks
+      const uint32_t* p0 = x32 + ((size_t)b * a.h + iy0) * a.w + ix0;
 #pragma unroll
-    for (int wy = 0; wy < WIN; ++wy)
+      for (int wy = 0; wy < WIN; ++wy)
 #pragma unroll
-      for (int wx = 0; wx < WIN; ++wx) {
-        const int iy = iy0 + wy, ix = ix0 + wx;
-        const bool in = (unsigned)iy < (unsigned)a.h && (unsigned)ix < (unsigned)a.w;   // else zero padding
-        win[wy * WIN + wx] = in ? __ldg(x32 + ((size_t)b * a.h + iy) * a.w + ix) : 0u;
-      }
+        for (int wx = 0; wx < WIN; ++wx) win[wy * WIN + wx] = __ldg(p0 + (size_t)wy * a.w + wx);
+    } else {
+#pragma unroll
+      for (int wy = 0; wy < WIN; ++wy)
+#pragma unroll
+        for (int wx = 0; wx < WIN; ++wx) {
+          const int iy = iy0 + wy, ix = ix0 + wx;
+          const bool in = (unsigned)iy < (unsigned)a.h && (unsigned)ix < (unsigned)a.w;   // else zero padding
+          win[wy * WIN + wx] = in ? __ldg(x32 + ((size_t)b * a.h + iy) * a.w + ix) : 0u;
+        }
+    }
     int acc[P * P][NC];
 #pragma unroll
     for (int q = 0; q < P * P; ++q)
@@ -205,7 +218,24 @@ __global__ void __launch_bounds__(kDirectThreads) conv_direct_rgb3_kernel(const 
       for (int n = 0; n < NC; ++n)
         if (n < a.cout) dst[n] = amax[n];
     }
-    if (a.y_codes) {
+    if (a.y_codes && a.lvl == 3 && a.sbo == 2 && (a.cout & 3) == 0) {
+      // 2-bit codes: thresholds and sign of a channel in one 16-byte load, the codes of 4 channels
+      // a byte
+      uint8_t* dst = a.y_codes + (size_t)it * (a.cout >> 2);
+#pragma unroll
+      for (int n4 = 0; n4 < NC; n4 += 4) {
+        if (n4 < a.cout) {
+          uint32_t byte = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const int4 t = sT3[n4 + q];
+            const int sv = t.w * amax[n4 + q];
+            byte |= ((uint32_t)(sv > t.x) + (uint32_t)(sv > t.y) + (uint32_t)(sv > t.z)) << (2 * q);
+          }
+          dst[n4 >> 2] = (uint8_t)byte;
+        }
+      }
+    } else if (a.y_codes) {
       uint8_t* dst = a.y_codes + (size_t)it * (a.cout * a.sbo / 8);
       uint32_t byte = 0;
       int nbits = 0, bi = 0;
