@@ -79,6 +79,21 @@ __device__ __forceinline__ uint32_t code15(float d, const float4* t5) {
 __device__ __forceinline__ float code3f(float d, const float4& t) {
   return sat_fma(d, t.w, t.x) + sat_fma(d, t.w, t.y) + sat_fma(d, t.w, t.z);
 }
+// 32 lanes x 32 consecutive columns of tensor memory -> 32 registers, the wait in the same asm
+// statement.
+__device__ __forceinline__ void tc_ld32_sync(uint32_t t0, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,"
+      "%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]), "=r"(v[8]),
+        "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]),
+        "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+        "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(t0)
+      : "memory");
+}
+
 // Codes are packed by accumulating code * 4^j into a float that starts at 2^23: its low mantissa
 // bits are then the packed field (exact while the sum stays below 2^23, i.e. up to 8 codes).
 constexpr float kPackBase = 8388608.0f;
@@ -529,8 +544,35 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       const float4* th = sThr + (size_t)(tb * BN + c_lo) * (SBO == 2 ? 1 : 5);
       constexpr int kPW = CW * SBO / 32;          // 32-bit words of packed codes per thread
       uint32_t packed[kPW];
+      // Plain 2-bit codes (no pool, no accumulators out, no K split): 32 columns per tensor-memory
+      // load and wait, twice the independent work between waits (the 1x1 512 -> 512 layer 107.3 ->
+      // 97.6 us).  Instances with 8- and 1-byte granules keep 16 columns: their gather leaves no
+      // registers for it.
+      constexpr bool kWide32 = (GB == 16 || GB == 4) && SB == 2 && SBO == 2 && KS == 1 && CW % 32 == 0;
+      const bool wide32 = kWide32 && args.lpool == 0 && !args.y_acc;
+      if constexpr (kWide32) {
+        if (wide32) {
 #pragma unroll
-      for (int c0 = 0; c0 < CW; c0 += 16) {
+          for (int c0 = 0; c0 < CW; c0 += 32) {
+            uint32_t v[32];
+            tc_ld32_sync(tacc + c0, v);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              float lo = kPackBase, hi = kPackBase;
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                lo = fmaf(code3f(__uint_as_float(v[16 * h + j]), th[c0 + 16 * h + j]), (float)(1 << (2 * j)), lo);
+                hi = fmaf(code3f(__uint_as_float(v[16 * h + j + 8]), th[c0 + 16 * h + j + 8]), (float)(1 << (2 * j)), hi);
+              }
+              packed[c0 / 16 + h] = __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x5410);
+              // the second half's thresholds are not loaded before the first half is done (registers)
+              asm volatile("" ::: "memory");
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int c0 = 0; c0 < CW && !wide32; c0 += 16) {
         uint32_t v[16];
         tmem_ld16_sync(tacc + c0, v);
         if constexpr (KS > 1) {   // + the partners' partial sums of these 16 columns
