@@ -244,7 +244,7 @@ int ifq_pack_weights(const ifq_conv_desc* d, const uint32_t* w_bits, void* w_pre
  * measured faster), and a request for it elsewhere takes the tensor-core
  * path.  The
  * tensor-core path needs (2^k - 1)*K <= 196608 (the accumulator range checked
- * exact on the fp8 tensor cores; 255*K for 8-bit inputs), kh, kw <= 32, and
+ * exact on the fp8 tensor cores; 255*K for 8-bit inputs), kh, kw <= 15, and
  * for k = 3, 4 cin % 8 == 0; a request for it outside that range takes the
  * bit-serial path.  The direct CUDA-core path serves layers on 8-bit inputs
  * with cout <= 32 and K <= 257 (the default for them); a request for it

@@ -279,6 +279,16 @@ def test_last_forward_mode_before_any_forward_is_einval():
     assert out.get("status") == ifq.IFQ_EINVAL
 
 
+def test_tensor_core_path_filter_size_limit():
+    """The tensor-core paths take filters of up to 15 x 15 (a row's valid filter rows and columns sit
+    in one 32-bit mask, 15 bits each, so a granule's tap test is one AND and one compare); larger
+    filters take the bit-serial path."""
+    plan = lambda *a, **k: ifq.ifq_conv_plan(ifq.conv_desc(*a, **k))
+    assert plan(1, 24, 24, 64, 64, 15, 1, 7) == ifq.IFQ_PATH_TC
+    assert plan(1, 24, 24, 64, 64, 17, 1, 8) == ifq.IFQ_PATH_BITSERIAL
+    assert plan(1, 24, 24, 64, 64, 17, 1, 8, path=ifq.IFQ_PATH_TC) == ifq.IFQ_PATH_BITSERIAL
+
+
 def test_window_path_plan():
     """The window path applies to stride-1 k x k 'same' layers on 2-bit codes with cin 16 or a
     multiple of 32, cout 32, 64 or a multiple of 128, whose resident filter block and buffers fit
