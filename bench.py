@@ -57,7 +57,7 @@ SUB_WORKLOADS = ["pr1", "resnet18", "alexnet", "tinyyolo_fused", "tinieryolo_fus
 FP8_PER_BF16 = 2.0          # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
 FALLBACK_BF16_TFLOPS = 1900.0
 PROFILES = os.path.join(ROOT, "profiles")
-KERNEL_SRC = [os.path.join(ROOT, "paper_1911_08076_gb300", "csrc", f) for f in ("conv_tc.cuh", "conv_common.cuh", "ptx.cuh")]
+KERNEL_DIR = os.path.join(ROOT, "paper_1911_08076_gb300", "csrc")
 RATES_SRC = os.path.join(ROOT, "bench_rates.cu")
 RATES_LIB = os.path.join(ROOT, "_build", "libbench_rates.so")
 
@@ -114,9 +114,11 @@ def read_peaks():
 
 
 def kernel_sha():
-    """Hash of the sources the conv kernel compiles from (a stale ncu summary must not be reused)."""
+    """Hash of every CUDA source of the library (all .cu and .cuh files), so that a change to any
+    kernel a workload launches marks its ncu summary stale and its traffic is not reused."""
     h = hashlib.sha256()
-    for path in KERNEL_SRC:
+    for path in sorted(glob.glob(os.path.join(KERNEL_DIR, "*.cu")) + glob.glob(os.path.join(KERNEL_DIR, "*.cuh"))):
+        h.update(os.path.basename(path).encode())
         with open(path, "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
