@@ -64,7 +64,7 @@ typedef enum {
   IFQ_ERANGE = 4,        /* a size exceeds what the library supports */
   IFQ_ECUDA = 5,         /* a CUDA runtime call failed */
   IFQ_ETIMEOUT = 6,      /* (device status) a bounded wait in a kernel ran out */
-  IFQ_EUNSUPPORTED = 7,  /* valid request that this build does not implement */
+  IFQ_EUNSUPPORTED = 7,  /* valid request that the library does not implement */
   IFQ_EWORKSPACE = 8     /* workspace missing or too small */
 } ifq_status;
 
